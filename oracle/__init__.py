@@ -1,0 +1,228 @@
+"""CPU oracle for the FASGD parameter-server path -- TEST INFRASTRUCTURE ONLY.
+
+Only the tests, ``__graft_entry__.smoke()`` and the CPU-baseline / reference
+legs of ``bench.py`` may import this package.  The CUDA path never does and
+shares no code with it.
+
+``fasgd_oracle.c`` holds the elementwise rules (Eq. 1-2, 4-8, 9 of the
+paper); this module compiles it twice (fp32 and fp64 parameter/state type)
+and adds the server protocol of Section 2.1 around it as a plain Python
+FIFO: a push carries (client, timestamp j, gradient); applying it computes
+the step-staleness tau = T - j against the current server timestamp T,
+updates every parameter, and increments T.
+
+Parity status: every function here is pinned by the ``-m "not gpu"`` tests
+(closed forms, hand traces, series brute force, exact-rational checks of the
+send decision, Philox known-answer vectors, invariants between variants).
+"""
+
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+import threading
+
+import numpy as np
+
+ASGD, SASGD, FASGD = 0, 1, 2
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "fasgd_oracle.c")
+_BUILD = os.path.join(_HERE, "_build")
+_LOCK = threading.Lock()
+_LIBS: dict = {}
+
+_CFLAGS = ["-O2", "-std=c11", "-fPIC", "-shared", "-ffp-contract=off",
+           "-fno-fast-math", "-Wall", "-Wextra"]
+
+
+def lib_path(real: str) -> str:
+    return os.path.join(_BUILD, f"libfasgd_oracle_{real}.so")
+
+
+def build(force: bool = False) -> None:
+    """Compile the oracle (fp32 and fp64 builds) with gcc if out of date."""
+    os.makedirs(_BUILD, exist_ok=True)
+    for real, ctype in (("f32", "float"), ("f64", "double")):
+        out = lib_path(real)
+        if (not force and os.path.exists(out)
+                and os.path.getmtime(out) >= os.path.getmtime(_SRC)):
+            continue
+        tmp = out + f".tmp{os.getpid()}"
+        subprocess.run(["gcc", *_CFLAGS, f"-DREAL={ctype}", _SRC, "-o", tmp, "-lm"],
+                       check=True)
+        os.replace(tmp, out)
+
+
+def load_library(path: str, real: str) -> ctypes.CDLL:
+    """Load one oracle build and declare its signatures."""
+    lib = ctypes.CDLL(path)
+    R = ctypes.c_float if real == "f32" else ctypes.c_double
+    P = ctypes.c_void_p
+    i64, u32, u64, i32 = ctypes.c_int64, ctypes.c_uint32, ctypes.c_uint64, ctypes.c_int
+    lib.ora_real_bytes.restype = i32
+    lib.ora_real_bytes.argtypes = []
+    lib.ora_coef.restype = R
+    lib.ora_coef.argtypes = [i32, ctypes.c_float, i64]
+    lib.ora_apply_dense.restype = None
+    lib.ora_apply_dense.argtypes = [i32, i64, P, P, P, P, P, R, R, R, R]
+    lib.ora_apply_sparse.restype = i32
+    lib.ora_apply_sparse.argtypes = [i32, i64, P, P, P, P, i64, P, P, R, R, R, R]
+    lib.ora_philox4x32_10.restype = None
+    lib.ora_philox4x32_10.argtypes = [P, P, P]
+    lib.ora_draw.restype = u32
+    lib.ora_draw.argtypes = [u64, u32, u64, i64]
+    lib.ora_decide.restype = i32
+    lib.ora_decide.argtypes = [u32, ctypes.c_float, ctypes.c_float, ctypes.c_float]
+    lib.ora_select.restype = i64
+    lib.ora_select.argtypes = [i64, P, P, ctypes.c_float, ctypes.c_float, u64, u32, u64, P, P]
+    assert lib.ora_real_bytes() == (4 if real == "f32" else 8)
+    return lib
+
+
+def _load(real: str) -> ctypes.CDLL:
+    with _LOCK:
+        if real not in _LIBS:
+            build()
+            _LIBS[real] = load_library(lib_path(real), real)
+        return _LIBS[real]
+
+
+def _dtype(real: str):
+    return np.float32 if real == "f32" else np.float64
+
+
+def _ptr(a: np.ndarray) -> int:
+    assert a.flags["C_CONTIGUOUS"]
+    return a.ctypes.data
+
+
+def coef(variant: int, alpha: float, tau: int, real: str = "f32", lib=None):
+    """alpha(tau): alpha for ASGD, alpha / max(tau, 1) otherwise (Eq. 1, 7)."""
+    return (lib or _load(real)).ora_coef(variant, alpha, tau)
+
+
+def philox4x32_10(ctr, key, lib=None) -> list:
+    """Philox4x32-10 block: four 32-bit words from a 4-word counter, 2-word key."""
+    c = np.ascontiguousarray(ctr, dtype=np.uint32)
+    k = np.ascontiguousarray(key, dtype=np.uint32)
+    o = np.zeros(4, dtype=np.uint32)
+    (lib or _load("f32")).ora_philox4x32_10(_ptr(c), _ptr(k), _ptr(o))
+    return [int(x) for x in o]
+
+
+def draw(seed: int, client: int, push_no: int, p: int, lib=None) -> int:
+    """24-bit uniform draw u_p of one parameter for one push."""
+    return int((lib or _load("f32")).ora_draw(seed, client, push_no, p))
+
+
+def decide(u: int, v: float, c: float, eps_b: float, lib=None) -> bool:
+    """Eq. 9 in fp32: transmit iff u/2^24 < 1 / (1 + c / (v + eps_b))."""
+    return bool((lib or _load("f32")).ora_decide(u, v, c, eps_b))
+
+
+def select(g: np.ndarray, v: np.ndarray, c: float, eps_b: float, seed: int,
+           client: int, push_no: int, lib=None):
+    """B-FASGD send decision + compaction; returns (idx int32[m], val fp32[m])."""
+    g = np.ascontiguousarray(g, dtype=np.float32)
+    v = np.ascontiguousarray(v, dtype=np.float32)
+    P = g.shape[0]
+    idx = np.empty(max(P, 1), dtype=np.int32)
+    val = np.empty(max(P, 1), dtype=np.float32)
+    m = (lib or _load("f32")).ora_select(P, _ptr(g), _ptr(v), c, eps_b, seed, client, push_no,
+                                _ptr(idx), _ptr(val))
+    return idx[:m].copy(), val[:m].copy()
+
+
+class OracleError(Exception):
+    pass
+
+
+class OracleServer:
+    """The parameter server of Sections 2.1-2.3, one push at a time.
+
+    State theta, n, b, v (REAL[P]; n = b = v = 0 at start), timestamp T = 0,
+    and a FIFO of pushes.  ``apply_pending(K)`` pops the first K pushes in
+    arrival order; push k sees the server timestamp T it finds, so its
+    step-staleness is tau = T - j.
+    """
+
+    def __init__(self, P: int, lam: int, alpha: float, variant: int, real: str = "f32",
+                 gamma: float = 0.95, beta: float = 0.95, eps: float = 1e-4,
+                 c_push: float = 0.0, eps_b: float = 1e-8, seed: int = 0, lib=None):
+        self.lib = lib or _load(real)
+        self.real = real
+        dt = _dtype(real)
+        self.P, self.lam, self.alpha, self.variant = int(P), int(lam), float(alpha), int(variant)
+        self.theta = np.zeros(P, dtype=dt)
+        self.n = np.zeros(P, dtype=dt)
+        self.b = np.zeros(P, dtype=dt)
+        self.v = np.zeros(P, dtype=dt)
+        self.T = 0
+        self.fifo: list = []
+        self.push_count = [0] * lam
+        self.set_hparams(gamma, beta, eps, c_push, eps_b, seed)
+
+    def set_hparams(self, gamma, beta, eps, c_push, eps_b, seed):
+        # Hyper-parameters are fp32 at the boundary; the fp64 build widens them.
+        f = lambda x: float(np.float32(x))
+        self.gamma, self.beta, self.eps = f(gamma), f(beta), f(eps)
+        self.c_push, self.eps_b, self.seed = f(c_push), f(eps_b), int(seed)
+
+    def set_params(self, theta0: np.ndarray):
+        self.theta[:] = theta0
+
+    def push(self, client: int, j: int, g: np.ndarray):
+        self._check(client, j)
+        self.fifo.append(("dense", int(client), int(j), np.asarray(g, dtype=np.float32)))
+
+    def push_sparse(self, client: int, j: int, idx: np.ndarray, val: np.ndarray):
+        self._check(client, j)
+        self.fifo.append(("sparse", int(client), int(j),
+                          (np.ascontiguousarray(idx, dtype=np.int32),
+                           np.ascontiguousarray(val, dtype=np.float32))))
+
+    def _check(self, client, j):
+        if not 0 <= client < self.lam:
+            raise OracleError("client out of range")
+        if not 0 <= j <= self.T:
+            raise OracleError("timestamp out of range")
+
+    def apply_pending(self, K: int):
+        if K > len(self.fifo):
+            raise OracleError("fewer pending pushes than K")
+        for _ in range(K):
+            kind, client, j, payload = self.fifo.pop(0)
+            tau = self.T - j
+            c = self.lib.ora_coef(self.variant, self.alpha, tau)
+            if kind == "dense":
+                g = np.ascontiguousarray(payload, dtype=np.float32)
+                self.lib.ora_apply_dense(self.variant, self.P, _ptr(self.theta), _ptr(self.n),
+                                         _ptr(self.b), _ptr(self.v), _ptr(g), c,
+                                         self.gamma, self.beta, self.eps)
+            else:
+                idx, val = payload
+                rc = self.lib.ora_apply_sparse(self.variant, self.P, _ptr(self.theta),
+                                               _ptr(self.n), _ptr(self.b), _ptr(self.v),
+                                               idx.shape[0], _ptr(idx), _ptr(val), c,
+                                               self.gamma, self.beta, self.eps)
+                if rc != 0:
+                    raise OracleError("bad sparse list")
+            self.T += 1
+
+    def select_compact(self, client: int, g: np.ndarray, v: np.ndarray | None = None):
+        """B-FASGD push side for one client gradient; v defaults to the server's v."""
+        if not 0 <= client < self.lam:
+            raise OracleError("client out of range")
+        vv = (self.v if v is None else v).astype(np.float32)
+        out = select(g, vv, self.c_push, self.eps_b, self.seed, client,
+                     self.push_count[client], lib=self.lib if self.real == "f32" else None)
+        self.push_count[client] += 1
+        return out
+
+    def pull(self):
+        return self.theta.copy(), self.T
+
+    def state(self):
+        return self.theta.copy(), self.n.copy(), self.b.copy(), self.v.copy(), self.T

@@ -1,0 +1,218 @@
+/*
+ * FASGD / SASGD / ASGD / B-FASGD reference oracle -- TEST INFRASTRUCTURE ONLY.
+ *
+ * A plain, slow, single-threaded restatement of the update rules of
+ * "Faster Asynchronous SGD" (Odena, 2016), written to check the CUDA path.
+ * Only the tests, the smoke check and the CPU-baseline leg of the benchmark
+ * load it; the product path never does.  It shares no code, header, table or
+ * constant with the CUDA path.
+ *
+ * Precision: REAL is the type of the parameters and statistics.  The build
+ * makes two copies: REAL=float (the fp32 parameters and state the server
+ * keeps; every operation rounded once, IEEE round-to-nearest, compiled with
+ * -ffp-contract=off so nothing is fused) and REAL=double (the same rules in
+ * fp64, the exact-arithmetic yardstick for drift).  The B-FASGD send
+ * decision is always taken in fp32, the precision the kernel takes it in.
+ *
+ * Every function is elementwise over the parameter vector and follows the
+ * paper's order of operations:
+ *   Eq. 1-2  (Sec. 2.1)  g = alpha(tau) * dtheta,  theta <- theta - g
+ *   Eq. 4-6  (Sec. 2.2)  n, b moving averages; v moving average of 1/std
+ *   Eq. 7-8  (Sec. 2.2)  theta <- theta - alpha / (v * tau) * dtheta
+ *   Eq. 9    (Sec. 2.3)  transmit iff r < 1 / (1 + c / (v + eps))
+ * Readings where the paper is silent:
+ *   tau = 0 divides by zero in Eq. 1 and Eq. 7: the divisor is max(tau, 1);
+ *   n - b^2 can round below zero in floating point: it is clamped at 0
+ *   before eps is added (a no-op in exact arithmetic);
+ *   the step of Eq. 7 uses the v just updated by Eq. 6 (subscript i);
+ *   Eq. 9 is applied per parameter with that parameter's own v_p, and r is
+ *   u / 2^24 for a 24-bit counter-based draw u, compared strictly.
+ */
+#include <math.h>
+#include <stdint.h>
+
+#ifndef REAL
+#define REAL float
+#endif
+
+#define ORA_ASGD 0
+#define ORA_SASGD 1
+#define ORA_FASGD 2
+
+/* Size of REAL, so the Python side can check which build it loaded. */
+int ora_real_bytes(void) { return (int)sizeof(REAL); }
+
+/*
+ * Per-push learning-rate factor alpha(tau) of Eq. 1 and alpha / tau of
+ * Eq. 7 (the division by v is per element, in the step).  ASGD uses the
+ * master rate alone (the protocol of Sec. 2.1).  The quotient is formed in
+ * fp64 and rounded once to REAL.
+ */
+REAL ora_coef(int variant, float alpha, int64_t tau)
+{
+    if (variant == ORA_ASGD)
+        return (REAL)alpha;
+    int64_t t = tau < 1 ? 1 : tau;
+    return (REAL)((double)alpha / (double)t);
+}
+
+static REAL ora_sqrt(REAL x)
+{
+    return sizeof(REAL) == sizeof(float) ? (REAL)sqrtf((float)x) : (REAL)sqrt((double)x);
+}
+
+static REAL ora_max0(REAL x)
+{
+    return sizeof(REAL) == sizeof(float) ? (REAL)fmaxf((float)x, 0.0f) : (REAL)fmax((double)x, 0.0);
+}
+
+/*
+ * One server update of one parameter with gradient entry g.
+ * FASGD: Eq. 4, Eq. 5, Eq. 6, then Eq. 7-8 with the new v.
+ * ASGD / SASGD: Eq. 1-2 (the statistics are not touched).
+ */
+static void ora_update_one(int variant, REAL *theta, REAL *n, REAL *b, REAL *v,
+                           REAL g, REAL coef, REAL gamma, REAL beta, REAL eps)
+{
+    if (variant == ORA_FASGD) {
+        *n = gamma * *n + (1 - gamma) * (g * g);          /* Eq. 4 */
+        *b = gamma * *b + (1 - gamma) * g;                /* Eq. 5 */
+        REAL var = ora_max0(*n - *b * *b);
+        REAL r = 1 / ora_sqrt(var + eps);
+        *v = beta * *v + (1 - beta) * r;                  /* Eq. 6 */
+        *theta = *theta - coef * g / *v;                  /* Eq. 7-8 */
+    } else {
+        *theta = *theta - coef * g;                       /* Eq. 1-2 */
+    }
+}
+
+/* One dense push: every parameter p in [0, P) receives g[p]. */
+void ora_apply_dense(int variant, int64_t P, REAL *theta, REAL *n, REAL *b, REAL *v,
+                     const float *g, REAL coef, REAL gamma, REAL beta, REAL eps)
+{
+    for (int64_t p = 0; p < P; p++)
+        ora_update_one(variant, &theta[p], &n[p], &b[p], &v[p], (REAL)g[p], coef,
+                       gamma, beta, eps);
+}
+
+/*
+ * One sparse push: parameter idx[i] receives val[i] for i < count; every
+ * other parameter is left as it is (no decay of its statistics).
+ * Returns 0, or -1 (and applies nothing) if an index is out of range or
+ * the list is not strictly ascending.
+ */
+int ora_apply_sparse(int variant, int64_t P, REAL *theta, REAL *n, REAL *b, REAL *v,
+                     int64_t count, const int32_t *idx, const float *val, REAL coef,
+                     REAL gamma, REAL beta, REAL eps)
+{
+    for (int64_t i = 0; i < count; i++) {
+        if (idx[i] < 0 || idx[i] >= P)
+            return -1;
+        if (i > 0 && idx[i] <= idx[i - 1])
+            return -1;
+    }
+    for (int64_t i = 0; i < count; i++) {
+        int64_t p = idx[i];
+        ora_update_one(variant, &theta[p], &n[p], &b[p], &v[p], (REAL)val[i], coef,
+                       gamma, beta, eps);
+    }
+    return 0;
+}
+
+/*
+ * Philox4x32-10 (Salmon, Moraes, Dror, Shaw, "Parallel random numbers: as
+ * easy as 1, 2, 3", SC'11): ten rounds of the Philox S-box on a 128-bit
+ * counter under a 64-bit key, the key advanced by the Weyl increments
+ * between rounds.
+ */
+static void ora_mulhilo(uint32_t a, uint32_t b, uint32_t *hi, uint32_t *lo)
+{
+    uint64_t prod = (uint64_t)a * (uint64_t)b;
+    *hi = (uint32_t)(prod >> 32);
+    *lo = (uint32_t)prod;
+}
+
+void ora_philox4x32_10(const uint32_t ctr_in[4], const uint32_t key_in[2], uint32_t out[4])
+{
+    const uint32_t mult0 = 0xD2511F53u, mult1 = 0xCD9E8D57u;
+    const uint32_t weyl0 = 0x9E3779B9u, weyl1 = 0xBB67AE85u;
+    uint32_t x0 = ctr_in[0], x1 = ctr_in[1], x2 = ctr_in[2], x3 = ctr_in[3];
+    uint32_t k0 = key_in[0], k1 = key_in[1];
+    for (int round = 0; round < 10; round++) {
+        if (round > 0) {
+            k0 += weyl0;
+            k1 += weyl1;
+        }
+        uint32_t hi0, lo0, hi1, lo1;
+        ora_mulhilo(mult0, x0, &hi0, &lo0);
+        ora_mulhilo(mult1, x2, &hi1, &lo1);
+        uint32_t y0 = hi1 ^ x1 ^ k0;
+        uint32_t y1 = lo1;
+        uint32_t y2 = hi0 ^ x3 ^ k1;
+        uint32_t y3 = lo0;
+        x0 = y0; x1 = y1; x2 = y2; x3 = y3;
+    }
+    out[0] = x0; out[1] = x1; out[2] = x2; out[3] = x3;
+}
+
+/*
+ * The 24-bit uniform draw u_p for parameter p of one push.  The counter is
+ * (p div 4, client, push# low word, push# high word), the key is the 64-bit
+ * seed, and word (p mod 4) of the Philox output is used, shifted down to its
+ * top 24 bits; r = u / 2^24 lies in [0, 1).
+ */
+uint32_t ora_draw(uint64_t seed, uint32_t client, uint64_t push_no, int64_t p)
+{
+    uint32_t ctr[4] = {(uint32_t)(p >> 2), client, (uint32_t)push_no,
+                       (uint32_t)(push_no >> 32)};
+    uint32_t key[2] = {(uint32_t)seed, (uint32_t)(seed >> 32)};
+    uint32_t out[4];
+    ora_philox4x32_10(ctr, key, out);
+    return out[p & 3] >> 8;
+}
+
+/*
+ * Eq. 9 for one parameter, decided in fp32.  With a = fl(v + eps_b),
+ * d = fl(a + c) and r = u / 2^24, and a, d > 0:
+ *     r < 1 / (1 + c / a)  <=>  r < a / (a + c)  <=>  u * d < a * 2^24.
+ * The product u * d (24 x 24 bits) is split without error into
+ * prod + err (prod = fl(u*d), err = fma(u, d, -prod)), so the strict
+ * comparison is exact: below when prod < A, or prod == A and err < 0.
+ * Returns 1 to transmit, 0 to drop.
+ */
+int ora_decide(uint32_t u, float v, float c, float eps_b)
+{
+    float a = v + eps_b;
+    float d = a + c;
+    float uf = (float)u;
+    float prod = uf * d;
+    float err = fmaf(uf, d, -prod);
+    float A = a * 16777216.0f;
+    if (prod < A)
+        return 1;
+    if (prod == A && err < 0.0f)
+        return 1;
+    return 0;
+}
+
+/*
+ * B-FASGD per-parameter push decision and compaction (Sec. 2.3, applied per
+ * parameter as the paper's future-work section proposes): for p ascending,
+ * keep p iff Eq. 9 holds for v[p]; write idx[m] = p and val[m] = g[p]
+ * (bit copy).  Returns the number m of parameters kept.
+ */
+int64_t ora_select(int64_t P, const float *g, const float *v, float c, float eps_b,
+                   uint64_t seed, uint32_t client, uint64_t push_no,
+                   int32_t *idx, float *val)
+{
+    int64_t m = 0;
+    for (int64_t p = 0; p < P; p++) {
+        uint32_t u = ora_draw(seed, client, push_no, p);
+        if (ora_decide(u, v[p], c, eps_b)) {
+            idx[m] = (int32_t)p;
+            val[m] = g[p];
+            m++;
+        }
+    }
+    return m;
+}

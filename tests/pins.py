@@ -1,0 +1,456 @@
+"""Checks that pin the CPU oracle to what the paper and the mathematics fix.
+
+Each ``check_*`` takes an ``Libs`` (the fp32 and fp64 oracle builds) and
+raises AssertionError on a mismatch.  ``test_oracle_pins.py`` runs them on
+the real oracle; ``test_oracle_mutants.py`` runs them on copies of the oracle
+with a planted mistake and requires that at least one fails.
+
+None of these re-types the oracle's recursion: the references are closed
+forms, the unrolled (non-recursive) series, hand-worked values, exact
+rational arithmetic, published known-answer vectors, numpy's own fp32 SGD
+step, and invariants between the variants.
+"""
+
+from __future__ import annotations
+
+import dataclasses
+import json
+import math
+import os
+from fractions import Fraction
+
+import numpy as np
+
+import oracle
+from oracle import ASGD, FASGD, SASGD
+
+GOLDEN = os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden")
+
+
+@dataclasses.dataclass
+class Libs:
+    f32: object
+    f64: object
+
+    def lib(self, real):
+        return self.f32 if real == "f32" else self.f64
+
+
+def real_libs() -> Libs:
+    return Libs(oracle._load("f32"), oracle._load("f64"))
+
+
+def _server(libs, real, P, variant, alpha=0.25, lam=4, **hp):
+    return oracle.OracleServer(P, lam, alpha, variant, real=real, lib=libs.lib(real), **hp)
+
+
+def _rel(a, b):
+    a = np.asarray(a, dtype=np.float64)
+    b = np.asarray(b, dtype=np.float64)
+    return np.max(np.abs(a - b) / np.maximum(np.abs(b), 1e-300))
+
+
+# --------------------------------------------------------------------------
+# Hand trace exact in binary (Eq. 4-8)
+# --------------------------------------------------------------------------
+def check_hand_trace(libs: Libs):
+    gold = json.load(open(os.path.join(GOLDEN, "hand_trace_fasgd.json")))
+    hp = gold["hparams"]
+    env = {"sqrt": math.sqrt}
+    for real in ("f32", "f64"):
+        s = _server(libs, real, 1, FASGD, alpha=hp["alpha"], gamma=hp["gamma"],
+                    beta=hp["beta"], eps=hp["eps"])
+        s.set_params(np.array([hp["theta0"]]))
+        g = np.array([hp["g"]], dtype=np.float32)
+        for k, st in enumerate(gold["steps"]):
+            s.push(0, s.T, g)          # tau = 0
+            s.apply_pending(1)
+            want = {key: eval(st[key], env) for key in ("n", "b", "v", "theta")}
+            got = {"n": s.n[0], "b": s.b[0], "v": s.v[0], "theta": s.theta[0]}
+            for key in want:
+                if st["exact_in_binary"]:
+                    assert float(got[key]) == want[key], (real, k, key, got[key], want[key])
+                else:
+                    tol = 4e-7 if real == "f32" else 1e-15
+                    assert abs(float(got[key]) - want[key]) <= tol * abs(want[key]), \
+                        (real, k, key, got[key], want[key])
+
+
+# --------------------------------------------------------------------------
+# Constant gradient: closed-form geometric series (Eq. 4-8)
+# --------------------------------------------------------------------------
+def check_constant_gradient_closed_form(libs: Libs):
+    gvals = np.array([1.0, -0.5, 0.03125, -2e-3, 0.3, 7e-5, -1.25, 0.0], dtype=np.float32)
+    P = gvals.shape[0]
+    gamma, beta, eps, alpha = 0.9, 0.8, 1e-4, 0.01
+    rng = np.random.default_rng(5)
+    taus = rng.integers(0, 6, 60)
+    theta0 = np.linspace(-0.02, 0.02, P).astype(np.float32)
+    for real, steps, tol in (("f32", 40, 2e-5), ("f64", 60, 1e-11)):
+        s = _server(libs, real, P, FASGD, alpha=alpha, gamma=gamma, beta=beta, eps=eps)
+        s.set_params(theta0)
+        G, B = float(np.float32(gamma)), float(np.float32(beta))
+        E, A = float(np.float32(eps)), float(np.float32(alpha))
+        g64 = gvals.astype(np.float64)
+        theta_ref = theta0.astype(np.float64).copy()
+        rs = []
+        for i in range(1, steps + 1):
+            tau = min(int(taus[i - 1]), s.T)     # j = T - tau must be >= 0
+            s.push(0, s.T - tau, gvals)
+            s.apply_pending(1)
+            gi = G ** i
+            n_ref = (1 - gi) * g64 ** 2
+            b_ref = (1 - gi) * g64
+            var_ref = gi * (1 - gi) * g64 ** 2
+            rs.append(1 / np.sqrt(var_ref + E))
+            v_ref = (1 - B) * sum(B ** (i - k) * rs[k - 1] for k in range(1, i + 1))
+            theta_ref = theta_ref - A / max(tau, 1) * g64 / v_ref
+            assert _rel(s.n, n_ref) <= tol, (real, i, "n")
+            assert _rel(s.b, b_ref) <= tol, (real, i, "b")
+            assert _rel(s.v, v_ref) <= tol, (real, i, "v")
+            assert np.max(np.abs(s.theta - theta_ref)) <= tol * (np.max(np.abs(theta_ref)) + 1e-3), \
+                (real, i, "theta")
+
+
+# --------------------------------------------------------------------------
+# Random gradients, mixed staleness, dense and sparse pushes: the unrolled
+# series form of Eq. 4-8 (and Eq. 1-2) evaluated directly in fp64.
+# --------------------------------------------------------------------------
+def _series_reference(variant, theta0, events, alpha, gamma, beta, eps):
+    """events: list of (tau, {p: g}) in arrival order.  Returns theta, n, b, v."""
+    P = theta0.shape[0]
+    th = theta0.astype(np.float64).copy()
+    n = np.zeros(P)
+    b = np.zeros(P)
+    v = np.zeros(P)
+    for p in range(P):
+        hist = [(tau, g[p]) for tau, g in events if p in g]
+        rs = []
+        step_sum = 0.0
+        for i in range(1, len(hist) + 1):
+            tau_i, g_i = hist[i - 1]
+            c_i = alpha if variant == ASGD else alpha / max(tau_i, 1)
+            if variant == FASGD:
+                n_i = sum((1 - gamma) * gamma ** (i - k) * hist[k - 1][1] ** 2 for k in range(1, i + 1))
+                b_i = sum((1 - gamma) * gamma ** (i - k) * hist[k - 1][1] for k in range(1, i + 1))
+                rs.append(1 / math.sqrt(max(n_i - b_i ** 2, 0.0) + eps))
+                v_i = sum((1 - beta) * beta ** (i - k) * rs[k - 1] for k in range(1, i + 1))
+                step_sum += c_i * g_i / v_i
+                n[p], b[p], v[p] = n_i, b_i, v_i
+            else:
+                step_sum += c_i * g_i
+        th[p] = float(theta0[p]) - step_sum
+    return th, n, b, v
+
+
+def check_series_bruteforce(libs: Libs):
+    rng = np.random.default_rng(11)
+    P = 7
+    theta0 = (rng.standard_normal(P) * 0.01).astype(np.float32)
+    gamma, beta, eps, alpha = 0.85, 0.7, 1e-3, 0.05
+    steps = 24
+    plan = []
+    T = 0
+    for t in range(steps):
+        g = (rng.standard_normal(P) * rng.choice([0.01, 0.3, 1.0])).astype(np.float32)
+        d = int(rng.integers(0, 5))
+        j = T - min(d, T)
+        if t % 3 == 2:      # a sparse push on a random ascending subset
+            idx = np.sort(rng.choice(P, int(rng.integers(0, P + 1)), replace=False)).astype(np.int32)
+            plan.append(("sparse", j, idx, g[idx]))
+        else:
+            plan.append(("dense", j, None, g))
+        T += 1
+    for variant in (ASGD, SASGD, FASGD):
+        events = []
+        for T, (kind, j, idx, g) in enumerate(plan):
+            tau = T - j
+            if kind == "dense":
+                events.append((tau, {p: float(g[p]) for p in range(P)}))
+            else:
+                events.append((tau, {int(p): float(x) for p, x in zip(idx, g)}))
+        G, B = float(np.float32(gamma)), float(np.float32(beta))
+        E, A = float(np.float32(eps)), float(np.float32(alpha))
+        ref = _series_reference(variant, theta0, events, A, G, B, E)
+        for real, tol in (("f32", 3e-5), ("f64", 1e-12)):
+            s = _server(libs, real, P, variant, alpha=alpha, gamma=gamma, beta=beta, eps=eps)
+            s.set_params(theta0)
+            for kind, j, idx, g in plan:
+                if kind == "dense":
+                    s.push(1, j, g)
+                else:
+                    s.push_sparse(1, j, idx, g)
+                s.apply_pending(1)
+            got = s.state()[:4]
+            for name, a, r in zip(("theta", "n", "b", "v"), got, ref):
+                # elementwise relative error, floored at tol * the array's scale
+                bound = tol * (np.abs(r) + np.max(np.abs(r)) + 1e-30)
+                assert np.all(np.abs(a - r) <= bound), (variant, real, name,
+                                                        np.max(np.abs(a - r) / bound) * tol)
+
+
+# --------------------------------------------------------------------------
+# Variant invariants (Eq. 1-2 vs plain SGD; SASGD vs ASGD)
+# --------------------------------------------------------------------------
+def check_variant_invariants(libs: Libs):
+    rng = np.random.default_rng(3)
+    P = 33
+    theta0 = (rng.standard_normal(P) * 0.01).astype(np.float32)
+    grads = [(rng.standard_normal(P) * 0.1).astype(np.float32) for _ in range(12)]
+    alpha = 0.0123
+    # tau = 0 for every push: ASGD == SASGD == plain fp32 SGD (numpy), bitwise.
+    outs = {}
+    for variant in (ASGD, SASGD):
+        s = _server(libs, "f32", P, variant, alpha=alpha)
+        s.set_params(theta0)
+        for g in grads:
+            s.push(0, s.T, g)
+            s.apply_pending(1)
+        outs[variant] = s.theta.copy()
+    sgd = theta0.copy()
+    a32 = np.float32(alpha)
+    for g in grads:
+        sgd = (sgd - a32 * g).astype(np.float32)
+    assert np.array_equal(outs[ASGD].view(np.uint32), sgd.view(np.uint32))
+    assert np.array_equal(outs[SASGD].view(np.uint32), sgd.view(np.uint32))
+    # Constant tau = 3: SASGD(alpha) == ASGD(fl(alpha / 3)), bitwise.
+    tau = 3
+    s1 = _server(libs, "f32", P, SASGD, alpha=alpha)
+    s2 = _server(libs, "f32", P, ASGD, alpha=float(np.float32(np.float32(alpha) / np.float64(tau))))
+    for s in (s1, s2):
+        s.set_params(theta0)
+        for _ in range(tau):        # advance T so that j = T - 3 is legal
+            s.push(0, s.T, np.zeros(P, np.float32))
+            s.apply_pending(1)
+    th_start = s1.theta.copy()
+    assert np.array_equal(s2.theta, th_start)
+    for g in grads:
+        for s in (s1, s2):
+            s.push(0, s.T - tau, g)
+            s.apply_pending(1)
+    assert np.array_equal(s1.theta.view(np.uint32), s2.theta.view(np.uint32))
+    # SASGD with tau = 0 and tau = 1 coincide (the max(tau, 1) reading).
+    assert oracle.coef(SASGD, alpha, 0, lib=libs.f32) == oracle.coef(SASGD, alpha, 1, lib=libs.f32)
+    assert oracle.coef(ASGD, alpha, 7, lib=libs.f32) == np.float32(alpha)
+    # The statistics never move under ASGD / SASGD.
+    for variant in (ASGD, SASGD):
+        s = _server(libs, "f32", P, variant, alpha=alpha)
+        s.push(0, 0, grads[0])
+        s.apply_pending(1)
+        assert not s.n.any() and not s.b.any() and not s.v.any()
+
+
+def check_dense_equals_full_sparse(libs: Libs):
+    rng = np.random.default_rng(4)
+    P = 40
+    theta0 = (rng.standard_normal(P) * 0.01).astype(np.float32)
+    full = np.arange(P, dtype=np.int32)
+    for variant in (ASGD, SASGD, FASGD):
+        a = _server(libs, "f32", P, variant)
+        c = _server(libs, "f32", P, variant)
+        a.set_params(theta0)
+        c.set_params(theta0)
+        for t in range(15):
+            g = (rng.standard_normal(P) * 0.2).astype(np.float32)
+            j = a.T - min(t % 4, a.T)
+            a.push(t % 4, j, g)
+            c.push_sparse(t % 4, j, full, g)
+            a.apply_pending(1)
+            c.apply_pending(1)
+        for x, y in zip(a.state()[:4], c.state()[:4]):
+            assert np.array_equal(x.view(np.uint32), y.view(np.uint32))
+
+
+# --------------------------------------------------------------------------
+# Eq. 9: the fp32 send decision against exact rational arithmetic
+# --------------------------------------------------------------------------
+def _exact_decide(u, v, c, eps_b):
+    a = np.float32(np.float32(v) + np.float32(eps_b))
+    d = np.float32(a + np.float32(c))
+    if not (np.isfinite(a) and np.isfinite(d)):
+        return None
+    # u/2^24 < a/d  <=>  u*d < a*2^24   (a, d > 0)
+    return Fraction(int(u)) * Fraction(float(d)) < Fraction(float(a)) * (1 << 24)
+
+
+def check_decide_exact(libs: Libs):
+    gold = json.load(open(os.path.join(GOLDEN, "eq9_threshold_cases.json")))
+    for case in gold["cases"]:
+        got = oracle.decide(case["u"], case["v"], case["c"], case["eps_b"], lib=libs.f32)
+        assert got == case["send"], case
+    rng = np.random.default_rng(9)
+    for _ in range(4000):
+        v = float(np.float32(10 ** rng.uniform(-4, 3)))
+        c = float(np.float32(10 ** rng.uniform(-4, 3))) if rng.random() < 0.9 else 0.0
+        eps_b = float(np.float32(rng.choice([0.0, 1e-8, 1e-3])))
+        a = float(np.float32(np.float32(v) + np.float32(eps_b)))
+        d = float(np.float32(np.float32(a) + np.float32(c)))
+        if rng.random() < 0.5:      # aim at the threshold: ties and near-ties
+            u = int(np.clip(round(a * 2 ** 24 / d) + int(rng.integers(-2, 3)), 0, 2 ** 24 - 1))
+        else:
+            u = int(rng.integers(0, 2 ** 24))
+        want = _exact_decide(u, v, c, eps_b)
+        got = oracle.decide(u, v, c, eps_b, lib=libs.f32)
+        assert got == want, (u, v, c, eps_b)
+    # Threshold ties constructed exactly: a = 2^k, d = 2^m.
+    for k in range(-3, 4):
+        for m in range(k, k + 6):
+            a, d = 2.0 ** k, 2.0 ** m
+            u_tie = int(2 ** 24 * a / d)
+            if u_tie >= 2 ** 24 or u_tie < 1:
+                continue
+            c = d - a
+            assert oracle.decide(u_tie, a, c, 0.0, lib=libs.f32) is False
+            assert oracle.decide(u_tie - 1, a, c, 0.0, lib=libs.f32) is True
+
+
+# --------------------------------------------------------------------------
+# Philox4x32-10 known-answer vectors and the draw layout
+# --------------------------------------------------------------------------
+def check_philox_kat(libs: Libs):
+    gold = json.load(open(os.path.join(GOLDEN, "philox4x32_10_kat.json")))
+    for vec in gold["vectors"]:
+        ctr = [int(x, 16) for x in vec["ctr"]]
+        key = [int(x, 16) for x in vec["key"]]
+        want = [int(x, 16) for x in vec["out"]]
+        assert oracle.philox4x32_10(ctr, key, lib=libs.f32) == want, vec
+
+
+def check_draw_layout_and_uniformity(libs: Libs):
+    seed = 0x1234_5678_9ABC_DEF0
+    client, push_no = 7, (3 << 32) + 5
+    for p in (0, 1, 2, 3, 4, 5, 1023, 4 * 12345 + 2):
+        block = oracle.philox4x32_10([p >> 2, client, push_no & 0xFFFFFFFF, push_no >> 32],
+                                     [seed & 0xFFFFFFFF, seed >> 32], lib=libs.f32)
+        assert oracle.draw(seed, client, push_no, p, lib=libs.f32) == block[p & 3] >> 8
+    # Uniformity of u over [0, 2^24): chi-square on 64 bins, 64k draws.
+    us = np.array([oracle.draw(seed, 1, 2, p, lib=libs.f32) for p in range(1 << 16)])
+    assert us.max() < (1 << 24) and us.min() >= 0
+    hist = np.bincount(us >> 18, minlength=64)
+    exp = us.size / 64
+    chi2 = float(((hist - exp) ** 2 / exp).sum())
+    assert chi2 < 130, chi2          # 63 dof: p ~ 1e-6 above 130
+    # Different clients / push numbers give unrelated draws.
+    a = np.array([oracle.draw(seed, 1, 2, p, lib=libs.f32) for p in range(4096)])
+    b = np.array([oracle.draw(seed, 2, 2, p, lib=libs.f32) for p in range(4096)])
+    c = np.array([oracle.draw(seed, 1, 3, p, lib=libs.f32) for p in range(4096)])
+    assert abs(np.corrcoef(a, b)[0, 1]) < 0.08 and abs(np.corrcoef(a, c)[0, 1]) < 0.08
+
+
+# --------------------------------------------------------------------------
+# B-FASGD select / compact
+# --------------------------------------------------------------------------
+def check_select_properties(libs: Libs):
+    rng = np.random.default_rng(21)
+    P = 20001
+    g = (rng.standard_normal(P) * 0.1).astype(np.float32)
+    v = (10 ** rng.uniform(-1, 2, P)).astype(np.float32)
+    seed, eps_b = 77, 1e-8
+    # c = 0 keeps everything, in order, bit-copied.
+    idx, val = oracle.select(g, v, 0.0, eps_b, seed, 3, 0, lib=libs.f32)
+    assert np.array_equal(idx, np.arange(P, dtype=np.int32))
+    assert np.array_equal(val.view(np.uint32), g.view(np.uint32))
+    # A huge or infinite c keeps nothing.
+    for c in (3e38, float("inf")):
+        idx, _ = oracle.select(g, v, c, eps_b, seed, 3, 0, lib=libs.f32)
+        assert idx.size == 0
+    # Moderate c: ascending unique indices, bit-copied values, and a count
+    # within 5 sigma of the expected sum of the per-parameter probabilities.
+    for c in (1.0, 10.0, 60.0):
+        idx, val = oracle.select(g, v, c, eps_b, seed, 5, 9, lib=libs.f32)
+        assert np.all(np.diff(idx.astype(np.int64)) > 0)
+        assert np.array_equal(val.view(np.uint32), g[idx].view(np.uint32))
+        a = v.astype(np.float64) + eps_b
+        t = 1.0 / (1.0 + c / a)
+        mu, sd = t.sum(), math.sqrt((t * (1 - t)).sum())
+        assert abs(idx.size - mu) <= 5 * sd, (c, idx.size, mu, sd)
+        # Every index kept satisfies Eq. 9 for its own draw, and every index
+        # dropped violates it (checked with exact rationals on a sample).
+        keep = np.zeros(P, bool)
+        keep[idx] = True
+        for p in rng.choice(P, 300, replace=False):
+            u = oracle.draw(seed, 5, 9, int(p), lib=libs.f32)
+            assert _exact_decide(u, v[p], c, eps_b) == keep[p]
+
+
+def check_bfasgd_c0_equals_fasgd(libs: Libs):
+    rng = np.random.default_rng(8)
+    P = 301
+    theta0 = (rng.standard_normal(P) * 0.01).astype(np.float32)
+    dense = _server(libs, "f32", P, FASGD)
+    sparse = _server(libs, "f32", P, FASGD, c_push=0.0)
+    for s in (dense, sparse):
+        s.set_params(theta0)
+    for t in range(20):
+        g = (rng.standard_normal(P) * 0.05).astype(np.float32)
+        j = dense.T - min(t % 3, dense.T)
+        dense.push(t % 4, j, g)
+        idx, val = sparse.select_compact(t % 4, g)
+        sparse.push_sparse(t % 4, j, idx, val)
+        dense.apply_pending(1)
+        sparse.apply_pending(1)
+    for x, y in zip(dense.state()[:4], sparse.state()[:4]):
+        assert np.array_equal(x.view(np.uint32), y.view(np.uint32))
+
+
+def check_sparse_leaves_unsent_untouched(libs: Libs):
+    rng = np.random.default_rng(13)
+    P = 50
+    s = _server(libs, "f32", P, FASGD)
+    theta0 = (rng.standard_normal(P) * 0.01).astype(np.float32)
+    s.set_params(theta0)
+    g = (rng.standard_normal(P) * 0.1).astype(np.float32)
+    s.push(0, 0, g)
+    s.apply_pending(1)
+    before = [x.copy() for x in s.state()[:4]]
+    idx = np.array([1, 5, 6, 40], dtype=np.int32)
+    s.push_sparse(0, 1, idx, g[idx])
+    s.apply_pending(1)
+    after = s.state()[:4]
+    mask = np.ones(P, bool)
+    mask[idx] = False
+    for x, y in zip(before, after):
+        assert np.array_equal(x[mask], y[mask])
+        assert not np.array_equal(x[idx], y[idx])
+
+
+def check_protocol_errors(libs: Libs):
+    s = _server(libs, "f32", 4, FASGD, lam=2)
+    g = np.zeros(4, np.float32)
+    for bad in ((2, 0), (-1, 0), (0, 1), (0, -1)):
+        try:
+            s.push(bad[0], bad[1], g)
+        except oracle.OracleError:
+            pass
+        else:
+            raise AssertionError(f"push {bad} accepted")
+    try:
+        s.apply_pending(1)
+    except oracle.OracleError:
+        pass
+    else:
+        raise AssertionError("apply with empty queue accepted")
+    s.push(0, 0, g)
+    try:
+        s.push_sparse(0, 0, np.array([2, 1], np.int32), np.zeros(2, np.float32))
+        s.apply_pending(2)
+    except oracle.OracleError:
+        pass
+    else:
+        raise AssertionError("descending sparse list accepted")
+
+
+ALL_CHECKS = [
+    check_hand_trace,
+    check_constant_gradient_closed_form,
+    check_series_bruteforce,
+    check_variant_invariants,
+    check_dense_equals_full_sparse,
+    check_decide_exact,
+    check_philox_kat,
+    check_draw_layout_and_uniformity,
+    check_select_properties,
+    check_bfasgd_c0_equals_fasgd,
+    check_sparse_leaves_unsent_untouched,
+    check_protocol_errors,
+]

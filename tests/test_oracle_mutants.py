@@ -1,0 +1,81 @@
+"""Planted mistakes in the oracle are caught by the pins (no GPU).
+
+Each mutant is a copy of ``oracle/fasgd_oracle.c`` with one plausible slip
+(a dropped term, a wrong sign, a swapped operand or index, an off-by-one),
+built on the CPU into a temporary directory.  Every mutant must fail at
+least one check of ``pins.ALL_CHECKS``; a mutant that passes them all would
+show a hole in the pins.
+"""
+
+import os
+import subprocess
+
+import pytest
+
+import oracle
+import pins
+
+MUTANTS = {
+    "n_drops_one_minus_gamma": ("(1 - gamma) * (g * g)", "(g * g)"),
+    "n_uses_g_not_g2": ("(1 - gamma) * (g * g)", "(1 - gamma) * g"),
+    "b_swaps_gamma": ("*b = gamma * *b + (1 - gamma) * g", "*b = (1 - gamma) * *b + gamma * g"),
+    "var_sign": ("*n - *b * *b", "*n + *b * *b"),
+    "var_drops_b2": ("ora_max0(*n - *b * *b)", "ora_max0(*n)"),
+    "eps_dropped": ("ora_sqrt(var + eps)", "ora_sqrt(var)"),
+    "r_not_inverted": ("REAL r = 1 / ora_sqrt(var + eps);", "REAL r = ora_sqrt(var + eps);"),
+    "v_swaps_beta": ("*v = beta * *v + (1 - beta) * r", "*v = (1 - beta) * *v + beta * r"),
+    "step_times_v": ("coef * g / *v", "coef * g * *v"),
+    "step_sign": ("*theta = *theta - coef * g / *v", "*theta = *theta + coef * g / *v"),
+    "step_uses_old_v": (
+        "*v = beta * *v + (1 - beta) * r;                  /* Eq. 6 */\n"
+        "        *theta = *theta - coef * g / *v;                  /* Eq. 7-8 */",
+        "*theta = *theta - coef * g / (*v == 0 ? 1 : *v);\n"
+        "        *v = beta * *v + (1 - beta) * r;"),
+    "sgd_sign": ("*theta = *theta - coef * g;", "*theta = *theta + coef * g;"),
+    "tau_not_clamped_at_1": ("int64_t t = tau < 1 ? 1 : tau;", "int64_t t = tau < 1 ? 2 : tau;"),
+    "sasgd_multiplies": ("(double)alpha / (double)t", "(double)alpha * (double)t"),
+    "asgd_divides_too": ("    if (variant == ORA_ASGD)\n        return (REAL)alpha;\n", ""),
+    "philox_swaps_lo": ("uint32_t y1 = lo1;", "uint32_t y1 = lo0;"),
+    "philox_bumps_first": ("if (round > 0) {", "if (round >= 0) {"),
+    "philox_mult_constant": ("mult1 = 0xCD9E8D57u", "mult1 = 0xCD9E8D55u"),
+    "draw_wrong_word": ("out[p & 3] >> 8", "out[(p + 1) & 3] >> 8"),
+    "draw_low_bits": ("out[p & 3] >> 8", "out[p & 3] & 0xFFFFFFu"),
+    "draw_counter_no_client": ("(uint32_t)(p >> 2), client,", "(uint32_t)(p >> 2), 0u,"),
+    "decide_not_strict": ("prod == A && err < 0.0f", "prod == A && err <= 0.0f"),
+    "decide_ignores_err": ("if (prod == A && err < 0.0f)\n        return 1;\n", ""),
+    "decide_drops_eps": ("float a = v + eps_b;", "float a = v;"),
+    "select_val_index": ("val[m] = g[p];", "val[m] = g[m];"),
+    "select_idx_off_by_one": ("idx[m] = (int32_t)p;", "idx[m] = (int32_t)(p + 1);"),
+    "sparse_val_reversed": ("(REAL)val[i], coef,", "(REAL)val[count - 1 - i], coef,"),
+    "sparse_no_order_check": ("if (i > 0 && idx[i] <= idx[i - 1])\n            return -1;\n", ""),
+    "dense_skips_last": ("for (int64_t p = 0; p < P; p++)\n        ora_update_one",
+                         "for (int64_t p = 0; p < P - 1; p++)\n        ora_update_one"),
+}
+
+
+def _build_mutant(tmp_path, name, old, new):
+    src = open(oracle._SRC).read()
+    assert old in src, f"mutant {name}: pattern no longer in the oracle source"
+    mutated = src.replace(old, new, 1)
+    cpath = tmp_path / f"{name}.c"
+    cpath.write_text(mutated)
+    libs = {}
+    for real, ctype in (("f32", "float"), ("f64", "double")):
+        out = tmp_path / f"lib{name}_{real}.so"
+        subprocess.run(["gcc", *oracle._CFLAGS, "-w", f"-DREAL={ctype}", str(cpath),
+                        "-o", str(out), "-lm"], check=True)
+        libs[real] = oracle.load_library(str(out), real)
+    return pins.Libs(libs["f32"], libs["f64"])
+
+
+@pytest.mark.parametrize("name", sorted(MUTANTS))
+def test_mutant_is_caught(tmp_path, name):
+    old, new = MUTANTS[name]
+    libs = _build_mutant(tmp_path, name, old, new)
+    caught = []
+    for check in pins.ALL_CHECKS:
+        try:
+            check(libs)
+        except Exception as e:      # any failure of a pin counts as a catch
+            caught.append(f"{check.__name__}: {type(e).__name__}")
+    assert caught, f"mutant {name} passed every pin"
