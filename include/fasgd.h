@@ -1,0 +1,227 @@
+/*
+ * fasgd.h -- C ABI of the GB300 FASGD parameter-server library.
+ *
+ * The library is the server side of "Faster Asynchronous SGD" (Odena, 2016):
+ * it keeps the parameter vector theta and the per-parameter gradient
+ * statistics n, b, v in device memory, queues client pushes in arrival
+ * order, and applies them with the update rules of Sec. 2.1-2.2
+ * (ASGD, SASGD Eq. 1-2, FASGD Eq. 4-8).  It also implements the push side
+ * of B-FASGD (Sec. 2.3, Eq. 9) per parameter: the send decision, the
+ * compaction of the sent entries into index/value lists, and the sparse
+ * server apply of such lists.
+ *
+ * Conventions shared by every call
+ *   - Return value: FASGD_OK (0) or a negative fasgd_status.  A call that
+ *     fails validation changes no state.  fasgd_last_error() describes the
+ *     most recent failure on a handle (or, with NULL, of fasgd_create).
+ *   - Asynchrony: every call that touches device memory is enqueued on the
+ *     handle's stream (fasgd_set_stream) and returns before the GPU is done.
+ *     Only values written to host memory by the call itself (timestamps,
+ *     counts) are final on return.  Device-side checks on caller-supplied
+ *     index lists are reported by fasgd_sync().
+ *   - Ownership: the handle owns theta, n, b, v and its scratch buffers.
+ *     Every other pointer belongs to the caller and is only borrowed; a
+ *     buffer passed to fasgd_push / fasgd_push_sparse must stay valid and
+ *     unmodified until the fasgd_apply_pending call that consumes it has
+ *     completed on the stream.
+ *   - Pointers: "device" pointers must be device-accessible (cudaMalloc,
+ *     torch CUDA tensors).  Dense fp32[P] vectors (gradients, v) must be
+ *     16-byte aligned (they are read 128 bits at a time); index / value
+ *     lists 4-byte and counts 8-byte aligned.  "host or device" pointers may
+ *     also be host memory (pinned host memory keeps the copy asynchronous).
+ *   - Sizes: 1 <= P < 2^31 (indices are int32), 1 <= lambda <= 2^20,
+ *     1 <= K <= FASGD_KMAX pushes per apply.
+ *   - Threads: a handle is used by one host thread at a time.
+ */
+#ifndef FASGD_H
+#define FASGD_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct fasgd_s fasgd_t;
+
+/* Every entry point is exported from the shared library. */
+#if defined(__GNUC__)
+#define FASGD_API __attribute__((visibility("default")))
+#else
+#define FASGD_API
+#endif
+
+/* Update rule of the server (Sec. 2.1-2.2). */
+enum fasgd_variant {
+    FASGD_ASGD = 0,   /* theta -= alpha * g                       (Sec. 2.1, protocol step 2) */
+    FASGD_SASGD = 1,  /* theta -= alpha / max(tau,1) * g           (Eq. 1-2) */
+    FASGD_FASGD = 2   /* n, b, v moving averages, then
+                         theta -= alpha / (v * max(tau,1)) * g     (Eq. 4-8) */
+};
+
+enum fasgd_status {
+    FASGD_OK = 0,
+    FASGD_EINVAL = -1,   /* bad argument: NULL or misaligned pointer, size or
+                            hyper-parameter outside its domain, bad variant */
+    FASGD_ERANGE = -2,   /* client outside [0, lambda) or timestamp outside [0, T] */
+    FASGD_EAGAIN = -3,   /* fewer than K pending pushes, queue or staging full,
+                            or pushes still pending where none may be */
+    FASGD_ENOMEM = -4,   /* device or pinned allocation failed */
+    FASGD_ECUDA = -5,    /* a CUDA runtime call failed (text in fasgd_last_error) */
+    FASGD_EDEVICE = -6   /* a kernel found a bad entry in a caller's sparse list */
+};
+
+#define FASGD_KMAX 32                         /* pushes one apply may fuse */
+#define FASGD_PMAX ((int64_t)2147483647)      /* P must be below 2^31 */
+
+/*
+ * fasgd_create -- make a server with P fp32 parameters for lambda clients.
+ * Sec. 2.1 notation: lambda clients, master learning rate alpha, timestamp
+ * T starting at 0.  theta, n, b, v are allocated on the current CUDA device
+ * and zero-filled (the statistics start at 0; set theta with
+ * fasgd_set_params).  Default hyper-parameters: gamma = beta = 0.95,
+ * eps = 1e-4, c_push = 0 (send everything), eps_b = 1e-8, seed = 0.
+ * Errors: EINVAL (h NULL, P or lambda out of range, alpha not finite, bad
+ * variant), ENOMEM, ECUDA.  On error *h is set to NULL.
+ */
+FASGD_API int fasgd_create(fasgd_t** h, int64_t P, int32_t lambda, float alpha, int32_t variant);
+
+/* Free every device buffer of the handle (after the stream drains).  NULL is ignored. */
+FASGD_API void fasgd_destroy(fasgd_t* h);
+
+/*
+ * fasgd_set_hparams -- gamma, beta (Eq. 4-6 moving-average factors),
+ * eps (Eq. 6 stabiliser), c_push and eps_b (Eq. 9 threshold and its
+ * stabiliser) and the 64-bit seed of the B-FASGD draws.
+ * Domain: 0 <= gamma <= 1, 0 <= beta < 1, eps and eps_b finite and >= 0,
+ * c_push >= 0 (+inf allowed: nothing is sent).  The send decision needs
+ * v_p + eps_b > 0 (eps_b > 0 guarantees it) and below 2^103 (so that
+ * (v_p + eps_b) * 2^24 stays finite in fp32).
+ * Errors: EINVAL (outside the domain), EAGAIN (pushes pending).
+ */
+FASGD_API int fasgd_set_hparams(fasgd_t* h, float gamma, float beta, float eps, float c_push,
+                      float eps_b, uint64_t seed);
+
+/* Stream every later call is enqueued on (a cudaStream_t; NULL = legacy default stream). */
+FASGD_API int fasgd_set_stream(fasgd_t* h, void* stream);
+
+/*
+ * fasgd_set_params -- copy P initial parameters (host or device pointer)
+ * into theta.  n, b, v are left as they are.  Errors: EINVAL, EAGAIN
+ * (pushes pending), ECUDA.
+ */
+FASGD_API int fasgd_set_params(fasgd_t* h, const float* theta0);
+
+/*
+ * fasgd_push -- queue one dense client gradient (Sec. 2.1, protocol step 1).
+ * client in [0, lambda); timestamp j = the server timestamp of the
+ * parameters the gradient was computed on, 0 <= j <= T (T = the server's
+ * current timestamp; pushes already queued do not advance it).
+ * grad: device pointer to P fp32 values, 16-byte aligned, borrowed until
+ * the apply that consumes it completes on the stream.
+ * Errors: EINVAL, ERANGE, EAGAIN (queue holds 2^20 pushes).
+ */
+FASGD_API int fasgd_push(fasgd_t* h, int32_t client, int64_t timestamp, const float* grad);
+
+/*
+ * fasgd_push_host -- as fasgd_push, for a gradient in host memory: the P
+ * values are copied (asynchronously, on the stream) into a device staging
+ * slot owned by the handle, so the host buffer must stay unchanged until
+ * the stream reaches the copy (pinned memory makes the copy asynchronous).
+ * At most FASGD_KMAX host pushes may be pending; the first use of each
+ * staging slot allocates it.  Errors: EINVAL, ERANGE, EAGAIN, ENOMEM, ECUDA.
+ */
+FASGD_API int fasgd_push_host(fasgd_t* h, int32_t client, int64_t timestamp, const float* grad_host);
+
+/*
+ * fasgd_push_sparse -- queue one sparse push: parameter idx[i] receives
+ * gradient entry val[i] for i < count; every other parameter is left alone
+ * (its statistics do not decay).  This is the server side of a B-FASGD push
+ * whose unsent entries are dropped.
+ * idx: device int32 list, strictly ascending, each in [0, P).
+ * val: device fp32 list.  count: read on the device from *n_dev when n_dev
+ * is not NULL (as written by bfasgd_select_compact), else count = n_max.
+ * n_max: host-side upper bound, 0 <= n_max <= P; idx and val hold at least
+ * n_max entries.  All three buffers are borrowed until the consuming apply
+ * completes.  A count above n_max, an index out of range or out of order
+ * is skipped on the device and reported by fasgd_sync() as EDEVICE.
+ * Errors: EINVAL, ERANGE, EAGAIN.
+ */
+FASGD_API int fasgd_push_sparse(fasgd_t* h, int32_t client, int64_t timestamp, const int32_t* idx,
+                      const float* val, const int64_t* n_dev, int64_t n_max);
+
+/*
+ * fasgd_apply_pending -- apply the first K queued pushes in arrival order
+ * (Sec. 2.1 protocol step 2; Eq. 1-2 or Eq. 4-8 per the variant).  Push k of
+ * the batch (k = 0..K-1) is applied at server timestamp T + k, so its
+ * step-staleness is tau_k = T + k - j_k, and alpha(tau) = alpha / max(tau,1).
+ * Consecutive dense pushes are fused into one pass over the parameters that
+ * keeps each element's theta, n, b, v in registers across them; each sparse
+ * push is its own pass.  T increases by K.
+ * Errors: EINVAL (K < 1 or K > FASGD_KMAX), EAGAIN (fewer than K pending), ECUDA.
+ */
+FASGD_API int fasgd_apply_pending(fasgd_t* h, int32_t K);
+
+/*
+ * bfasgd_select_compact -- B-FASGD push decision and compaction (Sec. 2.3,
+ * Eq. 9, taken per parameter with the parameter's own v_p).
+ * For every p, u_p is the top 24 bits of word (p mod 4) of Philox4x32-10
+ * (Salmon et al., SC'11) with counter (p div 4, client, push#, push# >> 32)
+ * and key = seed, where push# counts this client's earlier calls.  With
+ * a = fl(v_p + eps_b) and d = fl(a + c_push), p is sent iff
+ * u_p * d < a * 2^24 exactly, i.e. u_p / 2^24 < 1 / (1 + c_push / a).
+ * Outputs: idx[0..m) = the sent p in ascending order (int32), val[i] =
+ * grad[idx[i]] (bit copy), *n_dev = m (int64), all written on the stream.
+ * grad: device fp32[P]; v: device fp32[P] (the client's copy of the server
+ * statistic), or NULL to use the server's live v.  idx, val: device, room
+ * for P entries.  Uses handle-owned scratch (a bit mask and per-tile counts).
+ * Errors: EINVAL, ERANGE (client), ECUDA.  On success the client's push#
+ * advances by one.
+ */
+FASGD_API int bfasgd_select_compact(fasgd_t* h, int32_t client, const float* grad, const float* v,
+                          int32_t* idx, float* val, int64_t* n_dev);
+
+/*
+ * fasgd_pull -- copy theta (P fp32) into params (host or device) on the
+ * stream and return the server timestamp T in *T (Sec. 2.1 protocol step 3:
+ * the parameters handed back to a client).  Pending pushes are not applied.
+ * Either output may be NULL.  Errors: EINVAL, ECUDA.
+ */
+FASGD_API int fasgd_pull(fasgd_t* h, float* params, int64_t* T);
+
+/*
+ * fasgd_get_state / fasgd_set_state -- checkpoint and restore theta, n, b, v
+ * (P fp32 each; host or device; any may be NULL to skip it) and T.
+ * Both require an empty queue.  get_state blocks until the copies are done.
+ * Errors: EINVAL, EAGAIN (pushes pending), ECUDA.
+ */
+FASGD_API int fasgd_get_state(fasgd_t* h, float* theta, float* n, float* b, float* v, int64_t* T);
+FASGD_API int fasgd_set_state(fasgd_t* h, const float* theta, const float* n, const float* b,
+                    const float* v, int64_t T);
+
+/* Per-client B-FASGD push counters (lambda uint64 values, host memory). */
+FASGD_API int fasgd_get_push_counts(fasgd_t* h, uint64_t* counts);
+FASGD_API int fasgd_set_push_counts(fasgd_t* h, const uint64_t* counts);
+
+/*
+ * fasgd_sync -- wait until the handle's stream is idle, then report and
+ * clear the device-side error flags: FASGD_EDEVICE if a sparse list held a
+ * bad entry since the last sync, else FASGD_OK (or ECUDA).
+ */
+FASGD_API int fasgd_sync(fasgd_t* h);
+
+/* Server timestamp T (pushes applied so far) and number of queued pushes. */
+FASGD_API int64_t fasgd_timestamp(const fasgd_t* h);
+FASGD_API int64_t fasgd_pending(const fasgd_t* h);
+
+/* Number of kernels this handle has launched since it was created. */
+FASGD_API int64_t fasgd_kernel_launches(const fasgd_t* h);
+
+/* Text of the last failure on h (or of the last failed fasgd_create when h is NULL). */
+FASGD_API const char* fasgd_last_error(const fasgd_t* h);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* FASGD_H */

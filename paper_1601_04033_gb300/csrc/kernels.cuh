@@ -1,0 +1,84 @@
+// Internal interface between the host runtime (runtime.cu) and the kernels
+// (dense.cu, select.cu, sparse.cu).  Not part of the public C ABI.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "fasgd.h"
+
+namespace fasgd {
+
+// Hyper-parameters of Eq. 4-6 as the kernels consume them.  one_m_gamma and
+// one_m_beta are formed once on the host in fp32 (1 - gamma, 1 - beta).
+struct StatParams {
+    float gamma, one_m_gamma;
+    float beta, one_m_beta;
+    float eps;
+};
+
+// One fused pass over the parameters applying K dense pushes in order.
+struct DenseArgs {
+    float* theta;
+    float* n;
+    float* b;
+    float* v;
+    const float* grad[FASGD_KMAX];  // grad[k]: push k's gradient, fp32[P]
+    float coef[FASGD_KMAX];         // alpha(tau_k) of push k (Eq. 1 / Eq. 7 without v)
+    int64_t P;
+    int32_t K;
+    StatParams sp;
+};
+
+// One sparse push: idx[i] receives val[i] for i < count.
+struct SparseArgs {
+    float* theta;
+    float* n;
+    float* b;
+    float* v;
+    const int32_t* idx;
+    const float* val;
+    const int64_t* count_dev;  // may be null: count = count_max
+    int64_t count_max;
+    int64_t P;
+    float coef;
+    StatParams sp;
+    int32_t* err;              // device error flags (bit 0: count, bit 1: index, bit 2: order)
+};
+
+// Elements per tile of the select / compact kernels, and the bit mask words a
+// tile owns (one bit per element).
+constexpr int kSelectThreads = 256;
+constexpr int kSelectTile = 8192;
+constexpr int kSelectTileWords = kSelectTile / 32;
+
+struct SelectArgs {
+    const float* grad;
+    const float* v;
+    int32_t* idx;
+    float* val;
+    int64_t* count;      // total number sent (int64, device)
+    uint32_t* mask;      // scratch: ntiles * kSelectTileWords words
+    int32_t* tile_count; // scratch: ntiles
+    int64_t* tile_base;  // scratch: ntiles
+    int64_t P;
+    int32_t ntiles;
+    float c;
+    float eps_b;
+    uint32_t key0, key1;           // Philox key = seed
+    uint32_t client, push_lo, push_hi;
+};
+
+// Launchers: enqueue on `stream`, return the launch status.
+// `launches` is incremented by the number of kernels enqueued.
+cudaError_t launch_dense(const DenseArgs& a, bool fasgd_rule, int num_sms, cudaStream_t stream,
+                         int64_t* launches);
+cudaError_t launch_sparse(const SparseArgs& a, bool fasgd_rule, int num_sms, cudaStream_t stream,
+                          int64_t* launches);
+cudaError_t launch_select(const SelectArgs& a, cudaStream_t stream, int64_t* launches);
+
+inline int32_t select_tiles(int64_t P) {
+    return (int32_t)((P + kSelectTile - 1) / kSelectTile);
+}
+
+}  // namespace fasgd

@@ -1,0 +1,501 @@
+// Host runtime behind include/fasgd.h: the handle, argument checks, the
+// queue of pending pushes, the per-push staleness factors and the launches.
+//
+// Protocol (paper Sec. 2.1): a client push carries its gradient and the
+// timestamp j of the parameters it was computed on; the server applies
+// pushes one at a time in arrival order, each at the server timestamp T it
+// finds (step-staleness tau = T - j), and T grows by one per applied push.
+// Here a batch of K queued pushes is applied by one call: push k of the
+// batch sees T + k.  The per-push factor alpha(tau) = alpha / max(tau, 1)
+// (Eq. 1, Eq. 7 without the per-element v) is formed on the host in fp64 and
+// rounded once to fp32.
+
+#include <cuda_runtime.h>
+
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <deque>
+#include <new>
+#include <string>
+#include <vector>
+
+#include "fasgd.h"
+#include "kernels.cuh"
+
+namespace {
+
+constexpr int64_t kMaxQueue = int64_t(1) << 20;
+constexpr int32_t kMaxLambda = int32_t(1) << 20;
+
+thread_local std::string g_create_error;
+
+struct Push {
+    bool sparse;
+    int32_t client;
+    int64_t j;
+    const float* grad;     // dense
+    const int32_t* idx;    // sparse
+    const float* val;
+    const int64_t* n_dev;
+    int64_t n_max;
+    int stage;             // staging slot of a host push, -1 otherwise
+};
+
+bool aligned(const void* p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) & (a - 1)) == 0; }
+
+std::string vformat(const char* fmt, va_list ap) {
+    char buf[512];
+    vsnprintf(buf, sizeof buf, fmt, ap);
+    return buf;
+}
+
+// Makes h's device current for the lifetime of the guard.
+struct DeviceGuard {
+    int prev = -1;
+    explicit DeviceGuard(int dev) {
+        if (cudaGetDevice(&prev) == cudaSuccess && prev != dev) cudaSetDevice(dev);
+        else prev = -1;
+    }
+    ~DeviceGuard() {
+        if (prev >= 0) cudaSetDevice(prev);
+    }
+};
+
+}  // namespace
+
+struct fasgd_s {
+    int64_t P = 0;
+    int32_t lambda = 0;
+    float alpha = 0.f;
+    int32_t variant = FASGD_FASGD;
+    float gamma = 0.95f, beta = 0.95f, eps = 1e-4f, c_push = 0.f, eps_b = 1e-8f;
+    uint64_t seed = 0;
+    cudaStream_t stream = nullptr;
+    int device = 0;
+    int num_sms = 0;
+    float* theta = nullptr;
+    float* n = nullptr;
+    float* b = nullptr;
+    float* v = nullptr;
+    uint32_t* mask = nullptr;
+    int32_t* tile_count = nullptr;
+    int64_t* tile_base = nullptr;
+    int32_t* dev_err = nullptr;
+    int32_t ntiles = 0;
+    std::vector<float*> stage;
+    std::vector<char> stage_busy;
+    std::deque<Push> fifo;
+    int64_t T = 0;
+    int64_t launches = 0;
+    std::vector<uint64_t> push_count;
+    std::string err;
+
+    int fail(int code, const char* fmt, ...) {
+        va_list ap;
+        va_start(ap, fmt);
+        err = vformat(fmt, ap);
+        va_end(ap);
+        return code;
+    }
+    int cuda_fail(cudaError_t st, const char* what) {
+        return fail(st == cudaErrorMemoryAllocation ? FASGD_ENOMEM : FASGD_ECUDA, "%s: %s", what,
+                    cudaGetErrorString(st));
+    }
+    fasgd::StatParams stat_params() const {
+        fasgd::StatParams sp;
+        sp.gamma = gamma;
+        sp.one_m_gamma = 1.0f - gamma;
+        sp.beta = beta;
+        sp.one_m_beta = 1.0f - beta;
+        sp.eps = eps;
+        return sp;
+    }
+    // alpha(tau) of Eq. 1 / Eq. 7 (the v factor of Eq. 7 is per element).
+    float coef(int64_t tau) const {
+        if (variant == FASGD_ASGD) return alpha;
+        const int64_t t = tau < 1 ? 1 : tau;
+        return (float)((double)alpha / (double)t);
+    }
+    void free_all() {
+        float* arrs[] = {theta, n, b, v};
+        for (float* p : arrs) cudaFree(p);
+        cudaFree(mask);
+        cudaFree(tile_count);
+        cudaFree(tile_base);
+        cudaFree(dev_err);
+        for (float* s : stage) cudaFree(s);
+        theta = n = b = v = nullptr;
+        mask = nullptr;
+        tile_count = nullptr;
+        tile_base = nullptr;
+        dev_err = nullptr;
+        stage.clear();
+    }
+};
+
+extern "C" {
+
+int fasgd_create(fasgd_t** h, int64_t P, int32_t lambda, float alpha, int32_t variant) {
+    if (h == nullptr) {
+        g_create_error = "fasgd_create: h is NULL";
+        return FASGD_EINVAL;
+    }
+    *h = nullptr;
+    if (P < 1 || P > FASGD_PMAX) {
+        g_create_error = "fasgd_create: P must be in [1, 2^31)";
+        return FASGD_EINVAL;
+    }
+    if (lambda < 1 || lambda > kMaxLambda) {
+        g_create_error = "fasgd_create: lambda must be in [1, 2^20]";
+        return FASGD_EINVAL;
+    }
+    if (!std::isfinite(alpha)) {
+        g_create_error = "fasgd_create: alpha must be finite";
+        return FASGD_EINVAL;
+    }
+    if (variant != FASGD_ASGD && variant != FASGD_SASGD && variant != FASGD_FASGD) {
+        g_create_error = "fasgd_create: unknown variant";
+        return FASGD_EINVAL;
+    }
+    fasgd_s* s = new (std::nothrow) fasgd_s();
+    if (s == nullptr) {
+        g_create_error = "fasgd_create: out of host memory";
+        return FASGD_ENOMEM;
+    }
+    s->P = P;
+    s->lambda = lambda;
+    s->alpha = alpha;
+    s->variant = variant;
+    s->push_count.assign((size_t)lambda, 0);
+    s->ntiles = fasgd::select_tiles(P);
+    cudaError_t st = cudaGetDevice(&s->device);
+    if (st == cudaSuccess)
+        st = cudaDeviceGetAttribute(&s->num_sms, cudaDevAttrMultiProcessorCount, s->device);
+    const size_t bytes = (size_t)P * sizeof(float);
+    float** arrs[] = {&s->theta, &s->n, &s->b, &s->v};
+    for (float** a : arrs)
+        if (st == cudaSuccess) st = cudaMalloc(reinterpret_cast<void**>(a), bytes);
+    if (st == cudaSuccess)
+        st = cudaMalloc(reinterpret_cast<void**>(&s->mask),
+                        (size_t)s->ntiles * fasgd::kSelectTileWords * sizeof(uint32_t));
+    if (st == cudaSuccess)
+        st = cudaMalloc(reinterpret_cast<void**>(&s->tile_count), (size_t)s->ntiles * sizeof(int32_t));
+    if (st == cudaSuccess)
+        st = cudaMalloc(reinterpret_cast<void**>(&s->tile_base), (size_t)s->ntiles * sizeof(int64_t));
+    if (st == cudaSuccess) st = cudaMalloc(reinterpret_cast<void**>(&s->dev_err), sizeof(int32_t));
+    for (float** a : arrs)
+        if (st == cudaSuccess) st = cudaMemset(*a, 0, bytes);
+    if (st == cudaSuccess) st = cudaMemset(s->dev_err, 0, sizeof(int32_t));
+    if (st == cudaSuccess) st = cudaDeviceSynchronize();
+    if (st != cudaSuccess) {
+        g_create_error = std::string("fasgd_create: ") + cudaGetErrorString(st);
+        s->free_all();
+        delete s;
+        return st == cudaErrorMemoryAllocation ? FASGD_ENOMEM : FASGD_ECUDA;
+    }
+    *h = s;
+    return FASGD_OK;
+}
+
+void fasgd_destroy(fasgd_t* h) {
+    if (h == nullptr) return;
+    DeviceGuard g(h->device);
+    cudaStreamSynchronize(h->stream);
+    h->free_all();
+    delete h;
+}
+
+int fasgd_set_hparams(fasgd_t* h, float gamma, float beta, float eps, float c_push, float eps_b,
+                      uint64_t seed) {
+    if (h == nullptr) return FASGD_EINVAL;
+    if (!(gamma >= 0.f && gamma <= 1.f)) return h->fail(FASGD_EINVAL, "gamma must be in [0, 1]");
+    if (!(beta >= 0.f && beta < 1.f)) return h->fail(FASGD_EINVAL, "beta must be in [0, 1)");
+    if (!(eps >= 0.f) || !std::isfinite(eps)) return h->fail(FASGD_EINVAL, "eps must be finite and >= 0");
+    if (!(c_push >= 0.f)) return h->fail(FASGD_EINVAL, "c_push must be >= 0 (may be +inf)");
+    if (!(eps_b >= 0.f) || !std::isfinite(eps_b))
+        return h->fail(FASGD_EINVAL, "eps_b must be finite and >= 0");
+    if (!h->fifo.empty()) return h->fail(FASGD_EAGAIN, "pushes are pending");
+    h->gamma = gamma;
+    h->beta = beta;
+    h->eps = eps;
+    h->c_push = c_push;
+    h->eps_b = eps_b;
+    h->seed = seed;
+    return FASGD_OK;
+}
+
+int fasgd_set_stream(fasgd_t* h, void* stream) {
+    if (h == nullptr) return FASGD_EINVAL;
+    if (!h->fifo.empty()) return h->fail(FASGD_EAGAIN, "pushes are pending");
+    h->stream = static_cast<cudaStream_t>(stream);
+    return FASGD_OK;
+}
+
+int fasgd_set_params(fasgd_t* h, const float* theta0) {
+    if (h == nullptr) return FASGD_EINVAL;
+    if (theta0 == nullptr) return h->fail(FASGD_EINVAL, "theta0 is NULL");
+    if (!h->fifo.empty()) return h->fail(FASGD_EAGAIN, "pushes are pending");
+    DeviceGuard g(h->device);
+    cudaError_t st = cudaMemcpyAsync(h->theta, theta0, (size_t)h->P * sizeof(float),
+                                     cudaMemcpyDefault, h->stream);
+    if (st != cudaSuccess) return h->cuda_fail(st, "fasgd_set_params");
+    return FASGD_OK;
+}
+
+static int check_push(fasgd_t* h, int32_t client, int64_t timestamp) {
+    if (client < 0 || client >= h->lambda)
+        return h->fail(FASGD_ERANGE, "client %d outside [0, %d)", client, h->lambda);
+    if (timestamp < 0 || timestamp > h->T)
+        return h->fail(FASGD_ERANGE, "timestamp %lld outside [0, T=%lld]", (long long)timestamp,
+                       (long long)h->T);
+    if ((int64_t)h->fifo.size() >= kMaxQueue) return h->fail(FASGD_EAGAIN, "push queue is full");
+    return FASGD_OK;
+}
+
+int fasgd_push(fasgd_t* h, int32_t client, int64_t timestamp, const float* grad) {
+    if (h == nullptr) return FASGD_EINVAL;
+    if (grad == nullptr || !aligned(grad, 16))
+        return h->fail(FASGD_EINVAL, "grad must be a non-NULL 16-byte aligned device pointer");
+    int rc = check_push(h, client, timestamp);
+    if (rc != FASGD_OK) return rc;
+    h->fifo.push_back(Push{false, client, timestamp, grad, nullptr, nullptr, nullptr, 0, -1});
+    return FASGD_OK;
+}
+
+int fasgd_push_host(fasgd_t* h, int32_t client, int64_t timestamp, const float* grad_host) {
+    if (h == nullptr) return FASGD_EINVAL;
+    if (grad_host == nullptr) return h->fail(FASGD_EINVAL, "grad_host is NULL");
+    int rc = check_push(h, client, timestamp);
+    if (rc != FASGD_OK) return rc;
+    int slot = -1;
+    for (size_t s = 0; s < h->stage.size(); ++s)
+        if (!h->stage_busy[s]) {
+            slot = (int)s;
+            break;
+        }
+    DeviceGuard g(h->device);
+    if (slot < 0) {
+        if ((int)h->stage.size() >= FASGD_KMAX)
+            return h->fail(FASGD_EAGAIN, "%d host pushes already pending", FASGD_KMAX);
+        float* p = nullptr;
+        cudaError_t st = cudaMalloc(reinterpret_cast<void**>(&p), (size_t)h->P * sizeof(float));
+        if (st != cudaSuccess) return h->cuda_fail(st, "fasgd_push_host: staging slot");
+        h->stage.push_back(p);
+        h->stage_busy.push_back(0);
+        slot = (int)h->stage.size() - 1;
+    }
+    cudaError_t st = cudaMemcpyAsync(h->stage[slot], grad_host, (size_t)h->P * sizeof(float),
+                                     cudaMemcpyDefault, h->stream);
+    if (st != cudaSuccess) return h->cuda_fail(st, "fasgd_push_host: copy");
+    h->stage_busy[slot] = 1;
+    h->fifo.push_back(Push{false, client, timestamp, h->stage[slot], nullptr, nullptr, nullptr, 0, slot});
+    return FASGD_OK;
+}
+
+int fasgd_push_sparse(fasgd_t* h, int32_t client, int64_t timestamp, const int32_t* idx,
+                      const float* val, const int64_t* n_dev, int64_t n_max) {
+    if (h == nullptr) return FASGD_EINVAL;
+    if (n_max < 0 || n_max > h->P) return h->fail(FASGD_EINVAL, "n_max must be in [0, P]");
+    if (n_max > 0 && (idx == nullptr || val == nullptr))
+        return h->fail(FASGD_EINVAL, "idx and val must be non-NULL");
+    if (!aligned(idx, 4) || !aligned(val, 4) || !aligned(n_dev, 8))
+        return h->fail(FASGD_EINVAL, "idx, val must be 4-byte and n_dev 8-byte aligned");
+    int rc = check_push(h, client, timestamp);
+    if (rc != FASGD_OK) return rc;
+    h->fifo.push_back(Push{true, client, timestamp, nullptr, idx, val, n_dev, n_max, -1});
+    return FASGD_OK;
+}
+
+int fasgd_apply_pending(fasgd_t* h, int32_t K) {
+    if (h == nullptr) return FASGD_EINVAL;
+    if (K < 1 || K > FASGD_KMAX) return h->fail(FASGD_EINVAL, "K must be in [1, %d]", FASGD_KMAX);
+    if ((int64_t)h->fifo.size() < K)
+        return h->fail(FASGD_EAGAIN, "K=%d but only %zu pushes pending", K, h->fifo.size());
+    DeviceGuard g(h->device);
+    const bool fas = h->variant == FASGD_FASGD;
+    const fasgd::StatParams sp = h->stat_params();
+    int k = 0;
+    while (k < K) {
+        const Push& first = h->fifo[(size_t)k];
+        if (!first.sparse) {
+            // Fuse the run of consecutive dense pushes into one pass.
+            fasgd::DenseArgs a;
+            std::memset(&a, 0, sizeof a);
+            a.theta = h->theta;
+            a.n = h->n;
+            a.b = h->b;
+            a.v = h->v;
+            a.P = h->P;
+            a.sp = sp;
+            int r = 0;
+            while (k + r < K && !h->fifo[(size_t)(k + r)].sparse) {
+                const Push& p = h->fifo[(size_t)(k + r)];
+                a.grad[r] = p.grad;
+                a.coef[r] = h->coef(h->T + k + r - p.j);
+                ++r;
+            }
+            a.K = r;
+            cudaError_t st = fasgd::launch_dense(a, fas, h->num_sms, h->stream, &h->launches);
+            if (st != cudaSuccess) return h->cuda_fail(st, "fasgd_apply_pending: dense pass");
+            k += r;
+        } else {
+            fasgd::SparseArgs a;
+            std::memset(&a, 0, sizeof a);
+            a.theta = h->theta;
+            a.n = h->n;
+            a.b = h->b;
+            a.v = h->v;
+            a.idx = first.idx;
+            a.val = first.val;
+            a.count_dev = first.n_dev;
+            a.count_max = first.n_max;
+            a.P = h->P;
+            a.coef = h->coef(h->T + k - first.j);
+            a.sp = sp;
+            a.err = h->dev_err;
+            if (first.n_max > 0 || first.n_dev != nullptr) {
+                cudaError_t st = fasgd::launch_sparse(a, fas, h->num_sms, h->stream, &h->launches);
+                if (st != cudaSuccess) return h->cuda_fail(st, "fasgd_apply_pending: sparse pass");
+            }
+            k += 1;
+        }
+    }
+    for (int i = 0; i < K; ++i) {
+        const int slot = h->fifo.front().stage;
+        if (slot >= 0) h->stage_busy[(size_t)slot] = 0;
+        h->fifo.pop_front();
+    }
+    h->T += K;
+    return FASGD_OK;
+}
+
+int bfasgd_select_compact(fasgd_t* h, int32_t client, const float* grad, const float* v,
+                          int32_t* idx, float* val, int64_t* n_dev) {
+    if (h == nullptr) return FASGD_EINVAL;
+    if (client < 0 || client >= h->lambda)
+        return h->fail(FASGD_ERANGE, "client %d outside [0, %d)", client, h->lambda);
+    if (grad == nullptr || !aligned(grad, 16))
+        return h->fail(FASGD_EINVAL, "grad must be a non-NULL 16-byte aligned device pointer");
+    if (v != nullptr && !aligned(v, 16))
+        return h->fail(FASGD_EINVAL, "v must be 16-byte aligned (or NULL for the server's v)");
+    if (idx == nullptr || val == nullptr || n_dev == nullptr || !aligned(idx, 4) ||
+        !aligned(val, 4) || !aligned(n_dev, 8))
+        return h->fail(FASGD_EINVAL, "idx, val, n_dev must be non-NULL and aligned");
+    DeviceGuard g(h->device);
+    fasgd::SelectArgs a;
+    std::memset(&a, 0, sizeof a);
+    a.grad = grad;
+    a.v = v != nullptr ? v : h->v;
+    a.idx = idx;
+    a.val = val;
+    a.count = n_dev;
+    a.mask = h->mask;
+    a.tile_count = h->tile_count;
+    a.tile_base = h->tile_base;
+    a.P = h->P;
+    a.ntiles = h->ntiles;
+    a.c = h->c_push;
+    a.eps_b = h->eps_b;
+    a.key0 = (uint32_t)h->seed;
+    a.key1 = (uint32_t)(h->seed >> 32);
+    const uint64_t push_no = h->push_count[(size_t)client];
+    a.client = (uint32_t)client;
+    a.push_lo = (uint32_t)push_no;
+    a.push_hi = (uint32_t)(push_no >> 32);
+    cudaError_t st = fasgd::launch_select(a, h->stream, &h->launches);
+    if (st != cudaSuccess) return h->cuda_fail(st, "bfasgd_select_compact");
+    h->push_count[(size_t)client] = push_no + 1;
+    return FASGD_OK;
+}
+
+int fasgd_pull(fasgd_t* h, float* params, int64_t* T) {
+    if (h == nullptr) return FASGD_EINVAL;
+    if (params != nullptr) {
+        DeviceGuard g(h->device);
+        cudaError_t st = cudaMemcpyAsync(params, h->theta, (size_t)h->P * sizeof(float),
+                                         cudaMemcpyDefault, h->stream);
+        if (st != cudaSuccess) return h->cuda_fail(st, "fasgd_pull");
+    }
+    if (T != nullptr) *T = h->T;
+    return FASGD_OK;
+}
+
+int fasgd_get_state(fasgd_t* h, float* theta, float* n, float* b, float* v, int64_t* T) {
+    if (h == nullptr) return FASGD_EINVAL;
+    if (!h->fifo.empty()) return h->fail(FASGD_EAGAIN, "pushes are pending");
+    DeviceGuard g(h->device);
+    float* dst[] = {theta, n, b, v};
+    const float* src[] = {h->theta, h->n, h->b, h->v};
+    for (int i = 0; i < 4; ++i) {
+        if (dst[i] == nullptr) continue;
+        cudaError_t st = cudaMemcpyAsync(dst[i], src[i], (size_t)h->P * sizeof(float),
+                                         cudaMemcpyDefault, h->stream);
+        if (st != cudaSuccess) return h->cuda_fail(st, "fasgd_get_state");
+    }
+    cudaError_t st = cudaStreamSynchronize(h->stream);
+    if (st != cudaSuccess) return h->cuda_fail(st, "fasgd_get_state");
+    if (T != nullptr) *T = h->T;
+    return FASGD_OK;
+}
+
+int fasgd_set_state(fasgd_t* h, const float* theta, const float* n, const float* b,
+                    const float* v, int64_t T) {
+    if (h == nullptr) return FASGD_EINVAL;
+    if (T < 0) return h->fail(FASGD_EINVAL, "T must be >= 0");
+    if (!h->fifo.empty()) return h->fail(FASGD_EAGAIN, "pushes are pending");
+    DeviceGuard g(h->device);
+    float* dst[] = {h->theta, h->n, h->b, h->v};
+    const float* src[] = {theta, n, b, v};
+    for (int i = 0; i < 4; ++i) {
+        if (src[i] == nullptr) continue;
+        cudaError_t st = cudaMemcpyAsync(dst[i], src[i], (size_t)h->P * sizeof(float),
+                                         cudaMemcpyDefault, h->stream);
+        if (st != cudaSuccess) return h->cuda_fail(st, "fasgd_set_state");
+    }
+    h->T = T;
+    return FASGD_OK;
+}
+
+int fasgd_get_push_counts(fasgd_t* h, uint64_t* counts) {
+    if (h == nullptr || counts == nullptr) return FASGD_EINVAL;
+    std::memcpy(counts, h->push_count.data(), h->push_count.size() * sizeof(uint64_t));
+    return FASGD_OK;
+}
+
+int fasgd_set_push_counts(fasgd_t* h, const uint64_t* counts) {
+    if (h == nullptr || counts == nullptr) return FASGD_EINVAL;
+    std::memcpy(h->push_count.data(), counts, h->push_count.size() * sizeof(uint64_t));
+    return FASGD_OK;
+}
+
+int fasgd_sync(fasgd_t* h) {
+    if (h == nullptr) return FASGD_EINVAL;
+    DeviceGuard g(h->device);
+    cudaError_t st = cudaStreamSynchronize(h->stream);
+    if (st != cudaSuccess) return h->cuda_fail(st, "fasgd_sync");
+    int32_t flags = 0;
+    st = cudaMemcpy(&flags, h->dev_err, sizeof flags, cudaMemcpyDeviceToHost);
+    if (st != cudaSuccess) return h->cuda_fail(st, "fasgd_sync");
+    if (flags != 0) {
+        st = cudaMemset(h->dev_err, 0, sizeof(int32_t));
+        if (st == cudaSuccess) st = cudaDeviceSynchronize();
+        if (st != cudaSuccess) return h->cuda_fail(st, "fasgd_sync");
+        return h->fail(FASGD_EDEVICE, "sparse list error flags 0x%x (1: count > n_max, "
+                                      "2: index out of range, 4: indices not ascending)", flags);
+    }
+    return FASGD_OK;
+}
+
+int64_t fasgd_timestamp(const fasgd_t* h) { return h == nullptr ? -1 : h->T; }
+
+int64_t fasgd_pending(const fasgd_t* h) { return h == nullptr ? -1 : (int64_t)h->fifo.size(); }
+
+int64_t fasgd_kernel_launches(const fasgd_t* h) { return h == nullptr ? -1 : h->launches; }
+
+const char* fasgd_last_error(const fasgd_t* h) {
+    return h == nullptr ? g_create_error.c_str() : h->err.c_str();
+}
+
+}  // extern "C"

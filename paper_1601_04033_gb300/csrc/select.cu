@@ -1,0 +1,228 @@
+// B-FASGD push side, per parameter (paper Sec. 2.3, Eq. 9): the send
+// decision and the compaction of the sent entries into an ascending index
+// list and the matching values.
+//
+// Three kernels, all on the caller's stream:
+//   1. mask:    per tile of 8192 parameters, draw u_p (Philox4x32-10), take
+//               the Eq. 9 decision against v_p, write one bit per parameter
+//               and the tile's count of sent entries;
+//   2. scan:    exclusive prefix sum of the tile counts (one block) and the
+//               total m;
+//   3. compact: per tile, rebuild each parameter's rank among the sent ones
+//               from the bit mask (warp popc + shuffles, block scan over
+//               warps) and write idx[rank] = p, val[rank] = grad[p].
+// The order of the output is the order of p, so the result is unique and
+// does not depend on the launch; no atomics are used.  Traffic per
+// parameter: v (4 B) + grad (4 B, skipped where a whole quad is dropped) +
+// 2 x 1/8 B of mask, plus 8 B per sent entry.
+
+#include "kernels.cuh"
+
+namespace fasgd {
+namespace {
+
+constexpr int kWarps = kSelectThreads / 32;
+constexpr int kWarpSpan = kSelectTile / kWarps;  // 1024 parameters per warp
+constexpr int kIters = kWarpSpan / 128;          // 8 passes of 32 lanes x 4
+constexpr unsigned kFull = 0xffffffffu;
+
+// Philox4x32-10 (Salmon, Moraes, Dror, Shaw, SC'11): ten rounds of two
+// 32x32->64 multiplies on a 128-bit counter, the 64-bit key advanced by the
+// golden-ratio Weyl increments between rounds.
+struct Philox4 {
+    uint32_t x[4];
+};
+
+__device__ __forceinline__ Philox4 philox4x32_10(uint32_t c0, uint32_t c1, uint32_t c2,
+                                                 uint32_t c3, uint32_t k0, uint32_t k1) {
+#pragma unroll
+    for (int r = 0; r < 10; ++r) {
+        const uint32_t lo0 = 0xD2511F53u * c0;
+        const uint32_t hi0 = __umulhi(0xD2511F53u, c0);
+        const uint32_t lo1 = 0xCD9E8D57u * c2;
+        const uint32_t hi1 = __umulhi(0xCD9E8D57u, c2);
+        const uint32_t n0 = hi1 ^ c1 ^ k0;
+        const uint32_t n2 = hi0 ^ c3 ^ k1;
+        c0 = n0;
+        c1 = lo1;
+        c2 = n2;
+        c3 = lo0;
+        k0 += 0x9E3779B9u;
+        k1 += 0xBB67AE85u;
+    }
+    Philox4 o;
+    o.x[0] = c0;
+    o.x[1] = c1;
+    o.x[2] = c2;
+    o.x[3] = c3;
+    return o;
+}
+
+// Eq. 9 for one parameter: send iff u / 2^24 < 1 / (1 + c / a), a = fl(v + eps_b),
+// evaluated exactly as u * fl(a + c) < a * 2^24 with the product split into
+// its rounded value and its exact error.
+__device__ __forceinline__ uint32_t send_bit(uint32_t u, float v, float c, float eps_b) {
+    const float a = __fadd_rn(v, eps_b);
+    const float d = __fadd_rn(a, c);
+    const float uf = (float)u;  // exact: u < 2^24
+    const float prod = __fmul_rn(uf, d);
+    const float err = __fmaf_rn(uf, d, -prod);
+    const float A = __fmul_rn(a, 16777216.0f);
+    return (prod < A || (prod == A && err < 0.0f)) ? 1u : 0u;
+}
+
+__global__ void __launch_bounds__(kSelectThreads) bfasgd_mask_kernel(const __grid_constant__ SelectArgs a) {
+    __shared__ int32_t warp_cnt[kWarps];
+    const int lane = threadIdx.x & 31;
+    const int warp = threadIdx.x >> 5;
+    const int64_t tile_start = (int64_t)blockIdx.x * kSelectTile;
+    const int64_t warp_start = tile_start + (int64_t)warp * kWarpSpan;
+    int cnt = 0;
+#pragma unroll 2
+    for (int it = 0; it < kIters; ++it) {
+        const int64_t e = warp_start + it * 128 + 4 * lane;  // first parameter of this quad
+        uint32_t nib = 0;
+        if (e < a.P) {
+            const Philox4 r = philox4x32_10((uint32_t)(e >> 2), a.client, a.push_lo, a.push_hi,
+                                            a.key0, a.key1);
+            if (e + 3 < a.P) {
+                const float4 v4 = __ldcs(reinterpret_cast<const float4*>(a.v + e));
+                nib = send_bit(r.x[0] >> 8, v4.x, a.c, a.eps_b) |
+                      (send_bit(r.x[1] >> 8, v4.y, a.c, a.eps_b) << 1) |
+                      (send_bit(r.x[2] >> 8, v4.z, a.c, a.eps_b) << 2) |
+                      (send_bit(r.x[3] >> 8, v4.w, a.c, a.eps_b) << 3);
+            } else {
+                for (int j = 0; j < 4; ++j)
+                    if (e + j < a.P) nib |= send_bit(r.x[j] >> 8, a.v[e + j], a.c, a.eps_b) << j;
+            }
+        }
+        cnt += __popc(nib);
+        // Eight lanes' nibbles form one 32-bit mask word (32 consecutive parameters).
+        uint32_t w = nib << (4 * (lane & 7));
+        w |= __shfl_xor_sync(kFull, w, 1);
+        w |= __shfl_xor_sync(kFull, w, 2);
+        w |= __shfl_xor_sync(kFull, w, 4);
+        if ((lane & 7) == 0)
+            a.mask[(warp_start >> 5) + it * 4 + (lane >> 3)] = w;
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) cnt += __shfl_xor_sync(kFull, cnt, off);
+    if (lane == 0) warp_cnt[warp] = cnt;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        int32_t t = 0;
+#pragma unroll
+        for (int w = 0; w < kWarps; ++w) t += warp_cnt[w];
+        a.tile_count[blockIdx.x] = t;
+    }
+}
+
+constexpr int kScanThreads = 1024;
+
+__global__ void __launch_bounds__(kScanThreads) bfasgd_scan_kernel(const __grid_constant__ SelectArgs a) {
+    __shared__ int64_t warp_sum[kScanThreads / 32];
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int per = (a.ntiles + kScanThreads - 1) / kScanThreads;
+    const int lo = tid * per;
+    const int hi = min(lo + per, a.ntiles);
+    int64_t local = 0;
+    for (int t = lo; t < hi; ++t) local += a.tile_count[t];
+    // Inclusive scan of the per-thread sums across the block.
+    int64_t incl = local;
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+        const int64_t y = __shfl_up_sync(kFull, incl, off);
+        if (lane >= off) incl += y;
+    }
+    if (lane == 31) warp_sum[warp] = incl;
+    __syncthreads();
+    if (warp == 0) {
+        int64_t s = warp_sum[lane];
+#pragma unroll
+        for (int off = 1; off < 32; off <<= 1) {
+            const int64_t y = __shfl_up_sync(kFull, s, off);
+            if (lane >= off) s += y;
+        }
+        warp_sum[lane] = s;  // inclusive over warps
+    }
+    __syncthreads();
+    int64_t run = incl - local + (warp > 0 ? warp_sum[warp - 1] : 0);  // exclusive prefix
+    for (int t = lo; t < hi; ++t) {
+        a.tile_base[t] = run;
+        run += a.tile_count[t];
+    }
+    if (tid == kScanThreads - 1) *a.count = warp_sum[kScanThreads / 32 - 1];
+}
+
+__global__ void __launch_bounds__(kSelectThreads) bfasgd_compact_kernel(const __grid_constant__ SelectArgs a) {
+    __shared__ int32_t warp_cnt[kWarps];
+    const int lane = threadIdx.x & 31;
+    const int warp = threadIdx.x >> 5;
+    const int64_t tile_start = (int64_t)blockIdx.x * kSelectTile;
+    const int64_t warp_start = tile_start + (int64_t)warp * kWarpSpan;
+    // Lane l holds the mask word of parameters warp_start + 32 l .. + 31.
+    const uint32_t word = a.mask[(warp_start >> 5) + lane];
+    const int c = __popc(word);
+    int incl = c;
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+        const int y = __shfl_up_sync(kFull, incl, off);
+        if (lane >= off) incl += y;
+    }
+    const int excl = incl - c;
+    if (lane == 31) warp_cnt[warp] = incl;
+    __syncthreads();
+    int64_t out = a.tile_base[blockIdx.x];
+    for (int w = 0; w < warp; ++w) out += warp_cnt[w];
+#pragma unroll 2
+    for (int it = 0; it < kIters; ++it) {
+        // This lane's quad lies in word (4 it + lane / 8), bits 4 (lane mod 8) .. +3.
+        const int owner = it * 4 + (lane >> 3);
+        const uint32_t w = __shfl_sync(kFull, word, owner);
+        const int wbase = __shfl_sync(kFull, excl, owner);
+        const int sh = 4 * (lane & 7);
+        const uint32_t nib = (w >> sh) & 0xFu;
+        if (nib != 0) {
+            const int64_t e = warp_start + it * 128 + 4 * lane;
+            float g[4];
+            if (e + 3 < a.P) {
+                const float4 g4 = __ldcs(reinterpret_cast<const float4*>(a.grad + e));
+                g[0] = g4.x;
+                g[1] = g4.y;
+                g[2] = g4.z;
+                g[3] = g4.w;
+            } else {
+                for (int j = 0; j < 4; ++j) g[j] = (e + j < a.P) ? a.grad[e + j] : 0.0f;
+            }
+            int64_t pos = out + wbase + __popc(w & ((1u << sh) - 1u));
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                if ((nib >> j) & 1u) {
+                    a.idx[pos] = (int32_t)(e + j);
+                    a.val[pos] = g[j];
+                    ++pos;
+                }
+            }
+        }
+    }
+}
+
+}  // namespace
+
+cudaError_t launch_select(const SelectArgs& a, cudaStream_t stream, int64_t* launches) {
+    bfasgd_mask_kernel<<<a.ntiles, kSelectThreads, 0, stream>>>(a);
+    cudaError_t st = cudaGetLastError();
+    if (st != cudaSuccess) return st;
+    ++*launches;
+    bfasgd_scan_kernel<<<1, kScanThreads, 0, stream>>>(a);
+    st = cudaGetLastError();
+    if (st != cudaSuccess) return st;
+    ++*launches;
+    bfasgd_compact_kernel<<<a.ntiles, kSelectThreads, 0, stream>>>(a);
+    st = cudaGetLastError();
+    if (st != cudaSuccess) return st;
+    ++*launches;
+    return cudaSuccess;
+}
+
+}  // namespace fasgd

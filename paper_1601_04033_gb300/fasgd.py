@@ -1,0 +1,279 @@
+"""ctypes binding of include/fasgd.h (argument marshalling only).
+
+Every function here forwards to the entry point of the same name in
+libfasgd.so; all computation happens in the library's CUDA kernels.  The
+library must have been built (``paper_1601_04033_gb300.build.build()`` or
+``__graft_entry__.build()``); if it is missing, importing this module
+raises -- there is no fallback.
+
+``Server`` is a thin convenience wrapper over a handle that accepts torch
+tensors (CUDA tensors for device arguments) and the current torch stream.
+"""
+
+from __future__ import annotations
+
+import ctypes
+import os
+
+from . import build as _build
+
+ASGD, SASGD, FASGD = 0, 1, 2
+OK, EINVAL, ERANGE, EAGAIN, ENOMEM, ECUDA, EDEVICE = 0, -1, -2, -3, -4, -5, -6
+KMAX = 32
+STATUS_NAMES = {OK: "OK", EINVAL: "EINVAL", ERANGE: "ERANGE", EAGAIN: "EAGAIN",
+                ENOMEM: "ENOMEM", ECUDA: "ECUDA", EDEVICE: "EDEVICE"}
+
+_p = ctypes.c_void_p
+_i32, _i64, _u64, _f32 = ctypes.c_int32, ctypes.c_int64, ctypes.c_uint64, ctypes.c_float
+
+# name -> (restype, argtypes); the list mirrors include/fasgd.h one to one.
+SIGNATURES = {
+    "fasgd_create": (_i32, [ctypes.POINTER(_p), _i64, _i32, _f32, _i32]),
+    "fasgd_destroy": (None, [_p]),
+    "fasgd_set_hparams": (_i32, [_p, _f32, _f32, _f32, _f32, _f32, _u64]),
+    "fasgd_set_stream": (_i32, [_p, _p]),
+    "fasgd_set_params": (_i32, [_p, _p]),
+    "fasgd_push": (_i32, [_p, _i32, _i64, _p]),
+    "fasgd_push_host": (_i32, [_p, _i32, _i64, _p]),
+    "fasgd_push_sparse": (_i32, [_p, _i32, _i64, _p, _p, _p, _i64]),
+    "fasgd_apply_pending": (_i32, [_p, _i32]),
+    "bfasgd_select_compact": (_i32, [_p, _i32, _p, _p, _p, _p, _p]),
+    "fasgd_pull": (_i32, [_p, _p, ctypes.POINTER(_i64)]),
+    "fasgd_get_state": (_i32, [_p, _p, _p, _p, _p, ctypes.POINTER(_i64)]),
+    "fasgd_set_state": (_i32, [_p, _p, _p, _p, _p, _i64]),
+    "fasgd_get_push_counts": (_i32, [_p, _p]),
+    "fasgd_set_push_counts": (_i32, [_p, _p]),
+    "fasgd_sync": (_i32, [_p]),
+    "fasgd_timestamp": (_i64, [_p]),
+    "fasgd_pending": (_i64, [_p]),
+    "fasgd_kernel_launches": (_i64, [_p]),
+    "fasgd_last_error": (ctypes.c_char_p, [_p]),
+}
+
+
+def _load() -> ctypes.CDLL:
+    path = _build.LIB
+    if not os.path.exists(path):
+        raise ImportError(f"{path} is missing: build the CUDA library first "
+                          "(python -c 'import __graft_entry__ as g; g.build()')")
+    lib = ctypes.CDLL(path)
+    for name, (res, args) in SIGNATURES.items():
+        fn = getattr(lib, name)
+        fn.restype = res
+        fn.argtypes = args
+    return lib
+
+
+LIB = _load()
+LIB_PATH = _build.LIB
+
+
+class FasgdError(RuntimeError):
+    def __init__(self, code: int, msg: str):
+        super().__init__(f"{STATUS_NAMES.get(code, code)}: {msg}")
+        self.code = code
+
+
+# ---------------------------------------------------------------------------
+# Raw entry points, same names and arguments as the C ABI (pointers as ints).
+# ---------------------------------------------------------------------------
+def fasgd_create(P: int, lam: int, alpha: float, variant: int):
+    h = _p()
+    rc = LIB.fasgd_create(ctypes.byref(h), P, lam, alpha, variant)
+    return rc, h.value
+
+
+def fasgd_destroy(h):
+    LIB.fasgd_destroy(h)
+
+
+def fasgd_set_hparams(h, gamma, beta, eps, c_push, eps_b, seed):
+    return LIB.fasgd_set_hparams(h, gamma, beta, eps, c_push, eps_b, seed)
+
+
+def fasgd_set_stream(h, stream):
+    return LIB.fasgd_set_stream(h, stream)
+
+
+def fasgd_set_params(h, theta0):
+    return LIB.fasgd_set_params(h, theta0)
+
+
+def fasgd_push(h, client, timestamp, grad):
+    return LIB.fasgd_push(h, client, timestamp, grad)
+
+
+def fasgd_push_host(h, client, timestamp, grad_host):
+    return LIB.fasgd_push_host(h, client, timestamp, grad_host)
+
+
+def fasgd_push_sparse(h, client, timestamp, idx, val, n_dev, n_max):
+    return LIB.fasgd_push_sparse(h, client, timestamp, idx, val, n_dev, n_max)
+
+
+def fasgd_apply_pending(h, K):
+    return LIB.fasgd_apply_pending(h, K)
+
+
+def bfasgd_select_compact(h, client, grad, v, idx, val, n_dev):
+    return LIB.bfasgd_select_compact(h, client, grad, v, idx, val, n_dev)
+
+
+def fasgd_pull(h, params):
+    T = _i64()
+    rc = LIB.fasgd_pull(h, params, ctypes.byref(T))
+    return rc, T.value
+
+
+def fasgd_get_state(h, theta, n, b, v):
+    T = _i64()
+    rc = LIB.fasgd_get_state(h, theta, n, b, v, ctypes.byref(T))
+    return rc, T.value
+
+
+def fasgd_set_state(h, theta, n, b, v, T):
+    return LIB.fasgd_set_state(h, theta, n, b, v, T)
+
+
+def fasgd_get_push_counts(h, counts):
+    return LIB.fasgd_get_push_counts(h, counts)
+
+
+def fasgd_set_push_counts(h, counts):
+    return LIB.fasgd_set_push_counts(h, counts)
+
+
+def fasgd_sync(h):
+    return LIB.fasgd_sync(h)
+
+
+def fasgd_timestamp(h):
+    return LIB.fasgd_timestamp(h)
+
+
+def fasgd_pending(h):
+    return LIB.fasgd_pending(h)
+
+
+def fasgd_kernel_launches(h):
+    return LIB.fasgd_kernel_launches(h)
+
+
+def fasgd_last_error(h) -> str:
+    s = LIB.fasgd_last_error(h)
+    return s.decode() if s else ""
+
+
+# ---------------------------------------------------------------------------
+# Tensor-level wrapper
+# ---------------------------------------------------------------------------
+def _ptr(t) -> int | None:
+    if t is None:
+        return None
+    if not t.is_contiguous():
+        raise ValueError("tensor must be contiguous")
+    return t.data_ptr()
+
+
+class Server:
+    """One FASGD parameter server on the current CUDA device.
+
+    Device arguments are torch CUDA tensors (fp32 / int32 / int64); the
+    handle runs on torch's current stream at construction time unless a
+    stream is given.
+    """
+
+    def __init__(self, P: int, lam: int, alpha: float, variant: int = FASGD, *,
+                 gamma: float = 0.95, beta: float = 0.95, eps: float = 1e-4,
+                 c_push: float = 0.0, eps_b: float = 1e-8, seed: int = 0, stream=None):
+        import torch
+        rc, h = fasgd_create(P, lam, alpha, variant)
+        if rc != OK:
+            raise FasgdError(rc, fasgd_last_error(None))
+        self.h = h
+        self.P, self.lam, self.variant = P, lam, variant
+        self._check(fasgd_set_hparams(h, gamma, beta, eps, c_push, eps_b, seed))
+        s = stream if stream is not None else torch.cuda.current_stream()
+        self.stream = s
+        self._check(fasgd_set_stream(h, s.cuda_stream))
+
+    def _check(self, rc):
+        if rc != OK:
+            raise FasgdError(rc, fasgd_last_error(self.h))
+        return rc
+
+    def close(self):
+        if getattr(self, "h", None):
+            fasgd_destroy(self.h)
+            self.h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    # -- calls ---------------------------------------------------------------
+    def set_hparams(self, gamma, beta, eps, c_push, eps_b, seed):
+        self._check(fasgd_set_hparams(self.h, gamma, beta, eps, c_push, eps_b, seed))
+
+    def set_params(self, theta0):
+        self._check(fasgd_set_params(self.h, _ptr(theta0)))
+
+    def push(self, client: int, timestamp: int, grad):
+        self._check(fasgd_push(self.h, client, timestamp, _ptr(grad)))
+
+    def push_host(self, client: int, timestamp: int, grad_host):
+        self._check(fasgd_push_host(self.h, client, timestamp, _ptr(grad_host)))
+
+    def push_sparse(self, client: int, timestamp: int, idx, val, n_dev=None, n_max=None):
+        if n_max is None:
+            n_max = idx.numel()
+        self._check(fasgd_push_sparse(self.h, client, timestamp, _ptr(idx), _ptr(val),
+                                      _ptr(n_dev), n_max))
+
+    def apply_pending(self, K: int):
+        self._check(fasgd_apply_pending(self.h, K))
+
+    def select_compact(self, client: int, grad, idx, val, n_dev, v=None):
+        self._check(bfasgd_select_compact(self.h, client, _ptr(grad), _ptr(v), _ptr(idx),
+                                          _ptr(val), _ptr(n_dev)))
+
+    def pull(self, params=None) -> int:
+        rc, T = fasgd_pull(self.h, _ptr(params))
+        self._check(rc)
+        return T
+
+    def get_state(self, theta=None, n=None, b=None, v=None) -> int:
+        rc, T = fasgd_get_state(self.h, _ptr(theta), _ptr(n), _ptr(b), _ptr(v))
+        self._check(rc)
+        return T
+
+    def set_state(self, theta, n, b, v, T: int):
+        self._check(fasgd_set_state(self.h, _ptr(theta), _ptr(n), _ptr(b), _ptr(v), T))
+
+    def push_counts(self):
+        import numpy as np
+        out = np.zeros(self.lam, dtype=np.uint64)
+        self._check(fasgd_get_push_counts(self.h, out.ctypes.data))
+        return out
+
+    def set_push_counts(self, counts):
+        import numpy as np
+        c = np.ascontiguousarray(counts, dtype=np.uint64)
+        self._check(fasgd_set_push_counts(self.h, c.ctypes.data))
+
+    def sync(self):
+        self._check(fasgd_sync(self.h))
+
+    @property
+    def T(self) -> int:
+        return fasgd_timestamp(self.h)
+
+    @property
+    def pending(self) -> int:
+        return fasgd_pending(self.h)
+
+    @property
+    def launches(self) -> int:
+        return fasgd_kernel_launches(self.h)

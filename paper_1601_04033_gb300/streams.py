@@ -105,14 +105,20 @@ def pool_slot(w: Workload, r: int, m: np.ndarray, s: np.ndarray) -> np.ndarray:
     return z
 
 
-def gradient_pool(w: Workload, P: int | None = None, R: int | None = None) -> np.ndarray:
-    """All R pool slots as one fp32[R, P] array."""
+def gradient_pool(w: Workload, P: int | None = None, R: int | None = None,
+                  threads: int = 16) -> np.ndarray:
+    """All R pool slots as one fp32[R, P] array (slots drawn in parallel)."""
+    import concurrent.futures
     P = w.P if P is None else P
     R = w.R if R is None else R
     m, s = grad_model(w, P)
     out = np.empty((R, P), dtype=np.float32)
-    for r in range(R):
+
+    def fill(r):
         out[r] = pool_slot(w, r, m, s)
+
+    with concurrent.futures.ThreadPoolExecutor(max_workers=max(1, min(threads, R))) as ex:
+        list(ex.map(fill, range(R)))
     return out
 
 
@@ -199,3 +205,18 @@ def sample_indices(P: int, count: int, seed: int = 12345) -> np.ndarray:
     edge = np.array([0, 1, 2, 3, P - 4, P - 3, P - 2, P - 1], dtype=np.int64)
     edge = edge[(edge >= 0) & (edge < P)]
     return np.unique(np.concatenate([pick.astype(np.int64), edge]))
+
+
+_TAG_VSNAP = 6
+
+
+def client_v_snapshot(w: Workload, client: int, P: int | None = None,
+                      lo: float = 1.0, hi: float = 100.0) -> np.ndarray:
+    """A client's copy of the server statistic v (fp32[P], log-uniform[lo, hi]).
+
+    B-FASGD clients decide with the v they last fetched from the server; a
+    drawn snapshot stands in for it where both sides of a comparison must
+    decide on identical inputs."""
+    P = w.P if P is None else P
+    u = _rng(w.seed, _TAG_VSNAP, client).uniform(math.log(lo), math.log(hi), P)
+    return np.exp(u).astype(np.float32)

@@ -1,0 +1,133 @@
+"""Helpers shared by the GPU parity tests: drive the CUDA path (through the
+C ABI binding) and the CPU oracle on the same seeded stream, and compare."""
+
+from __future__ import annotations
+
+import math
+
+import numpy as np
+
+import oracle
+from paper_1601_04033_gb300 import streams
+
+# Tolerance for fp32 parameters and statistics against the oracle, per
+# element: |gpu - oracle| <= RTOL * |oracle| + ATOL.
+RTOL = 1e-5
+ATOL = 1e-7
+
+HP = dict(gamma=0.95, beta=0.95, eps=1e-4, eps_b=1e-8)
+
+
+def torch_cuda():
+    import torch
+    return torch
+
+
+def binding():
+    from paper_1601_04033_gb300 import fasgd
+    return fasgd
+
+
+def assert_close(gpu, ora, what):
+    gpu = np.asarray(gpu, dtype=np.float64)
+    ora = np.asarray(ora, dtype=np.float64)
+    d = np.abs(gpu - ora)
+    bound = RTOL * np.abs(ora) + ATOL
+    bad = np.nonzero(~(d <= bound))[0]
+    if bad.size:
+        i = bad[np.argmax((d[bad] - bound[bad]))]
+        raise AssertionError(f"{what}: {bad.size} of {gpu.size} outside tolerance; worst at {i}: "
+                             f"gpu={gpu[i]!r} oracle={ora[i]!r} |d|={d[i]:.3e} bound={bound[i]:.3e}")
+
+
+def assert_bitwise(gpu, ora, what):
+    g = np.ascontiguousarray(gpu)
+    o = np.ascontiguousarray(ora)
+    assert g.dtype == o.dtype and g.shape == o.shape, (what, g.dtype, o.dtype, g.shape, o.shape)
+    if g.dtype == np.float32:
+        g, o = g.view(np.uint32), o.view(np.uint32)
+    bad = np.nonzero(g != o)[0]
+    assert bad.size == 0, f"{what}: {bad.size} elements differ, first at {bad[:5]}"
+
+
+class GpuRun:
+    """A CUDA-path server fed from a device-resident gradient pool."""
+
+    def __init__(self, w: streams.Workload, variant: int, P: int, pool: np.ndarray,
+                 theta0: np.ndarray, **hp):
+        torch = torch_cuda()
+        f = binding()
+        h = dict(HP)
+        h.update(hp)
+        self.srv = f.Server(P, w.lam, w.alpha, variant, gamma=h["gamma"], beta=h["beta"],
+                            eps=h["eps"], c_push=h.get("c_push", 0.0), eps_b=h["eps_b"],
+                            seed=h.get("seed", 0))
+        self.P = P
+        self.pool = torch.from_numpy(pool).cuda()
+        self.srv.set_params(torch.from_numpy(theta0).cuda())
+
+    def push_batch(self, clients, js, slots):
+        for c, j, s in zip(clients, js, slots):
+            self.srv.push(int(c), int(j), self.pool[int(s)])
+        self.srv.apply_pending(len(clients))
+
+    def state(self):
+        torch = torch_cuda()
+        out = [torch.empty(self.P, dtype=torch.float32, device="cuda") for _ in range(4)]
+        T = self.srv.get_state(*out)
+        return [x.cpu().numpy() for x in out] + [T]
+
+
+class OracleRun:
+    def __init__(self, w: streams.Workload, variant: int, P: int, pool: np.ndarray,
+                 theta0: np.ndarray, real: str = "f32", **hp):
+        h = dict(HP)
+        h.update(hp)
+        self.srv = oracle.OracleServer(P, w.lam, w.alpha, variant, real=real,
+                                       gamma=h["gamma"], beta=h["beta"], eps=h["eps"],
+                                       c_push=h.get("c_push", 0.0), eps_b=h["eps_b"],
+                                       seed=h.get("seed", 0))
+        self.srv.set_params(theta0)
+        self.pool = pool
+
+    def push_batch(self, clients, js, slots):
+        for c, j, s in zip(clients, js, slots):
+            self.srv.push(int(c), int(j), self.pool[int(s)])
+        self.srv.apply_pending(len(clients))
+
+    def state(self):
+        return list(self.srv.state())
+
+
+def compare_states(gs, os_, variant, where):
+    names = ("theta", "n", "b", "v")
+    assert gs[4] == os_[4], f"{where}: timestamps differ {gs[4]} vs {os_[4]}"
+    if variant != oracle.FASGD:
+        assert_bitwise(gs[0], os_[0].astype(np.float32), f"{where} theta")
+        return
+    # n and b are formed with the same once-rounded fp32 sequence on both sides.
+    assert_bitwise(gs[1], os_[1].astype(np.float32), f"{where} n")
+    assert_bitwise(gs[2], os_[2].astype(np.float32), f"{where} b")
+    for k in (0, 3):
+        assert_close(gs[k], os_[k], f"{where} {names[k]}")
+
+
+def run_parity(w, variant, P, n_pushes, K, check_every=None, real="f32", **hp):
+    """Run GPU and oracle in lockstep; compare at every T multiple of lcm(100, K)."""
+    check_every = check_every or (100 * K // math.gcd(100, K))
+    pool = streams.gradient_pool(w, P)
+    th0 = streams.theta0(w, P)
+    ps = streams.push_stream(w, n_pushes, K)
+    g = GpuRun(w, variant, P, pool, th0, **hp)
+    o = OracleRun(w, variant, P, pool, th0, real=real, **hp)
+    checks = 0
+    for b in range(n_pushes // K):
+        cl, js, sl = ps.batch(b)
+        g.push_batch(cl, js, sl)
+        o.push_batch(cl, js, sl)
+        T = (b + 1) * K
+        if T % check_every == 0:
+            compare_states(g.state(), o.state(), variant, f"{w.name} var={variant} P={P} K={K} T={T}")
+            checks += 1
+    assert checks > 0
+    return g, o

@@ -1,0 +1,115 @@
+"""Error codes of the C ABI with a live handle; a failed call changes nothing."""
+
+import numpy as np
+import pytest
+
+import oracle
+from gpu_util import GpuRun, assert_bitwise
+from paper_1601_04033_gb300 import streams
+
+pytestmark = pytest.mark.gpu
+
+
+def _f():
+    from paper_1601_04033_gb300 import fasgd
+    return fasgd
+
+
+def _snapshot(srv, P):
+    import torch
+    out = [torch.empty(P, device="cuda") for _ in range(4)]
+    T = srv.get_state(*out) if srv.pending == 0 else None
+    return [x.cpu().numpy() for x in out], T, srv.pending
+
+
+def test_error_codes_leave_state_unchanged():
+    import torch
+    f = _f()
+    P = 1001
+    srv = f.Server(P, 4, 0.01, f.FASGD)
+    srv.set_params(torch.linspace(-1, 1, P, device="cuda"))
+    g = torch.ones(P + 8, device="cuda")
+    srv.push(0, 0, g)
+    srv.apply_pending(1)
+    h = srv.h
+    before, T0, _ = _snapshot(srv, P)
+    checks = [
+        (f.ERANGE, lambda: f.fasgd_push(h, 4, 0, g.data_ptr())),            # client == lambda
+        (f.ERANGE, lambda: f.fasgd_push(h, -1, 0, g.data_ptr())),
+        (f.ERANGE, lambda: f.fasgd_push(h, 0, T0 + 1, g.data_ptr())),      # j > T
+        (f.ERANGE, lambda: f.fasgd_push(h, 0, -1, g.data_ptr())),
+        (f.EINVAL, lambda: f.fasgd_push(h, 0, 0, None)),                    # NULL
+        (f.EINVAL, lambda: f.fasgd_push(h, 0, 0, g.data_ptr() + 4)),        # misaligned
+        (f.EAGAIN, lambda: f.fasgd_apply_pending(h, 1)),                    # nothing pending
+        (f.EINVAL, lambda: f.fasgd_apply_pending(h, 0)),
+        (f.EINVAL, lambda: f.fasgd_apply_pending(h, f.KMAX + 1)),
+        (f.EINVAL, lambda: f.fasgd_set_hparams(h, 1.5, 0.9, 1e-4, 0, 0, 0)),
+        (f.EINVAL, lambda: f.fasgd_set_hparams(h, 0.9, 1.0, 1e-4, 0, 0, 0)),
+        (f.EINVAL, lambda: f.fasgd_set_hparams(h, 0.9, 0.9, -1.0, 0, 0, 0)),
+        (f.EINVAL, lambda: f.fasgd_set_hparams(h, 0.9, 0.9, 1e-4, -1.0, 0, 0)),
+        (f.EINVAL, lambda: f.fasgd_set_hparams(h, 0.9, 0.9, 1e-4, 0, float("nan"), 0)),
+        (f.EINVAL, lambda: f.fasgd_push_sparse(h, 0, 0, None, None, None, 5)),
+        (f.EINVAL, lambda: f.fasgd_push_sparse(h, 0, 0, g.data_ptr(), g.data_ptr(), None, P + 1)),
+        (f.EINVAL, lambda: f.fasgd_push_sparse(h, 0, 0, g.data_ptr() + 2, g.data_ptr(), None, 3)),
+        (f.ERANGE, lambda: f.bfasgd_select_compact(h, 9, g.data_ptr(), None, g.data_ptr(),
+                                                    g.data_ptr(), g.data_ptr())),
+        (f.EINVAL, lambda: f.bfasgd_select_compact(h, 0, g.data_ptr() + 4, None, g.data_ptr(),
+                                                    g.data_ptr(), g.data_ptr())),
+        (f.EINVAL, lambda: f.bfasgd_select_compact(h, 0, g.data_ptr(), None, None,
+                                                    g.data_ptr(), g.data_ptr())),
+        (f.EINVAL, lambda: f.fasgd_set_params(h, None)),
+        (f.EINVAL, lambda: f.fasgd_set_state(h, None, None, None, None, -1)),
+    ]
+    for want, call in checks:
+        rc = call()
+        assert rc == want, (rc, want, f.fasgd_last_error(h))
+        assert f.fasgd_last_error(h)
+        assert srv.T == T0 and srv.pending == 0
+    after, T1, _ = _snapshot(srv, P)
+    for x, y in zip(before, after):
+        assert_bitwise(x, y, "state after rejected calls")
+    assert list(srv.push_counts()) == [0, 0, 0, 0]
+    # Calls that need an empty queue refuse while pushes are pending.
+    srv.push(1, 1, g)
+    assert f.fasgd_set_stream(h, None) == f.EAGAIN
+    assert f.fasgd_set_params(h, g.data_ptr()) == f.EAGAIN
+    assert f.fasgd_get_state(h, None, None, None, None)[0] == f.EAGAIN
+    assert f.fasgd_set_hparams(h, 0.9, 0.9, 1e-4, 0, 0, 0) == f.EAGAIN
+    assert f.fasgd_apply_pending(h, 2) == f.EAGAIN and srv.pending == 1
+    srv.apply_pending(1)
+    srv.sync()
+    srv.close()
+    srv.close()
+
+
+def test_host_push_and_pull_match_device_path():
+    """fasgd_push_host (pinned host gradients, device staging) == fasgd_push."""
+    import torch
+    f = _f()
+    w = streams.WORKLOADS["fasgd-1.29m"]
+    P = 40_003
+    pool = streams.gradient_pool(w, P, 8)
+    th0 = streams.theta0(w, P)
+    ps = streams.push_stream(w.replace(R=8, K=4), 40, 4)
+    a = GpuRun(w, oracle.FASGD, P, pool, th0)
+    b = GpuRun(w, oracle.FASGD, P, pool, th0)
+    host_pool = torch.from_numpy(pool).pin_memory()
+    out = torch.empty(P, dtype=torch.float32).pin_memory()
+    for k in range(10):
+        cl, js, sl = ps.batch(k)
+        a.push_batch(cl, js, sl)
+        for c, j, s in zip(cl, js, sl):
+            b.srv.push_host(int(c), int(j), host_pool[int(s)])
+        b.srv.apply_pending(4)
+        T = b.srv.pull(out)
+        torch.cuda.current_stream().synchronize()
+        assert T == 4 * (k + 1)
+        assert_bitwise(out.numpy(), a.state()[0], f"pull after batch {k}")
+    # At most KMAX host pushes may wait for an apply.
+    for i in range(f.KMAX):
+        b.srv.push_host(0, b.srv.T, host_pool[i % 8])
+    with pytest.raises(f.FasgdError) as e:
+        b.srv.push_host(0, b.srv.T, host_pool[0])
+    assert e.value.code == f.EAGAIN
+    b.srv.apply_pending(f.KMAX)
+    b.srv.sync()

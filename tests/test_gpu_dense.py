@@ -1,0 +1,160 @@
+"""CUDA dense path (ASGD / SASGD / FASGD, fused K pass) against the oracle."""
+
+import numpy as np
+import pytest
+
+import oracle
+from gpu_util import (GpuRun, OracleRun, assert_bitwise, assert_close, compare_states,
+                      run_parity)
+from paper_1601_04033_gb300 import streams
+
+pytestmark = pytest.mark.gpu
+
+W = streams.WORKLOADS
+
+
+@pytest.mark.parametrize("variant", [oracle.ASGD, oracle.SASGD, oracle.FASGD])
+def test_workload_7850_full_stream(variant):
+    """P = 7,850 (784x10 shape), lambda = 4, 200 pushes, K = 1: the full stream."""
+    w = W["fasgd-7850"]
+    run_parity(w, variant, w.P, w.pushes, 1)
+
+
+@pytest.mark.parametrize("variant", [oracle.ASGD, oracle.SASGD, oracle.FASGD])
+def test_workload_1_29m_prefix(variant):
+    """P = 1,290,510 (ragged), lambda = 32, Poisson(4) staleness: 200-push prefix."""
+    w = W["fasgd-1.29m"]
+    run_parity(w, variant, w.P, 200, 1)
+
+
+def test_workload_25m_shape_fused_k8_small_p():
+    """The K = 8 fused pass with Geometric(0.05) staleness on P = 100,003."""
+    w = W["fasgd-25m-k8"]
+    run_parity(w, oracle.FASGD, 100_003, 400, 8)
+
+
+@pytest.mark.parametrize("K", [2, 3, 5, 13, 16, 32])
+def test_fused_k_values(K):
+    w = W["fasgd-25m-k8"].replace(R=max(2 * K, 16))
+    n = 100 * K // np.gcd(100, K)
+    run_parity(w, oracle.FASGD, 50_001, n, K)
+
+
+@pytest.mark.parametrize("variant", [oracle.ASGD, oracle.FASGD])
+def test_against_fp64_oracle(variant):
+    """The fp32 GPU state stays within the same bound of the fp64 oracle."""
+    w = W["fasgd-1.29m"]
+    P = 65_537
+    pool = streams.gradient_pool(w, P)
+    th0 = streams.theta0(w, P)
+    ps = streams.push_stream(w, 300, 1)
+    g = GpuRun(w, variant, P, pool, th0)
+    o = OracleRun(w, variant, P, pool, th0, real="f64")
+    for b in range(300):
+        cl, js, sl = ps.batch(b)
+        g.push_batch(cl, js, sl)
+        o.push_batch(cl, js, sl)
+        if (b + 1) % 100 == 0:
+            gs, os_ = g.state(), o.state()
+            names = ("theta", "n", "b", "v") if variant == oracle.FASGD else ("theta",)
+            for k, name in enumerate(names):
+                assert_close(gs[k], os_[k], f"fp64 T={b + 1} {name}")
+
+
+@pytest.mark.parametrize("P", [1, 2, 3, 4, 5, 7, 255, 1023, 1025, 4097])
+def test_tiny_and_ragged(P):
+    w = W["fasgd-7850"]
+    for variant in (oracle.ASGD, oracle.FASGD):
+        run_parity(w, variant, P, 100, 4, check_every=100)
+
+
+def test_fused_equals_sequential_bitwise():
+    """One K = 8 pass == eight K = 1 passes, bit for bit (same element sequence)."""
+    w = W["fasgd-25m-k8"]
+    P = 200_003
+    pool = streams.gradient_pool(w, P)
+    th0 = streams.theta0(w, P)
+    ps = streams.push_stream(w, 64, 8)
+    a = GpuRun(w, oracle.FASGD, P, pool, th0)
+    b = GpuRun(w, oracle.FASGD, P, pool, th0)
+    for k in range(8):
+        cl, js, sl = ps.batch(k)
+        a.push_batch(cl, js, sl)                 # one fused pass of 8
+        for c, j, s in zip(cl, js, sl):          # the same 8 pushes queued ...
+            b.srv.push(int(c), int(j), b.pool[int(s)])
+        for _ in range(8):                       # ... applied one pass at a time
+            b.srv.apply_pending(1)
+    sa, sb = a.state(), b.state()
+    for x, y, name in zip(sa[:4], sb[:4], ("theta", "n", "b", "v")):
+        assert_bitwise(x, y, name)
+    assert sa[4] == sb[4] == 64
+    assert a.srv.launches == 8 and b.srv.launches == 64
+
+
+def test_checkpoint_restore_bitwise():
+    import torch
+    w = W["fasgd-1.29m"]
+    P = 30_001
+    pool = streams.gradient_pool(w, P)
+    th0 = streams.theta0(w, P)
+    ps = streams.push_stream(w, 120, 4)
+    a = GpuRun(w, oracle.FASGD, P, pool, th0)
+    for k in range(15):
+        a.push_batch(*ps.batch(k))
+    mid = [torch.empty(P, device="cuda") for _ in range(4)]
+    T = a.srv.get_state(*mid)
+    b = GpuRun(w, oracle.FASGD, P, pool, np.zeros(P, np.float32))
+    b.srv.set_state(*mid, T)
+    for k in range(15, 30):
+        a.push_batch(*ps.batch(k))
+        b.push_batch(*ps.batch(k))
+    for x, y in zip(a.state()[:4], b.state()[:4]):
+        assert_bitwise(x, y, "restore")
+
+
+@pytest.mark.slow
+def test_full_size_25m_k8_sampled():
+    """P = 25,000,000, K = 8, the launch the benchmark times: 200 pushes,
+    then every sampled parameter against the oracle run on those parameters
+    alone (the update is elementwise, so the sub-problem is exact)."""
+    w = W["fasgd-25m-k8"]
+    P = w.P
+    pool = streams.gradient_pool(w, P)
+    th0 = streams.theta0(w, P)
+    ps = streams.push_stream(w, 200, 8)
+    g = GpuRun(w, oracle.FASGD, P, pool, th0)
+    for b in range(25):
+        g.push_batch(*ps.batch(b))
+    gs = g.state()
+    del g
+    idx = streams.sample_indices(P, 20_000)
+    o = OracleRun(w, oracle.FASGD, idx.size, np.ascontiguousarray(pool[:, idx]), th0[idx])
+    for b in range(25):
+        o.push_batch(*ps.batch(b))
+    os_ = o.state()
+    compare_states([x[idx] for x in gs[:4]] + [gs[4]], os_, oracle.FASGD, "25M sampled")
+
+
+@pytest.mark.slow
+def test_full_size_268m_k16_sampled():
+    """P = 2^28, K = 16, Pareto(1.5) staleness, s_p up to 1: 64 pushes, sampled."""
+    import torch
+    w = W["fasgd-268m-k16"].replace(R=16)
+    P = w.P
+    pool = streams.gradient_pool(w, P)
+    th0 = streams.theta0(w, P)
+    ps = streams.push_stream(w, 64, 16)
+    g = GpuRun(w, oracle.FASGD, P, pool, th0)
+    for b in range(4):
+        g.push_batch(*ps.batch(b))
+    idx = streams.sample_indices(P, 20_000)
+    idx_t = torch.from_numpy(idx).cuda()
+    full = [torch.empty(P, device="cuda") for _ in range(4)]
+    T = g.srv.get_state(*full)
+    gs = [x[idx_t].cpu().numpy() for x in full] + [T]
+    del full, g
+    torch.cuda.empty_cache()
+    o = OracleRun(w, oracle.FASGD, idx.size, np.ascontiguousarray(pool[:, idx]), th0[idx])
+    for b in range(4):
+        o.push_batch(*ps.batch(b))
+    compare_states(gs, o.state(), oracle.FASGD, "2^28 sampled")
