@@ -247,11 +247,10 @@ def run_dense(args, w, world, rank, local):
     th0 = streams.theta0(wr, P)
     n_batches = args.warmup + args.steps
     ps = streams.push_stream(w, n_batches * K, K)
-    pool_t = torch.from_numpy(pool).to(device)
+    pool_t, slots = fasgd.aligned_vectors(pool, device)
     stream = torch.cuda.current_stream()
     srv = fasgd.Server(P, w.lam, w.alpha, variant, stream=stream)
     srv.set_params(torch.from_numpy(th0).to(device))
-    slots = [pool_t[r] for r in range(pool_t.shape[0])]
     batches = [ps.batch(b) for b in range(n_batches)]
     batches = [([int(c) for c in cl], [int(j) for j in js], [int(s) for s in sl])
                for cl, js, sl in batches]
@@ -369,11 +368,10 @@ def run_bfasgd(args, w, world, rank, local):
     th0 = streams.theta0(wr, P)
     n_steps = args.warmup + args.steps + w.lam
     ps = streams.push_stream(w.replace(R=R), n_steps, 1)
-    pool_t = torch.from_numpy(pool).to(device)
+    pool_t, slots = fasgd.aligned_vectors(pool, device)
     stream = torch.cuda.current_stream()
     srv = fasgd.Server(P, w.lam, w.alpha, streams.FASGD, stream=stream, seed=w.seed)
     srv.set_params(torch.from_numpy(th0).to(device))
-    slots = [pool_t[r] for r in range(R)]
     # Dense FASGD warm-up of lambda pushes, then c tuned on the live v for the target rate.
     t = 0
     for _ in range(w.lam):

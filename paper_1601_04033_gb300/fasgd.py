@@ -175,6 +175,20 @@ def _ptr(t) -> int | None:
     return t.data_ptr()
 
 
+def aligned_vectors(data, device="cuda"):
+    """Copy a [R, P] array (numpy or torch) to the device as R fp32 vectors of
+    length P whose starts are 16-byte aligned, as fasgd_push and
+    bfasgd_select_compact require: rows are padded to a multiple of four
+    floats inside one allocation.  Returns (backing tensor, list of views)."""
+    import torch
+    src = torch.as_tensor(data)
+    R, P = src.shape
+    pad = (P + 3) // 4 * 4
+    buf = torch.empty((R, pad), dtype=torch.float32, device=device)
+    buf[:, :P].copy_(src)
+    return buf, [buf[r, :P] for r in range(R)]
+
+
 class Server:
     """One FASGD parameter server on the current CUDA device.
 

@@ -63,7 +63,7 @@ class GpuRun:
                             eps=h["eps"], c_push=h.get("c_push", 0.0), eps_b=h["eps_b"],
                             seed=h.get("seed", 0))
         self.P = P
-        self.pool = torch.from_numpy(pool).cuda()
+        self._pool_buf, self.pool = f.aligned_vectors(pool)
         self.srv.set_params(torch.from_numpy(theta0).cuda())
 
     def push_batch(self, clients, js, slots):
