@@ -217,7 +217,49 @@ FASGD_API int64_t fasgd_pending(const fasgd_t* h);
 /* Number of kernels this handle has launched since it was created. */
 FASGD_API int64_t fasgd_kernel_launches(const fasgd_t* h);
 
-/* Text of the last failure on h (or of the last failed fasgd_create when h is NULL). */
+/*
+ * bfasgd_select_compact_noalloc -- the same send decision and compaction as
+ * bfasgd_select_compact, for callers that cannot allocate device memory.
+ * The paper has no counterpart; this entry point exists for deployment.
+ *
+ * Who needs it: code that may not call cudaMalloc when it runs -- for
+ * example a host framework that owns every device allocation through its
+ * own memory pool and forbids others, a process held to a fixed device
+ * memory budget, or a latency-critical loop that cannot afford the implicit
+ * device synchronisation an allocation can cause.  Such a caller cannot use
+ * bfasgd_select_compact, because a handle allocates its state and scratch.
+ *
+ * This entry point needs no handle and allocates nothing.  Its scratch (the
+ * per-parameter bit mask and the per-tile counts and offsets) lives in a
+ * fixed static device array of BFASGD_NOALLOC_SCRATCH_BYTES (about 2 MiB)
+ * that every GPU which loads the library holds until the process exits.
+ * The first call on a device looks up that array's device address (once per
+ * device, with that device current); make that first call before any
+ * stream capture.  All calls share the one array and the kernels rewrite
+ * every scratch word before reading it, so nothing carries over between
+ * calls -- but calls that overlap on the GPU (other streams, other host
+ * threads) race on it and must be serialised by the caller.
+ *
+ * Arguments: P parameters, 1 <= P <= BFASGD_NOALLOC_PMAX (larger P is
+ * rejected with FASGD_EINVAL and a message); grad and v: device fp32[P],
+ * 16-byte aligned (v is the client's copy of the statistic; there is no
+ * server here); c >= 0 (+inf allowed), eps_b finite >= 0; seed, client >= 0
+ * and push_no form the Philox counter and key exactly as in
+ * bfasgd_select_compact (push_no is the caller's per-client counter, not
+ * advanced here); idx, val: device, room for P entries; n_dev: device int64;
+ * stream: a cudaStream_t (NULL = legacy default stream).  Outputs as for
+ * bfasgd_select_compact, written on the stream.
+ * Errors: EINVAL (bad argument or P too large), ECUDA.
+ */
+#define BFASGD_NOALLOC_PMAX ((int64_t)1 << 24)              /* 16,777,216 parameters */
+#define BFASGD_NOALLOC_SCRATCH_BYTES ((int64_t)2121728)     /* mask + tile counts + tile bases */
+FASGD_API int bfasgd_select_compact_noalloc(int64_t P, const float* grad, const float* v, float c,
+                                            float eps_b, uint64_t seed, int32_t client,
+                                            uint64_t push_no, int32_t* idx, float* val,
+                                            int64_t* n_dev, void* stream);
+
+/* Text of the last failure on h, or, when h is NULL, of the last failed call
+ * made without a handle (fasgd_create, bfasgd_select_compact_noalloc). */
 FASGD_API const char* fasgd_last_error(const fasgd_t* h);
 
 #ifdef __cplusplus

@@ -65,6 +65,12 @@ struct DeviceGuard {
 
 }  // namespace
 
+namespace fasgd {
+// Records the failure of a call made without a handle (read back through
+// fasgd_last_error(NULL)).
+void set_handleless_error(const char* msg) { g_create_error = msg; }
+}  // namespace fasgd
+
 struct fasgd_s {
     int64_t P = 0;
     int32_t lambda = 0;

@@ -226,3 +226,118 @@ cudaError_t launch_select(const SelectArgs& a, cudaStream_t stream, int64_t* lau
 }
 
 }  // namespace fasgd
+
+// ---------------------------------------------------------------------------
+// Allocation-free variant of bfasgd_select_compact for callers that may not
+// allocate device memory (see include/fasgd.h).  The same three kernels run
+// with their scratch in one fixed static device array instead of handle-owned
+// buffers.
+// ---------------------------------------------------------------------------
+#include <cmath>
+#include <cstdio>
+#include <mutex>
+
+namespace fasgd {
+void set_handleless_error(const char* msg);  // defined in runtime.cu
+}
+
+namespace {
+
+constexpr int64_t kNoallocTiles = BFASGD_NOALLOC_PMAX / fasgd::kSelectTile;          // 2048
+constexpr int64_t kNoallocMaskBytes = kNoallocTiles * fasgd::kSelectTileWords * 4;  // 2 MiB
+constexpr int64_t kNoallocCountBytes = kNoallocTiles * 4;
+constexpr int64_t kNoallocBaseBytes = kNoallocTiles * 8;
+static_assert(kNoallocMaskBytes + kNoallocCountBytes + kNoallocBaseBytes ==
+                  BFASGD_NOALLOC_SCRATCH_BYTES,
+              "scratch size in fasgd.h out of date");
+static_assert(kNoallocMaskBytes % 256 == 0 && kNoallocCountBytes % 8 == 0, "scratch layout");
+
+// Mask words, then int32 tile counts, then int64 tile bases.
+static __device__ __align__(256) unsigned char g_noalloc_scratch[BFASGD_NOALLOC_SCRATCH_BYTES];
+
+constexpr int kMaxDevices = 64;
+std::mutex g_noalloc_mutex;
+void* g_noalloc_addr[kMaxDevices] = {};
+
+// Device address of the static scratch on the current device, looked up once
+// per device.  Host code cannot use the symbol itself as a device pointer.
+cudaError_t noalloc_scratch(unsigned char** out) {
+    int dev = 0;
+    cudaError_t st = cudaGetDevice(&dev);
+    if (st != cudaSuccess) return st;
+    if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
+    std::lock_guard<std::mutex> lock(g_noalloc_mutex);
+    if (g_noalloc_addr[dev] == nullptr) {
+        void* p = nullptr;
+        st = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+        if (st != cudaSuccess) return st;
+        g_noalloc_addr[dev] = p;
+    }
+    *out = static_cast<unsigned char*>(g_noalloc_addr[dev]);
+    return cudaSuccess;
+}
+
+bool aligned_to(const void* p, uintptr_t a) {
+    return (reinterpret_cast<uintptr_t>(p) & (a - 1)) == 0;
+}
+
+int noalloc_fail(int code, const char* msg) {
+    fasgd::set_handleless_error(msg);
+    return code;
+}
+
+}  // namespace
+
+extern "C" int bfasgd_select_compact_noalloc(int64_t P, const float* grad, const float* v,
+                                             float c, float eps_b, uint64_t seed, int32_t client,
+                                             uint64_t push_no, int32_t* idx, float* val,
+                                             int64_t* n_dev, void* stream) {
+    if (P < 1 || P > BFASGD_NOALLOC_PMAX) {
+        char buf[160];
+        snprintf(buf, sizeof buf,
+                 "bfasgd_select_compact_noalloc: P=%lld outside [1, %lld], the size of its "
+                 "static scratch", (long long)P, (long long)BFASGD_NOALLOC_PMAX);
+        return noalloc_fail(FASGD_EINVAL, buf);
+    }
+    if (client < 0) return noalloc_fail(FASGD_EINVAL, "bfasgd_select_compact_noalloc: client < 0");
+    if (grad == nullptr || v == nullptr || !aligned_to(grad, 16) || !aligned_to(v, 16))
+        return noalloc_fail(FASGD_EINVAL,
+                            "bfasgd_select_compact_noalloc: grad and v must be non-NULL "
+                            "16-byte aligned device pointers");
+    if (idx == nullptr || val == nullptr || n_dev == nullptr || !aligned_to(idx, 4) ||
+        !aligned_to(val, 4) || !aligned_to(n_dev, 8))
+        return noalloc_fail(FASGD_EINVAL,
+                            "bfasgd_select_compact_noalloc: idx, val, n_dev must be non-NULL "
+                            "and aligned");
+    if (!(c >= 0.f) || !(eps_b >= 0.f) || !std::isfinite(eps_b))
+        return noalloc_fail(FASGD_EINVAL,
+                            "bfasgd_select_compact_noalloc: need c >= 0 and finite eps_b >= 0");
+    unsigned char* scratch = nullptr;
+    cudaError_t st = noalloc_scratch(&scratch);
+    if (st != cudaSuccess)
+        return noalloc_fail(FASGD_ECUDA, "bfasgd_select_compact_noalloc: cannot address the "
+                                         "static scratch on this device");
+    fasgd::SelectArgs a;
+    a.grad = grad;
+    a.v = v;
+    a.idx = idx;
+    a.val = val;
+    a.count = n_dev;
+    a.mask = reinterpret_cast<uint32_t*>(scratch);
+    a.tile_count = reinterpret_cast<int32_t*>(scratch + kNoallocMaskBytes);
+    a.tile_base = reinterpret_cast<int64_t*>(scratch + kNoallocMaskBytes + kNoallocCountBytes);
+    a.P = P;
+    a.ntiles = fasgd::select_tiles(P);
+    a.c = c;
+    a.eps_b = eps_b;
+    a.key0 = (uint32_t)seed;
+    a.key1 = (uint32_t)(seed >> 32);
+    a.client = (uint32_t)client;
+    a.push_lo = (uint32_t)push_no;
+    a.push_hi = (uint32_t)(push_no >> 32);
+    int64_t launches = 0;
+    st = fasgd::launch_select(a, static_cast<cudaStream_t>(stream), &launches);
+    if (st != cudaSuccess)
+        return noalloc_fail(FASGD_ECUDA, cudaGetErrorString(st));
+    return FASGD_OK;
+}

@@ -47,8 +47,12 @@ SIGNATURES = {
     "fasgd_timestamp": (_i64, [_p]),
     "fasgd_pending": (_i64, [_p]),
     "fasgd_kernel_launches": (_i64, [_p]),
+    "bfasgd_select_compact_noalloc": (_i32, [_i64, _p, _p, _f32, _f32, _u64, _i32, _u64,
+                                             _p, _p, _p, _p]),
     "fasgd_last_error": (ctypes.c_char_p, [_p]),
 }
+
+NOALLOC_PMAX = 1 << 24
 
 
 def _load() -> ctypes.CDLL:
@@ -157,6 +161,12 @@ def fasgd_pending(h):
 
 def fasgd_kernel_launches(h):
     return LIB.fasgd_kernel_launches(h)
+
+
+def bfasgd_select_compact_noalloc(P, grad, v, c, eps_b, seed, client, push_no, idx, val,
+                                  n_dev, stream):
+    return LIB.bfasgd_select_compact_noalloc(P, grad, v, c, eps_b, seed, client, push_no, idx,
+                                             val, n_dev, stream)
 
 
 def fasgd_last_error(h) -> str:
