@@ -336,7 +336,7 @@ def run_dense(args, w, world, rank, local):
     achieved = alg / (kern_avg_ms / 1e3) / 1e9
     roofline = {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
                 "frac": round(achieved / peak, 4), "peak_source": peak_kind,
-                "kernel": "fasgd_dense_kernel<FASGD, G=%d>" % min(16, 1 << (K.bit_length() - 1)),
+                "kernel": "fasgd_dense_kernel<FASGD> (bulk-copy ring)",
                 "bytes_per_launch": alg, "launch_ms": round(kern_avg_ms, 5),
                 "traffic": profiled_traffic(w.name if not args.P else f"{w.name}-P{P}",
                                             DENSE_KERNEL_SOURCES)}

@@ -206,7 +206,9 @@ FASGD_API int fasgd_set_push_counts(fasgd_t* h, const uint64_t* counts);
 /*
  * fasgd_sync -- wait until the handle's stream is idle, then report and
  * clear the device-side error flags: FASGD_EDEVICE if a sparse list held a
- * bad entry since the last sync, else FASGD_OK (or ECUDA).
+ * bad entry, or a wait inside the dense pass's copy pipeline expired (it
+ * gives up after about a second rather than hang), since the last sync;
+ * else FASGD_OK (or ECUDA).
  */
 FASGD_API int fasgd_sync(fasgd_t* h);
 

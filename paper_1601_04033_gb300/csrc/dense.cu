@@ -1,15 +1,28 @@
 // Fused dense server pass: K pending pushes applied in one sweep over P.
 //
-// Each thread owns four consecutive parameters at a time (128-bit loads and
-// stores).  theta (and n, b, v for FASGD) are loaded once, the K gradient
-// slices are streamed in groups of G, every push is applied in arrival order
-// with the state held in registers, and the state is stored once.  The pass
-// therefore moves (8 + 4K) bytes per parameter for ASGD/SASGD and
-// (32 + 4K) for FASGD, the minimum for K pushes (paper Sec. 2.1 protocol,
-// Eq. 1-2 and Eq. 4-8 applied K times).
+// Every parameter's theta (and n, b, v for FASGD) is read once, the K
+// gradient slices are read once, all K pushes are applied in arrival order
+// with the state held in registers, and the state is written once.  The pass
+// therefore moves (8 + 4K) bytes per parameter for ASGD/SASGD and (32 + 4K)
+// for FASGD, the minimum for K pushes (paper Sec. 2.1 protocol, Eq. 1-2 and
+// Eq. 4-8 applied K times).
 //
-// Elements are independent, so the result does not depend on the grid: the
-// per-element operation sequence is the same for every launch shape.
+// Structure: a persistent kernel, one block per SM, one producer warp and
+// 16 consumer warps.  The parameter range is cut into tiles of 2048; the
+// producer's elected lane stages each tile's state slices and up to 8
+// gradient slices into a shared-memory ring with 1-D bulk async copies
+// (cp.async.bulk, completion counted on an mbarrier), while the consumer
+// warps compute on the previous stage: each thread takes four consecutive
+// parameters (128-bit shared loads), frees the stage as soon as its inputs
+// are in registers, applies the pushes, and stores the state with 128-bit
+// global stores.  A stage holds up to 8 gradient slices; larger K runs as
+// several stages per tile (the state travels with the first one only).  The
+// last P mod 2048 parameters are handled by plain loads in the last block.
+//
+// Every wait on an mbarrier is bounded (about one second of wall clock);
+// on expiry the block sets flag 8 of the error word, waits (bounded) for its
+// own copies in flight, and returns.  Elements are independent, so the
+// result does not depend on the grid or on which path handled an element.
 
 #include "kernels.cuh"
 #include "update.cuh"
@@ -17,29 +30,89 @@
 namespace fasgd {
 namespace {
 
-constexpr int kDenseThreads = 256;
+constexpr int kConsumers = 512;                 // consumer threads per block
+constexpr int kTile = 4 * kConsumers;           // parameters per tile
+constexpr int kThreads = kConsumers + 32;       // + one producer warp
+constexpr int kMaxStages = 8;
+constexpr int kSmemBudget = 220 * 1024;         // ring + barriers, per block
+constexpr unsigned kFull = 0xffffffffu;
+constexpr int kErrWaitTimeout = 8;
 
-__device__ __forceinline__ float4 ld_state(const float* p) {
-    return *reinterpret_cast<const float4*>(p);
+// ---- PTX wrappers: mbarrier and bulk async copy ---------------------------
+__device__ __forceinline__ uint32_t smem_addr(const void* p) {
+    return (uint32_t)__cvta_generic_to_shared(p);
+}
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_addr(bar)), "r"(count)
+                 : "memory");
+}
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t* bar, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_addr(bar)),
+                 "r"(bytes)
+                 : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_addr(bar)) : "memory");
+}
+__device__ __forceinline__ bool mbar_test(uint64_t* bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+        " selp.u32 %0, 1, 0, p;\n}\n"
+        : "=r"(ok)
+        : "r"(smem_addr(bar)), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+__device__ __forceinline__ uint64_t global_ns() {
+    uint64_t t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+constexpr uint64_t kWaitLimitNs = 1000000000ull;
+
+// One thread waits for the phase with the given parity to complete.
+__device__ bool wait_one(uint64_t* bar, uint32_t parity, int32_t* err) {
+    if (mbar_test(bar, parity)) return true;
+    const uint64_t t0 = global_ns();
+    for (uint32_t i = 0; i < (1u << 26); ++i) {
+        if (mbar_test(bar, parity)) return true;
+        if ((i & 255u) == 255u && global_ns() - t0 > kWaitLimitNs) break;
+    }
+    atomicOr(err, kErrWaitTimeout);
+    return false;
+}
+// A whole warp waits; every lane observes the barrier (acquire) and the warp
+// leaves together.
+__device__ bool wait_warp(uint64_t* bar, uint32_t parity, int32_t* err) {
+    const uint64_t t0 = global_ns();
+    for (uint32_t i = 0; i < (1u << 26); ++i) {
+        if (__all_sync(kFull, mbar_test(bar, parity))) return true;
+        const bool late = (i & 255u) == 255u && global_ns() - t0 > kWaitLimitNs;
+        if (__any_sync(kFull, late)) break;
+    }
+    if ((threadIdx.x & 31) == 0) atomicOr(err, kErrWaitTimeout);
+    return false;
+}
+// 1-D bulk copy global -> shared (16-byte aligned, size a multiple of 16),
+// completion signalled on `bar` as transaction bytes.
+__device__ __forceinline__ void bulk_load(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
+    asm volatile(
+        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+            smem_addr(dst)),
+        "l"(src), "r"(bytes), "r"(smem_addr(bar))
+        : "memory");
 }
 
-__device__ __forceinline__ void st_state(float* p, const float4& x) {
-    *reinterpret_cast<float4*>(p) = x;
-}
-
-// Gradient slices are read exactly once: streaming (evict-first) loads.
-__device__ __forceinline__ float4 ld_grad(const float* p) {
-    return __ldcs(reinterpret_cast<const float4*>(p));
-}
-
-template <bool FAS>
-__device__ __forceinline__ void update4(float4& th, float4& n, float4& b, float4& v,
-                                        const float4& g, float coef, const StatParams& sp) {
+// ---- the element update on four consecutive parameters --------------------
+template <bool FAS, bool FTZ>
+__device__ __forceinline__ void update4(float4& th, float4& n, float4& b, float4& v, const float4& g,
+                                        float coef, const StatParams& sp) {
     if (FAS) {
-        fasgd_update(th.x, n.x, b.x, v.x, g.x, coef, sp);
-        fasgd_update(th.y, n.y, b.y, v.y, g.y, coef, sp);
-        fasgd_update(th.z, n.z, b.z, v.z, g.z, coef, sp);
-        fasgd_update(th.w, n.w, b.w, v.w, g.w, coef, sp);
+        fasgd_update<FTZ>(th.x, n.x, b.x, v.x, g.x, coef, sp);
+        fasgd_update<FTZ>(th.y, n.y, b.y, v.y, g.y, coef, sp);
+        fasgd_update<FTZ>(th.z, n.z, b.z, v.z, g.z, coef, sp);
+        fasgd_update<FTZ>(th.w, n.w, b.w, v.w, g.w, coef, sp);
     } else {
         sgd_update(th.x, g.x, coef);
         sgd_update(th.y, g.y, coef);
@@ -48,60 +121,42 @@ __device__ __forceinline__ void update4(float4& th, float4& n, float4& b, float4
     }
 }
 
-template <bool FAS, int G>
-__global__ void __launch_bounds__(kDenseThreads)
-fasgd_dense_kernel(const __grid_constant__ DenseArgs a) {
-    const int64_t nquads = a.P >> 2;
-    const int64_t stride = (int64_t)gridDim.x * kDenseThreads;
-    const int K = a.K;
-    for (int64_t q = (int64_t)blockIdx.x * kDenseThreads + threadIdx.x; q < nquads; q += stride) {
-        const int64_t e = q << 2;
-        float4 th = ld_state(a.theta + e);
+// Parameters [begin, P) with plain loads, by the consumer threads of one
+// block; begin is a multiple of 4.
+template <bool FAS, bool FTZ>
+__device__ void apply_range_direct(const DenseArgs& a, int64_t begin, int tid) {
+    const int64_t end_q = a.P & ~int64_t(3);
+    for (int64_t e = begin + 4 * (int64_t)tid; e < end_q; e += 4 * (int64_t)kConsumers) {
+        float4 th = *reinterpret_cast<const float4*>(a.theta + e);
         float4 n = make_float4(0.f, 0.f, 0.f, 0.f), b = n, v = n;
         if (FAS) {
-            n = ld_state(a.n + e);
-            b = ld_state(a.b + e);
-            v = ld_state(a.v + e);
+            n = *reinterpret_cast<const float4*>(a.n + e);
+            b = *reinterpret_cast<const float4*>(a.b + e);
+            v = *reinterpret_cast<const float4*>(a.v + e);
         }
-        int k0 = 0;
-        for (; k0 + G <= K; k0 += G) {
-            float4 g[G];
-#pragma unroll
-            for (int j = 0; j < G; ++j) g[j] = ld_grad(a.grad[k0 + j] + e);
-#pragma unroll
-            for (int j = 0; j < G; ++j) update4<FAS>(th, n, b, v, g[j], a.coef[k0 + j], a.sp);
+        for (int k = 0; k < a.K; ++k) {
+            const float4 g = __ldcs(reinterpret_cast<const float4*>(a.grad[k] + e));
+            update4<FAS, FTZ>(th, n, b, v, g, a.coef[k], a.sp);
         }
-        if (k0 < K) {  // last, partial group
-            float4 g[G];
-#pragma unroll
-            for (int j = 0; j < G; ++j)
-                if (k0 + j < K) g[j] = ld_grad(a.grad[k0 + j] + e);
-#pragma unroll
-            for (int j = 0; j < G; ++j)
-                if (k0 + j < K) update4<FAS>(th, n, b, v, g[j], a.coef[k0 + j], a.sp);
-        }
-        st_state(a.theta + e, th);
+        *reinterpret_cast<float4*>(a.theta + e) = th;
         if (FAS) {
-            st_state(a.n + e, n);
-            st_state(a.b + e, b);
-            st_state(a.v + e, v);
+            *reinterpret_cast<float4*>(a.n + e) = n;
+            *reinterpret_cast<float4*>(a.b + e) = b;
+            *reinterpret_cast<float4*>(a.v + e) = v;
         }
     }
-    // Ragged tail: the last P mod 4 parameters, one per thread of the last block.
-    const int rem = (int)(a.P & 3);
-    if (rem != 0 && blockIdx.x == gridDim.x - 1 && (int)threadIdx.x < rem) {
-        const int64_t p = (nquads << 2) + threadIdx.x;
-        float th = a.theta[p];
-        float n = 0.f, b = 0.f, v = 0.f;
+    const int64_t p = end_q + tid;  // the last P mod 4 parameters
+    if (tid < (int)(a.P & 3) && p < a.P) {
+        float th = a.theta[p], n = 0.f, b = 0.f, v = 0.f;
         if (FAS) {
             n = a.n[p];
             b = a.b[p];
             v = a.v[p];
         }
-        for (int k = 0; k < K; ++k) {
+        for (int k = 0; k < a.K; ++k) {
             const float g = __ldcs(a.grad[k] + p);
             if (FAS)
-                fasgd_update(th, n, b, v, g, a.coef[k], a.sp);
+                fasgd_update<FTZ>(th, n, b, v, g, a.coef[k], a.sp);
             else
                 sgd_update(th, g, a.coef[k]);
         }
@@ -114,40 +169,181 @@ fasgd_dense_kernel(const __grid_constant__ DenseArgs a) {
     }
 }
 
-template <bool FAS, int G>
-cudaError_t launch_g(const DenseArgs& a, int num_sms, cudaStream_t stream) {
-    static int blocks_per_sm = 0;  // resident blocks of this instantiation, queried once
-    if (blocks_per_sm == 0) {
-        cudaError_t st = cudaOccupancyMaxActiveBlocksPerMultiprocessor(
-            &blocks_per_sm, fasgd_dense_kernel<FAS, G>, kDenseThreads, 0);
-        if (st != cudaSuccess) return st;
-        if (blocks_per_sm < 1) blocks_per_sm = 1;
+// Ring geometry, identical on host and device.
+struct Ring {
+    int stages;     // stages in the ring
+    int chunks;     // stages per tile: ceil(K / CH)
+};
+
+// FAS: FASGD rule (else ASGD/SASGD); FTZ: flush-to-zero MUFU forms (see
+// update.cuh); CH: gradient slices per stage.
+template <bool FAS, bool FTZ, int CH>
+__global__ void __launch_bounds__(kThreads, 1)
+fasgd_dense_kernel(const __grid_constant__ DenseArgs a, const Ring ring, const int64_t ntiles) {
+    constexpr int kState = FAS ? 4 : 1;              // theta (, n, b, v)
+    constexpr int kStageFloats = (kState + CH) * kTile;
+    extern __shared__ __align__(128) unsigned char smem[];
+    float* buf = reinterpret_cast<float*>(smem);
+    uint64_t* full = reinterpret_cast<uint64_t*>(smem + (size_t)ring.stages * kStageFloats * 4);
+    uint64_t* empty = full + ring.stages;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    constexpr int kConsumerWarps = kConsumers / 32;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < ring.stages; ++s) {
+            mbar_init(&full[s], 1);
+            mbar_init(&empty[s], kConsumerWarps);
+        }
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
-    const int64_t nquads = a.P >> 2;
-    int64_t want = (nquads + kDenseThreads - 1) / kDenseThreads;
-    const int64_t cap = (int64_t)num_sms * blocks_per_sm;
-    if (want > cap) want = cap;
-    if (want < 1) want = 1;
-    fasgd_dense_kernel<FAS, G><<<(unsigned)want, kDenseThreads, 0, stream>>>(a);
+    __syncthreads();
+
+    if (warp == kConsumerWarps) {
+        // ---------------- producer: one elected lane ----------------
+        if (lane == 0) {
+            int s = 0;
+            uint32_t ph = 0;
+            bool ok = true;
+            uint32_t issued = 0;            // bit s: stage s has been filled
+            uint32_t issued_phase = 0;      // bit s: the phase parity of its last fill
+            for (int64_t t = blockIdx.x; t < ntiles && ok; t += gridDim.x) {
+                const int64_t off = t * kTile;
+                for (int c = 0; c < ring.chunks; ++c) {
+                    ok = wait_one(&empty[s], ph ^ 1u, a.err);
+                    if (!ok) break;
+                    const int k0 = c * CH;
+                    const int ng = min(CH, a.K - k0);
+                    const int ns = (c == 0) ? kState : 0;
+                    mbar_arrive_expect_tx(&full[s], (uint32_t)((ns + ng) * kTile * 4));
+                    float* st = buf + (size_t)s * kStageFloats;
+                    if (ns > 0) {
+                        bulk_load(st, a.theta + off, kTile * 4, &full[s]);
+                        if (FAS) {
+                            bulk_load(st + 1 * kTile, a.n + off, kTile * 4, &full[s]);
+                            bulk_load(st + 2 * kTile, a.b + off, kTile * 4, &full[s]);
+                            bulk_load(st + 3 * kTile, a.v + off, kTile * 4, &full[s]);
+                        }
+                    }
+                    float* gs = st + kState * kTile;
+                    for (int j = 0; j < ng; ++j)
+                        bulk_load(gs + j * kTile, a.grad[k0 + j] + off, kTile * 4, &full[s]);
+                    issued |= 1u << s;
+                    issued_phase = (issued_phase & ~(1u << s)) | (ph << s);
+                    if (++s == ring.stages) {
+                        s = 0;
+                        ph ^= 1u;
+                    }
+                }
+            }
+            // Every fill issued by this block has landed before it exits.
+            for (int i = 0; i < ring.stages; ++i)
+                if (issued & (1u << i)) wait_one(&full[i], (issued_phase >> i) & 1u, a.err);
+        }
+        return;
+    }
+
+    // ---------------- consumers ----------------
+    const int tid = threadIdx.x;
+    int s = 0;
+    uint32_t ph = 0;
+    bool ok = true;
+    for (int64_t t = blockIdx.x; t < ntiles && ok; t += gridDim.x) {
+        float4 th = make_float4(0.f, 0.f, 0.f, 0.f), n = th, b = th, v = th;
+        for (int c = 0; c < ring.chunks; ++c) {
+            ok = wait_warp(&full[s], ph, a.err);
+            if (!ok) break;
+            const float* st = buf + (size_t)s * kStageFloats;
+            if (c == 0) {
+                th = reinterpret_cast<const float4*>(st)[tid];
+                if (FAS) {
+                    n = reinterpret_cast<const float4*>(st + 1 * kTile)[tid];
+                    b = reinterpret_cast<const float4*>(st + 2 * kTile)[tid];
+                    v = reinterpret_cast<const float4*>(st + 3 * kTile)[tid];
+                }
+            }
+            const int k0 = c * CH;
+            const float4* gs = reinterpret_cast<const float4*>(st + kState * kTile);
+            float4 g[CH];
+            if (k0 + CH <= a.K) {  // a full chunk
+#pragma unroll
+                for (int j = 0; j < CH; ++j) g[j] = gs[j * (kTile / 4) + tid];
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&empty[s]);  // inputs are in registers
+#pragma unroll
+                for (int j = 0; j < CH; ++j) update4<FAS, FTZ>(th, n, b, v, g[j], a.coef[k0 + j], a.sp);
+            } else {               // the last, partial chunk
+                const int ng = a.K - k0;
+#pragma unroll
+                for (int j = 0; j < CH; ++j)
+                    if (j < ng) g[j] = gs[j * (kTile / 4) + tid];
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&empty[s]);
+#pragma unroll
+                for (int j = 0; j < CH; ++j)
+                    if (j < ng) update4<FAS, FTZ>(th, n, b, v, g[j], a.coef[k0 + j], a.sp);
+            }
+            if (++s == ring.stages) {
+                s = 0;
+                ph ^= 1u;
+            }
+        }
+        if (!ok) break;
+        const int64_t e = t * kTile + 4 * (int64_t)tid;
+        *reinterpret_cast<float4*>(a.theta + e) = th;
+        if (FAS) {
+            *reinterpret_cast<float4*>(a.n + e) = n;
+            *reinterpret_cast<float4*>(a.b + e) = b;
+            *reinterpret_cast<float4*>(a.v + e) = v;
+        }
+    }
+    // Parameters after the last full tile.
+    if (ok && blockIdx.x == gridDim.x - 1) apply_range_direct<FAS, FTZ>(a, ntiles * kTile, tid);
+}
+
+template <bool FAS, bool FTZ, int CH>
+cudaError_t launch_ch(const DenseArgs& a, int num_sms, cudaStream_t stream) {
+    constexpr int kState = FAS ? 4 : 1;
+    constexpr int kStageBytes = (kState + CH) * kTile * 4;
+    Ring ring;
+    ring.chunks = (a.K + CH - 1) / CH;
+    ring.stages = (kSmemBudget - 2 * kMaxStages * 8) / kStageBytes;
+    if (ring.stages > kMaxStages) ring.stages = kMaxStages;
+    const size_t smem = (size_t)ring.stages * kStageBytes + 2 * ring.stages * sizeof(uint64_t);
+    static bool configured = false;  // per instantiation
+    if (!configured) {
+        cudaError_t st = cudaFuncSetAttribute(fasgd_dense_kernel<FAS, FTZ, CH>,
+                                              cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                              kSmemBudget);
+        if (st != cudaSuccess) return st;
+        configured = true;
+    }
+    const int64_t ntiles = a.P / kTile;
+    int64_t grid = ntiles < num_sms ? ntiles : num_sms;  // one block per SM (shared-memory bound)
+    if (grid < 1) grid = 1;
+    fasgd_dense_kernel<FAS, FTZ, CH><<<(unsigned)grid, kThreads, smem, stream>>>(a, ring, ntiles);
     return cudaGetLastError();
 }
 
-template <bool FAS>
+template <bool FAS, bool FTZ>
 cudaError_t launch_rule(const DenseArgs& a, int num_sms, cudaStream_t stream) {
-    // Group size: the largest power of two <= K, at most 16.
-    if (a.K >= 16) return launch_g<FAS, 16>(a, num_sms, stream);
-    if (a.K >= 8) return launch_g<FAS, 8>(a, num_sms, stream);
-    if (a.K >= 4) return launch_g<FAS, 4>(a, num_sms, stream);
-    if (a.K >= 2) return launch_g<FAS, 2>(a, num_sms, stream);
-    return launch_g<FAS, 1>(a, num_sms, stream);
+    // Gradient slices per stage: K rounded up to a power of two, at most 8.
+    if (a.K > 4) return launch_ch<FAS, FTZ, 8>(a, num_sms, stream);
+    if (a.K > 2) return launch_ch<FAS, FTZ, 4>(a, num_sms, stream);
+    if (a.K > 1) return launch_ch<FAS, FTZ, 2>(a, num_sms, stream);
+    return launch_ch<FAS, FTZ, 1>(a, num_sms, stream);
 }
 
 }  // namespace
 
 cudaError_t launch_dense(const DenseArgs& a, bool fasgd_rule, int num_sms, cudaStream_t stream,
                          int64_t* launches) {
-    cudaError_t st = fasgd_rule ? launch_rule<true>(a, num_sms, stream)
-                                : launch_rule<false>(a, num_sms, stream);
+    cudaError_t st;
+    if (!fasgd_rule)
+        st = launch_rule<false, false>(a, num_sms, stream);
+    else if (a.sp.eps >= kFtzSafeEps)
+        st = launch_rule<true, true>(a, num_sms, stream);
+    else
+        st = launch_rule<true, false>(a, num_sms, stream);
     if (st == cudaSuccess) ++*launches;
     return st;
 }

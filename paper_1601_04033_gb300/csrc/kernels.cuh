@@ -28,6 +28,7 @@ struct DenseArgs {
     int64_t P;
     int32_t K;
     StatParams sp;
+    int32_t* err;                   // device error flags (bit 3: a pipeline wait expired)
 };
 
 // One sparse push: idx[i] receives val[i] for i < count.

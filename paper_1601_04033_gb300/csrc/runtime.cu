@@ -335,6 +335,7 @@ int fasgd_apply_pending(fasgd_t* h, int32_t K) {
             a.v = h->v;
             a.P = h->P;
             a.sp = sp;
+            a.err = h->dev_err;
             int r = 0;
             while (k + r < K && !h->fifo[(size_t)(k + r)].sparse) {
                 const Push& p = h->fifo[(size_t)(k + r)];
@@ -488,8 +489,9 @@ int fasgd_sync(fasgd_t* h) {
         st = cudaMemset(h->dev_err, 0, sizeof(int32_t));
         if (st == cudaSuccess) st = cudaDeviceSynchronize();
         if (st != cudaSuccess) return h->cuda_fail(st, "fasgd_sync");
-        return h->fail(FASGD_EDEVICE, "sparse list error flags 0x%x (1: count > n_max, "
-                                      "2: index out of range, 4: indices not ascending)", flags);
+        return h->fail(FASGD_EDEVICE, "device error flags 0x%x (1: sparse count > n_max, "
+                                      "2: sparse index out of range, 4: sparse indices not "
+                                      "ascending, 8: a dense-pass pipeline wait expired)", flags);
     }
     return FASGD_OK;
 }

@@ -5,20 +5,36 @@
 
 namespace fasgd {
 
-// Hardware approximations (PTX rsqrt.approx.f32 / rcp.approx.f32, subnormals
-// kept).  Their error is a few ulp, far inside the 1e-5 relative bound the
-// results are held to; see the rounding notes on fasgd_update below.
+// Hardware approximations (PTX rsqrt.approx / rcp.approx).  Their error is a
+// few ulp, far inside the 1e-5 relative bound the results are held to; see
+// the rounding notes on fasgd_update below.  FTZ selects the forms that flush
+// subnormal inputs and outputs to zero.  In fasgd_update they give the same
+// results as the subnormal-preserving forms whenever eps >= 2^-126 and the
+// gradients are finite: the radicand is then at least 2^-126, and v, a
+// weighted mean of r >= (1 - beta) / sqrt(FLT_MAX) with 1 - beta >= 2^-24,
+// is at least 2^-88; neither they nor their reciprocals are subnormal.
+template <bool FTZ>
 __device__ __forceinline__ float rsqrt_approx(float x) {
     float y;
-    asm("rsqrt.approx.f32 %0, %1;" : "=f"(y) : "f"(x));
+    if (FTZ)
+        asm("rsqrt.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    else
+        asm("rsqrt.approx.f32 %0, %1;" : "=f"(y) : "f"(x));
     return y;
 }
 
+template <bool FTZ>
 __device__ __forceinline__ float rcp_approx(float x) {
     float y;
-    asm("rcp.approx.f32 %0, %1;" : "=f"(y) : "f"(x));
+    if (FTZ)
+        asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    else
+        asm("rcp.approx.f32 %0, %1;" : "=f"(y) : "f"(x));
     return y;
 }
+
+// Smallest eps for which the flush-to-zero forms are exact substitutes.
+constexpr float kFtzSafeEps = 1.17549435e-38f;  // 2^-126
 
 // ASGD / SASGD (Eq. 1-2): theta <- theta - alpha(tau) * g.  Both operations
 // are rounded separately (no fused multiply-add), so the result is the
@@ -38,14 +54,15 @@ __device__ __forceinline__ void sgd_update(float& theta, float g, float coef) {
 // v and theta updates differ from a once-rounded sequence by a few ulp; v is
 // a positive weighted mean, so that difference does not grow, and theta only
 // accumulates it relative to the size of each step.
+template <bool FTZ = false>
 __device__ __forceinline__ void fasgd_update(float& theta, float& n, float& b, float& v,
                                              float g, float coef, const StatParams& sp) {
     n = __fadd_rn(__fmul_rn(sp.gamma, n), __fmul_rn(sp.one_m_gamma, __fmul_rn(g, g)));
     b = __fadd_rn(__fmul_rn(sp.gamma, b), __fmul_rn(sp.one_m_gamma, g));
     const float var = fmaxf(__fsub_rn(n, __fmul_rn(b, b)), 0.0f);
-    const float r = rsqrt_approx(__fadd_rn(var, sp.eps));
+    const float r = rsqrt_approx<FTZ>(__fadd_rn(var, sp.eps));
     v = fmaf(sp.beta, v, sp.one_m_beta * r);
-    theta = fmaf(-(coef * g), rcp_approx(v), theta);
+    theta = fmaf(-(coef * g), rcp_approx<FTZ>(v), theta);
 }
 
 }  // namespace fasgd

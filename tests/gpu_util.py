@@ -31,9 +31,10 @@ def binding():
 def assert_close(gpu, ora, what):
     gpu = np.asarray(gpu, dtype=np.float64)
     ora = np.asarray(ora, dtype=np.float64)
-    d = np.abs(gpu - ora)
+    with np.errstate(invalid="ignore"):
+        d = np.abs(gpu - ora)
     bound = RTOL * np.abs(ora) + ATOL
-    bad = np.nonzero(~(d <= bound))[0]
+    bad = np.nonzero(~((d <= bound) | (gpu == ora)))[0]   # equal infinities match
     if bad.size:
         i = bad[np.argmax((d[bad] - bound[bad]))]
         raise AssertionError(f"{what}: {bad.size} of {gpu.size} outside tolerance; worst at {i}: "

@@ -158,3 +158,18 @@ def test_full_size_268m_k16_sampled():
     for b in range(4):
         o.push_batch(*ps.batch(b))
     compare_states(gs, o.state(), oracle.FASGD, "2^28 sampled")
+
+
+@pytest.mark.parametrize("K", [3, 8, 16])
+def test_eps_zero_subnormal_preserving_path(K):
+    """eps = 0 selects the MUFU forms that keep subnormals (the flush-to-zero
+    forms are used only for eps >= 2^-126, where they are exact substitutes)."""
+    w = W["fasgd-25m-k8"].replace(R=max(2 * K, 16))
+    n = 100 * K // np.gcd(100, K)
+    run_parity(w, oracle.FASGD, 20_483, n, K, eps=0.0)
+
+
+def test_eps_at_ftz_threshold():
+    """eps = 2^-126 exactly (the smallest eps on the flush-to-zero path)."""
+    w = W["fasgd-7850"]
+    run_parity(w, oracle.FASGD, w.P, 200, 4, eps=float(np.float32(2.0 ** -126)))
