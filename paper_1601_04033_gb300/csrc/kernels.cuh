@@ -66,7 +66,8 @@ struct SelectArgs {
     int32_t ntiles;
     float c;
     float eps_b;
-    uint32_t key0, key1;           // Philox key = seed
+    uint32_t round_key0[10];       // Philox key schedule: seed advanced by the
+    uint32_t round_key1[10];       // Weyl constants, one pair per round
     uint32_t client, push_lo, push_hi;
 };
 
@@ -81,5 +82,8 @@ cudaError_t launch_select(const SelectArgs& a, cudaStream_t stream, int64_t* lau
 inline int32_t select_tiles(int64_t P) {
     return (int32_t)((P + kSelectTile - 1) / kSelectTile);
 }
+
+// Fills the Philox key schedule of `a` from the 64-bit seed.
+void select_key_schedule(SelectArgs& a, uint64_t seed);
 
 }  // namespace fasgd

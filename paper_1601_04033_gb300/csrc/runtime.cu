@@ -405,8 +405,7 @@ int bfasgd_select_compact(fasgd_t* h, int32_t client, const float* grad, const f
     a.ntiles = h->ntiles;
     a.c = h->c_push;
     a.eps_b = h->eps_b;
-    a.key0 = (uint32_t)h->seed;
-    a.key1 = (uint32_t)(h->seed >> 32);
+    fasgd::select_key_schedule(a, h->seed);
     const uint64_t push_no = h->push_count[(size_t)client];
     a.client = (uint32_t)client;
     a.push_lo = (uint32_t)push_no;

@@ -13,8 +13,8 @@
 //               warps) and write idx[rank] = p, val[rank] = grad[p].
 // The order of the output is the order of p, so the result is unique and
 // does not depend on the launch; no atomics are used.  Traffic per
-// parameter: v (4 B) + grad (4 B, skipped where a whole quad is dropped) +
-// 2 x 1/8 B of mask, plus 8 B per sent entry.
+// parameter: v (4 B) + grad (4 B) + 2 x 1/8 B of mask, plus 8 B per sent
+// entry.  Each lane issues all eight of its 128-bit loads before it computes.
 
 #include "kernels.cuh"
 
@@ -26,29 +26,27 @@ constexpr int kWarpSpan = kSelectTile / kWarps;  // 1024 parameters per warp
 constexpr int kIters = kWarpSpan / 128;          // 8 passes of 32 lanes x 4
 constexpr unsigned kFull = 0xffffffffu;
 
-// Philox4x32-10 (Salmon, Moraes, Dror, Shaw, SC'11): ten rounds of two
-// 32x32->64 multiplies on a 128-bit counter, the 64-bit key advanced by the
-// golden-ratio Weyl increments between rounds.
+// Philox4x32-10 (Salmon, Moraes, Dror, Shaw, SC'11): ten rounds, each two
+// 32x32->64 products of the counter's even words with the round multipliers,
+// the high halves xor-ed with the odd words and the round key.  The key
+// schedule (seed advanced by the Weyl constants) is precomputed on the host.
+constexpr uint32_t kPhiloxM0 = 0xD2511F53u, kPhiloxM1 = 0xCD9E8D57u;
+constexpr uint32_t kPhiloxW0 = 0x9E3779B9u, kPhiloxW1 = 0xBB67AE85u;
+
 struct Philox4 {
     uint32_t x[4];
 };
 
 __device__ __forceinline__ Philox4 philox4x32_10(uint32_t c0, uint32_t c1, uint32_t c2,
-                                                 uint32_t c3, uint32_t k0, uint32_t k1) {
+                                                 uint32_t c3, const SelectArgs& a) {
 #pragma unroll
     for (int r = 0; r < 10; ++r) {
-        const uint32_t lo0 = 0xD2511F53u * c0;
-        const uint32_t hi0 = __umulhi(0xD2511F53u, c0);
-        const uint32_t lo1 = 0xCD9E8D57u * c2;
-        const uint32_t hi1 = __umulhi(0xCD9E8D57u, c2);
-        const uint32_t n0 = hi1 ^ c1 ^ k0;
-        const uint32_t n2 = hi0 ^ c3 ^ k1;
-        c0 = n0;
-        c1 = lo1;
-        c2 = n2;
-        c3 = lo0;
-        k0 += 0x9E3779B9u;
-        k1 += 0xBB67AE85u;
+        const uint64_t p0 = (uint64_t)kPhiloxM0 * c0;
+        const uint64_t p1 = (uint64_t)kPhiloxM1 * c2;
+        c0 = (uint32_t)(p1 >> 32) ^ c1 ^ a.round_key0[r];
+        c1 = (uint32_t)p1;
+        c2 = (uint32_t)(p0 >> 32) ^ c3 ^ a.round_key1[r];
+        c3 = (uint32_t)p0;
     }
     Philox4 o;
     o.x[0] = c0;
@@ -59,8 +57,12 @@ __device__ __forceinline__ Philox4 philox4x32_10(uint32_t c0, uint32_t c1, uint3
 }
 
 // Eq. 9 for one parameter: send iff u / 2^24 < 1 / (1 + c / a), a = fl(v + eps_b),
-// evaluated exactly as u * fl(a + c) < a * 2^24 with the product split into
-// its rounded value and its exact error.
+// i.e. iff u * d < A with d = fl(a + c) and A = a * 2^24, decided exactly:
+// u * d = prod + err exactly (prod = fl(u * d), err = fma(u, d, -prod)), and
+// u * d < A  <=>  err < A - prod  <=>  err < fl(A - prod).  The last step is
+// exact: when A and prod are within a factor of two, A - prod is exact
+// (Sterbenz); otherwise |A - prod| > 2^-24 prod >= |err|, and rounding
+// A - prod keeps it on the same side of err.
 __device__ __forceinline__ uint32_t send_bit(uint32_t u, float v, float c, float eps_b) {
     const float a = __fadd_rn(v, eps_b);
     const float d = __fadd_rn(a, c);
@@ -68,7 +70,7 @@ __device__ __forceinline__ uint32_t send_bit(uint32_t u, float v, float c, float
     const float prod = __fmul_rn(uf, d);
     const float err = __fmaf_rn(uf, d, -prod);
     const float A = __fmul_rn(a, 16777216.0f);
-    return (prod < A || (prod == A && err < 0.0f)) ? 1u : 0u;
+    return err < __fsub_rn(A, prod) ? 1u : 0u;
 }
 
 __global__ void __launch_bounds__(kSelectThreads) bfasgd_mask_kernel(const __grid_constant__ SelectArgs a) {
@@ -77,24 +79,33 @@ __global__ void __launch_bounds__(kSelectThreads) bfasgd_mask_kernel(const __gri
     const int warp = threadIdx.x >> 5;
     const int64_t tile_start = (int64_t)blockIdx.x * kSelectTile;
     const int64_t warp_start = tile_start + (int64_t)warp * kWarpSpan;
-    int cnt = 0;
-#pragma unroll 2
+    // All of this lane's v loads first (eight quads), then the draws.
+    float4 v4[kIters];
+#pragma unroll
     for (int it = 0; it < kIters; ++it) {
         const int64_t e = warp_start + it * 128 + 4 * lane;  // first parameter of this quad
+        if (e + 3 < a.P) {
+            v4[it] = __ldcs(reinterpret_cast<const float4*>(a.v + e));
+        } else {
+            float t[4] = {0.f, 0.f, 0.f, 0.f};
+            for (int j = 0; j < 4; ++j)
+                if (e + j < a.P) t[j] = a.v[e + j];
+            v4[it] = make_float4(t[0], t[1], t[2], t[3]);
+        }
+    }
+    int cnt = 0;
+#pragma unroll
+    for (int it = 0; it < kIters; ++it) {
+        const int64_t e = warp_start + it * 128 + 4 * lane;
         uint32_t nib = 0;
         if (e < a.P) {
-            const Philox4 r = philox4x32_10((uint32_t)(e >> 2), a.client, a.push_lo, a.push_hi,
-                                            a.key0, a.key1);
-            if (e + 3 < a.P) {
-                const float4 v4 = __ldcs(reinterpret_cast<const float4*>(a.v + e));
-                nib = send_bit(r.x[0] >> 8, v4.x, a.c, a.eps_b) |
-                      (send_bit(r.x[1] >> 8, v4.y, a.c, a.eps_b) << 1) |
-                      (send_bit(r.x[2] >> 8, v4.z, a.c, a.eps_b) << 2) |
-                      (send_bit(r.x[3] >> 8, v4.w, a.c, a.eps_b) << 3);
-            } else {
-                for (int j = 0; j < 4; ++j)
-                    if (e + j < a.P) nib |= send_bit(r.x[j] >> 8, a.v[e + j], a.c, a.eps_b) << j;
-            }
+            const Philox4 r = philox4x32_10((uint32_t)(e >> 2), a.client, a.push_lo, a.push_hi, a);
+            nib = send_bit(r.x[0] >> 8, v4[it].x, a.c, a.eps_b) |
+                  (send_bit(r.x[1] >> 8, v4[it].y, a.c, a.eps_b) << 1) |
+                  (send_bit(r.x[2] >> 8, v4[it].z, a.c, a.eps_b) << 2) |
+                  (send_bit(r.x[3] >> 8, v4[it].w, a.c, a.eps_b) << 3);
+            const int64_t valid = a.P - e;  // parameters past P are never sent
+            if (valid < 4) nib &= (1u << valid) - 1u;
         }
         cnt += __popc(nib);
         // Eight lanes' nibbles form one 32-bit mask word (32 consecutive parameters).
@@ -160,8 +171,24 @@ __global__ void __launch_bounds__(kSelectThreads) bfasgd_compact_kernel(const __
     const int warp = threadIdx.x >> 5;
     const int64_t tile_start = (int64_t)blockIdx.x * kSelectTile;
     const int64_t warp_start = tile_start + (int64_t)warp * kWarpSpan;
-    // Lane l holds the mask word of parameters warp_start + 32 l .. + 31.
+    // Lane l holds the mask word of parameters warp_start + 32 l .. + 31.  The
+    // word, the tile's output base and the gradient quads are all loaded
+    // before anything waits on them.
     const uint32_t word = a.mask[(warp_start >> 5) + lane];
+    const int64_t tile_out = a.tile_base[blockIdx.x];
+    float4 g4[kIters];
+#pragma unroll
+    for (int it = 0; it < kIters; ++it) {
+        const int64_t e = warp_start + it * 128 + 4 * lane;
+        if (e + 3 < a.P) {
+            g4[it] = __ldcs(reinterpret_cast<const float4*>(a.grad + e));
+        } else {
+            float t[4] = {0.f, 0.f, 0.f, 0.f};
+            for (int j = 0; j < 4; ++j)
+                if (e + j < a.P) t[j] = a.grad[e + j];
+            g4[it] = make_float4(t[0], t[1], t[2], t[3]);
+        }
+    }
     const int c = __popc(word);
     int incl = c;
 #pragma unroll
@@ -172,9 +199,9 @@ __global__ void __launch_bounds__(kSelectThreads) bfasgd_compact_kernel(const __
     const int excl = incl - c;
     if (lane == 31) warp_cnt[warp] = incl;
     __syncthreads();
-    int64_t out = a.tile_base[blockIdx.x];
+    int64_t out = tile_out;
     for (int w = 0; w < warp; ++w) out += warp_cnt[w];
-#pragma unroll 2
+#pragma unroll
     for (int it = 0; it < kIters; ++it) {
         // This lane's quad lies in word (4 it + lane / 8), bits 4 (lane mod 8) .. +3.
         const int owner = it * 4 + (lane >> 3);
@@ -184,16 +211,7 @@ __global__ void __launch_bounds__(kSelectThreads) bfasgd_compact_kernel(const __
         const uint32_t nib = (w >> sh) & 0xFu;
         if (nib != 0) {
             const int64_t e = warp_start + it * 128 + 4 * lane;
-            float g[4];
-            if (e + 3 < a.P) {
-                const float4 g4 = __ldcs(reinterpret_cast<const float4*>(a.grad + e));
-                g[0] = g4.x;
-                g[1] = g4.y;
-                g[2] = g4.z;
-                g[3] = g4.w;
-            } else {
-                for (int j = 0; j < 4; ++j) g[j] = (e + j < a.P) ? a.grad[e + j] : 0.0f;
-            }
+            const float g[4] = {g4[it].x, g4[it].y, g4[it].z, g4[it].w};
             int64_t pos = out + wbase + __popc(w & ((1u << sh) - 1u));
 #pragma unroll
             for (int j = 0; j < 4; ++j) {
@@ -208,6 +226,16 @@ __global__ void __launch_bounds__(kSelectThreads) bfasgd_compact_kernel(const __
 }
 
 }  // namespace
+
+void select_key_schedule(SelectArgs& a, uint64_t seed) {
+    uint32_t k0 = (uint32_t)seed, k1 = (uint32_t)(seed >> 32);
+    for (int r = 0; r < 10; ++r) {
+        a.round_key0[r] = k0;
+        a.round_key1[r] = k1;
+        k0 += kPhiloxW0;
+        k1 += kPhiloxW1;
+    }
+}
 
 cudaError_t launch_select(const SelectArgs& a, cudaStream_t stream, int64_t* launches) {
     bfasgd_mask_kernel<<<a.ntiles, kSelectThreads, 0, stream>>>(a);
@@ -330,8 +358,7 @@ extern "C" int bfasgd_select_compact_noalloc(int64_t P, const float* grad, const
     a.ntiles = fasgd::select_tiles(P);
     a.c = c;
     a.eps_b = eps_b;
-    a.key0 = (uint32_t)seed;
-    a.key1 = (uint32_t)(seed >> 32);
+    fasgd::select_key_schedule(a, seed);
     a.client = (uint32_t)client;
     a.push_lo = (uint32_t)push_no;
     a.push_hi = (uint32_t)(push_no >> 32);

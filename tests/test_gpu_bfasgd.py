@@ -267,3 +267,30 @@ def test_select_max_p():
                     assert np.float32(vals[k]).view(np.uint32) == np.float32(g_s[k]).view(np.uint32)
         srv.close()
         del srv
+
+
+def test_select_at_the_threshold_bit_exact():
+    """Every parameter's v is set so that its Eq. 9 threshold falls within an
+    ulp of its own draw u_p (computed by the oracle): the decisions then hinge
+    on the exact comparison, which both sides must take identically."""
+    import torch
+    P = 40_000
+    c = 3.0
+    eps_b = 0.0
+    seed, client, push_no = 0xABCDEF, 2, 0
+    u = np.array([oracle.draw(seed, client, push_no, p) for p in range(P)], dtype=np.float64)
+    u = np.clip(u, 1, 2 ** 24 - 2)
+    # a / (a + c) = u / 2^24  <=>  a = c u / (2^24 - u); nudge by -1, 0, +1 ulp.
+    a = (c * u / (2.0 ** 24 - u)).astype(np.float32)
+    nudge = np.random.default_rng(7).integers(-1, 2, P)
+    a = np.nextafter(a, np.where(nudge > 0, np.inf, -np.inf).astype(np.float32)).astype(np.float32)
+    a = np.where(nudge == 0, (c * u / (2.0 ** 24 - u)).astype(np.float32), a)
+    v = a.astype(np.float32)
+    g = np.random.default_rng(8).standard_normal(P).astype(np.float32)
+    srv = _server(P, c=c, seed=seed)
+    srv.set_hparams(0.95, 0.95, 1e-4, c, eps_b, seed)
+    gi, gv, m, _ = _select_gpu(srv, client, torch.from_numpy(g).cuda(), torch.from_numpy(v).cuda())
+    oi, ov = oracle.select(g, v, c, eps_b, seed, client, push_no)
+    assert 0.2 * P < m < 0.8 * P          # the decisions really are split
+    assert_bitwise(gi, oi, "idx at threshold")
+    assert_bitwise(gv, ov, "val at threshold")
