@@ -77,6 +77,13 @@ def load_library(path: str, real: str) -> ctypes.CDLL:
     lib.ora_decide.argtypes = [u32, ctypes.c_float, ctypes.c_float, ctypes.c_float]
     lib.ora_select.restype = i64
     lib.ora_select.argtypes = [i64, P, P, ctypes.c_float, ctypes.c_float, u64, u32, u64, P, P]
+    lib.ora_draw_stream.restype = u32
+    lib.ora_draw_stream.argtypes = [u64, u32, u32, u64, i64]
+    lib.ora_fetch_select.restype = i64
+    lib.ora_fetch_select.argtypes = [i64, P, P, ctypes.c_float, ctypes.c_float, u64, u32, u64,
+                                     P, P]
+    lib.ora_fetch_apply.restype = None
+    lib.ora_fetch_apply.argtypes = [P, i64, P, P]
     assert lib.ora_real_bytes() == (4 if real == "f32" else 8)
     return lib
 
@@ -135,6 +142,33 @@ def select(g: np.ndarray, v: np.ndarray, c: float, eps_b: float, seed: int,
     return idx[:m].copy(), val[:m].copy()
 
 
+def draw_stream(seed: int, stream: int, client: int, n: int, p: int, lib=None) -> int:
+    """24-bit draw of parameter p for a client's n-th transmission of a stream
+    (0: push, 1: fetch)."""
+    return int((lib or _load("f32")).ora_draw_stream(seed, stream, client, n, p))
+
+
+def fetch_select(theta: np.ndarray, v: np.ndarray, c: float, eps_b: float, seed: int,
+                 client: int, fetch_no: int, lib=None):
+    """B-FASGD per-parameter fetch decision + compaction of theta; (idx, val)."""
+    th = np.ascontiguousarray(theta, dtype=np.float32)
+    v = np.ascontiguousarray(v, dtype=np.float32)
+    P = th.shape[0]
+    idx = np.empty(max(P, 1), dtype=np.int32)
+    val = np.empty(max(P, 1), dtype=np.float32)
+    m = (lib or _load("f32")).ora_fetch_select(P, _ptr(th), _ptr(v), c, eps_b, seed, client,
+                                               fetch_no, _ptr(idx), _ptr(val))
+    return idx[:m].copy(), val[:m].copy()
+
+
+def fetch_apply(theta_client: np.ndarray, idx: np.ndarray, val: np.ndarray, lib=None):
+    """Client side of a fetch: overwrite theta_client at idx with val (in place)."""
+    assert theta_client.dtype == np.float32 and theta_client.flags["C_CONTIGUOUS"]
+    i = np.ascontiguousarray(idx, dtype=np.int32)
+    x = np.ascontiguousarray(val, dtype=np.float32)
+    (lib or _load("f32")).ora_fetch_apply(_ptr(theta_client), i.shape[0], _ptr(i), _ptr(x))
+
+
 class OracleError(Exception):
     pass
 
@@ -162,6 +196,8 @@ class OracleServer:
         self.T = 0
         self.fifo: list = []
         self.push_count = [0] * lam
+        self.fetch_count = [0] * lam
+        self.c_fetch = 0.0
         self.set_hparams(gamma, beta, eps, c_push, eps_b, seed)
 
     def set_hparams(self, gamma, beta, eps, c_push, eps_b, seed):
@@ -219,6 +255,20 @@ class OracleServer:
         out = select(g, vv, self.c_push, self.eps_b, self.seed, client,
                      self.push_count[client], lib=self.lib if self.real == "f32" else None)
         self.push_count[client] += 1
+        return out
+
+    def set_fetch_threshold(self, c_fetch: float):
+        self.c_fetch = float(np.float32(c_fetch))
+
+    def fetch_compact(self, client: int, v: np.ndarray | None = None):
+        """B-FASGD fetch for one client: the kept (idx, theta[idx]) pairs."""
+        if not 0 <= client < self.lam:
+            raise OracleError("client out of range")
+        vv = (self.v if v is None else v).astype(np.float32)
+        out = fetch_select(self.theta.astype(np.float32), vv, self.c_fetch, self.eps_b,
+                           self.seed, client, self.fetch_count[client],
+                           lib=self.lib if self.real == "f32" else None)
+        self.fetch_count[client] += 1
         return out
 
     def pull(self):

@@ -19,7 +19,7 @@
  *   Eq. 1-2  (Sec. 2.1)  g = alpha(tau) * dtheta,  theta <- theta - g
  *   Eq. 4-6  (Sec. 2.2)  n, b moving averages; v moving average of 1/std
  *   Eq. 7-8  (Sec. 2.2)  theta <- theta - alpha / (v * tau) * dtheta
- *   Eq. 9    (Sec. 2.3)  transmit iff r < 1 / (1 + c / (v + eps))
+ *   Eq. 9    (Sec. 2.3)  transmit (push or fetch) iff r < 1 / (1 + c / (v + eps))
  * Readings where the paper is silent:
  *   tau = 0 divides by zero in Eq. 1 and Eq. 7: the divisor is max(tau, 1);
  *   n - b^2 can round below zero in floating point: it is clamped at 0
@@ -156,19 +156,28 @@ void ora_philox4x32_10(const uint32_t ctr_in[4], const uint32_t key_in[2], uint3
 }
 
 /*
- * The 24-bit uniform draw u_p for parameter p of one push.  The counter is
- * (p div 4, client, push# low word, push# high word), the key is the 64-bit
- * seed, and word (p mod 4) of the Philox output is used, shifted down to its
- * top 24 bits; r = u / 2^24 lies in [0, 1).
+ * The 24-bit uniform draw u_p for parameter p of one transmission.  The
+ * counter is (p div 4, client + 2^31 * stream, n low word, n high word),
+ * where n counts the client's earlier transmissions of that stream (stream
+ * 0: pushes, stream 1: fetches); the key is the 64-bit seed; word (p mod 4)
+ * of the Philox output is used, shifted down to its top 24 bits; r = u / 2^24
+ * lies in [0, 1).
  */
-uint32_t ora_draw(uint64_t seed, uint32_t client, uint64_t push_no, int64_t p)
+uint32_t ora_draw_stream(uint64_t seed, uint32_t stream, uint32_t client, uint64_t push_no,
+                         int64_t p)
 {
-    uint32_t ctr[4] = {(uint32_t)(p >> 2), client, (uint32_t)push_no,
+    uint32_t ctr[4] = {(uint32_t)(p >> 2), client | (stream << 31), (uint32_t)push_no,
                        (uint32_t)(push_no >> 32)};
     uint32_t key[2] = {(uint32_t)seed, (uint32_t)(seed >> 32)};
     uint32_t out[4];
     ora_philox4x32_10(ctr, key, out);
     return out[p & 3] >> 8;
+}
+
+/* The push decisions use stream 0, the fetch decisions (below) stream 1. */
+uint32_t ora_draw(uint64_t seed, uint32_t client, uint64_t push_no, int64_t p)
+{
+    return ora_draw_stream(seed, 0, client, push_no, p);
 }
 
 /*
@@ -201,13 +210,13 @@ int ora_decide(uint32_t u, float v, float c, float eps_b)
  * keep p iff Eq. 9 holds for v[p]; write idx[m] = p and val[m] = g[p]
  * (bit copy).  Returns the number m of parameters kept.
  */
-int64_t ora_select(int64_t P, const float *g, const float *v, float c, float eps_b,
-                   uint64_t seed, uint32_t client, uint64_t push_no,
-                   int32_t *idx, float *val)
+int64_t ora_select_stream(int64_t P, const float *g, const float *v, float c, float eps_b,
+                          uint64_t seed, uint32_t stream, uint32_t client, uint64_t push_no,
+                          int32_t *idx, float *val)
 {
     int64_t m = 0;
     for (int64_t p = 0; p < P; p++) {
-        uint32_t u = ora_draw(seed, client, push_no, p);
+        uint32_t u = ora_draw_stream(seed, stream, client, push_no, p);
         if (ora_decide(u, v[p], c, eps_b)) {
             idx[m] = (int32_t)p;
             val[m] = g[p];
@@ -215,4 +224,32 @@ int64_t ora_select(int64_t P, const float *g, const float *v, float c, float eps
         }
     }
     return m;
+}
+
+int64_t ora_select(int64_t P, const float *g, const float *v, float c, float eps_b,
+                   uint64_t seed, uint32_t client, uint64_t push_no,
+                   int32_t *idx, float *val)
+{
+    return ora_select_stream(P, g, v, c, eps_b, seed, 0, client, push_no, idx, val);
+}
+
+/*
+ * B-FASGD fetch, per parameter (Sec. 2.3: "given an opportunity to ...
+ * receive a parameter update", with the per-parameter extension of the
+ * future-work section): the server keeps p iff Eq. 9 holds for v[p] with the
+ * fetch threshold c (stream 1 draws) and sends (p, theta[p]); the client
+ * overwrites its copy at the kept indices and keeps computing with its own
+ * stale values everywhere else.
+ */
+int64_t ora_fetch_select(int64_t P, const float *theta, const float *v, float c, float eps_b,
+                         uint64_t seed, uint32_t client, uint64_t fetch_no,
+                         int32_t *idx, float *val)
+{
+    return ora_select_stream(P, theta, v, c, eps_b, seed, 1, client, fetch_no, idx, val);
+}
+
+void ora_fetch_apply(float *theta_client, int64_t count, const int32_t *idx, const float *val)
+{
+    for (int64_t i = 0; i < count; i++)
+        theta_client[idx[i]] = val[i];
 }

@@ -414,6 +414,61 @@ def check_sparse_leaves_unsent_untouched(libs: Libs):
         assert not np.array_equal(x[idx], y[idx])
 
 
+def check_fetch_path(libs: Libs):
+    """B-FASGD per-parameter fetch: Eq. 9 with the fetch threshold on its own
+    draw stream; the client overwrites only the fetched parameters."""
+    rng = np.random.default_rng(31)
+    P = 12001
+    theta = (rng.standard_normal(P) * 0.01).astype(np.float32)
+    v = (10 ** rng.uniform(-1, 2, P)).astype(np.float32)
+    seed, eps_b = 4242, 1e-8
+    # c = 0 fetches everything: the client ends up with the server's theta.
+    idx, val = oracle.fetch_select(theta, v, 0.0, eps_b, seed, 2, 0, lib=libs.f32)
+    assert np.array_equal(idx, np.arange(P, dtype=np.int32))
+    client = np.zeros(P, np.float32)
+    oracle.fetch_apply(client, idx, val, lib=libs.f32)
+    assert np.array_equal(client.view(np.uint32), theta.view(np.uint32))
+    # c = inf fetches nothing.
+    idx, _ = oracle.fetch_select(theta, v, float("inf"), eps_b, seed, 2, 0, lib=libs.f32)
+    assert idx.size == 0
+    # Moderate c: exact Eq. 9 membership on the fetch stream, binomial count,
+    # unfetched client entries untouched.
+    for c in (5.0, 40.0):
+        idx, val = oracle.fetch_select(theta, v, c, eps_b, seed, 3, 7, lib=libs.f32)
+        assert np.all(np.diff(idx.astype(np.int64)) > 0)
+        assert np.array_equal(val.view(np.uint32), theta[idx].view(np.uint32))
+        a = v.astype(np.float64) + eps_b
+        t = 1.0 / (1.0 + c / a)
+        assert abs(idx.size - t.sum()) <= 5 * math.sqrt((t * (1 - t)).sum())
+        keep = np.zeros(P, bool)
+        keep[idx] = True
+        for p in rng.choice(P, 300, replace=False):
+            u = oracle.draw_stream(seed, 1, 3, 7, int(p), lib=libs.f32)
+            assert _exact_decide(u, v[p], c, eps_b) == keep[p]
+        stale = np.full(P, 7.0, np.float32)
+        oracle.fetch_apply(stale, idx, val, lib=libs.f32)
+        assert np.all(stale[~keep] == 7.0) and np.array_equal(stale[keep], theta[keep])
+    # The fetch stream is not the push stream.
+    same = [oracle.draw_stream(seed, 0, 3, 7, p, lib=libs.f32) ==
+            oracle.draw_stream(seed, 1, 3, 7, p, lib=libs.f32) for p in range(2000)]
+    assert sum(same) < 5
+    assert oracle.draw_stream(seed, 0, 3, 7, 11, lib=libs.f32) == oracle.draw(seed, 3, 7, 11,
+                                                                              lib=libs.f32)
+
+
+def check_server_fetch_counters(libs: Libs):
+    s = _server(libs, "f32", 64, FASGD, lam=3)
+    s.set_fetch_threshold(1.0)
+    g = np.ones(64, np.float32)
+    s.select_compact(1, g)
+    s.fetch_compact(1)
+    s.fetch_compact(1)
+    assert s.push_count == [0, 1, 0] and s.fetch_count == [0, 2, 0]
+    a = s.fetch_compact(2)
+    b = oracle.fetch_select(s.theta, s.v, 1.0, s.eps_b, s.seed, 2, 0, lib=libs.f32)
+    assert np.array_equal(a[0], b[0])
+
+
 def check_protocol_errors(libs: Libs):
     s = _server(libs, "f32", 4, FASGD, lam=2)
     g = np.zeros(4, np.float32)
@@ -452,5 +507,7 @@ ALL_CHECKS = [
     check_select_properties,
     check_bfasgd_c0_equals_fasgd,
     check_sparse_leaves_unsent_untouched,
+    check_fetch_path,
+    check_server_fetch_counters,
     check_protocol_errors,
 ]

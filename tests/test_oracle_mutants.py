@@ -40,7 +40,11 @@ MUTANTS = {
     "philox_mult_constant": ("mult1 = 0xCD9E8D57u", "mult1 = 0xCD9E8D55u"),
     "draw_wrong_word": ("out[p & 3] >> 8", "out[(p + 1) & 3] >> 8"),
     "draw_low_bits": ("out[p & 3] >> 8", "out[p & 3] & 0xFFFFFFu"),
-    "draw_counter_no_client": ("(uint32_t)(p >> 2), client,", "(uint32_t)(p >> 2), 0u,"),
+    "draw_counter_no_client": ("client | (stream << 31)", "0u | (stream << 31)"),
+    "draw_streams_collide": ("client | (stream << 31)", "client"),
+    "fetch_uses_push_stream": ("return ora_select_stream(P, theta, v, c, eps_b, seed, 1,",
+                               "return ora_select_stream(P, theta, v, c, eps_b, seed, 0,"),
+    "fetch_apply_wrong_slot": ("theta_client[idx[i]] = val[i];", "theta_client[i] = val[i];"),
     "decide_not_strict": ("prod == A && err < 0.0f", "prod == A && err <= 0.0f"),
     "decide_ignores_err": ("if (prod == A && err < 0.0f)\n        return 1;\n", ""),
     "decide_drops_eps": ("float a = v + eps_b;", "float a = v;"),
