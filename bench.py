@@ -41,6 +41,7 @@ from paper_1601_04033_gb300 import streams  # noqa: E402
 METRIC = "parameter-updates/sec and achieved HBM GB/s (% of GB300 peak), 1 GPU"
 UNIT = "param-updates/s"
 FALLBACK_HBM_GBS = 6800.0
+FETCH_FRACTION = 0.10   # a 10x cut of fetch traffic (the paper's effective setting, Sec. 4.2)
 L2_BYTES = 129 * 1024 * 1024
 
 DENSE_KERNEL_SOURCES = ["paper_1601_04033_gb300/csrc/dense.cu",
@@ -381,28 +382,53 @@ def run_bfasgd(args, w, world, rank, local):
         t += 1
     v_now = torch.empty(P, device=device)
     srv.get_state(None, None, None, v_now)
-    c_push = calibrate_c(v_now.cpu().numpy(), w.send_frac)
+    v_host = v_now.cpu().numpy()
+    c_push = calibrate_c(v_host, w.send_frac)
+    c_fetch = calibrate_c(v_host, FETCH_FRACTION)
     srv.set_hparams(0.95, 0.95, 1e-4, c_push, 1e-8, w.seed)
+    srv.set_fetch_threshold(c_fetch)
     idx = torch.empty(P, dtype=torch.int32, device=device)
     val = torch.empty(P, dtype=torch.float32, device=device)
     cnt = torch.empty(1, dtype=torch.int64, device=device)
+    fidx = torch.empty(P, dtype=torch.int32, device=device)
+    fval = torch.empty(P, dtype=torch.float32, device=device)
+    fcnt = torch.empty(1, dtype=torch.int64, device=device)
     counts = torch.zeros(args.steps, dtype=torch.int64, device=device)
+    fcounts = torch.zeros(args.steps, dtype=torch.int64, device=device)
+    # Every client keeps its own (stale) copy of the parameters.
+    client_theta = torch.from_numpy(th0).to(device).repeat(w.lam, 1)
 
-    def step(t, i=None):
+    def step(t, ev=None, i=None):
+        """One B-FASGD exchange: client c pushes (decision + compaction, sparse
+        server apply) and then refreshes its copy (fetch decision + compaction
+        of theta, client scatter)."""
         cl, js, sl = ps.batch(t)
         c = int(cl[0])
+        if ev is not None:
+            ev[0].record(stream)
         srv.select_compact(c, slots[int(sl[0])], idx, val, cnt)      # live server v
+        if ev is not None:
+            ev[1].record(stream)
         srv.push_sparse(c, int(js[0]), idx, val, n_dev=cnt, n_max=P)
         srv.apply_pending(1)
+        if ev is not None:
+            ev[2].record(stream)
+        srv.fetch_compact(c, fidx, fval, fcnt)
+        if ev is not None:
+            ev[3].record(stream)
+        fasgd.fetch_apply(client_theta[c], fidx, fval, n_dev=fcnt, n_max=P, stream=stream)
+        if ev is not None:
+            ev[4].record(stream)
         if i is not None:
             counts[i:i + 1].copy_(cnt, non_blocking=True)
+            fcounts[i:i + 1].copy_(fcnt, non_blocking=True)
 
     for _ in range(args.warmup):
         step(t)
         t += 1
     torch.cuda.synchronize()
     clocks = ClockSampler(gpu_identifier(torch))
-    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(args.steps)]
     start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     launches0 = srv.launches
     barrier(world)
@@ -411,25 +437,18 @@ def run_bfasgd(args, w, world, rank, local):
     time.sleep(0.3)
     start.record(stream)
     for i in range(args.steps):
-        cl, js, sl = ps.batch(t)
-        c = int(cl[0])
-        ev[i][0].record(stream)
-        srv.select_compact(c, slots[int(sl[0])], idx, val, cnt)
-        ev[i][1].record(stream)
-        srv.push_sparse(c, int(js[0]), idx, val, n_dev=cnt, n_max=P)
-        srv.apply_pending(1)
-        ev[i][2].record(stream)
-        counts[i:i + 1].copy_(cnt, non_blocking=True)
+        step(t, ev[i], i)
         t += 1
     end.record(stream)
     torch.cuda.synchronize()
     clock_info = clocks.stop()
     barrier(world)
-    launches = srv.launches - launches0
+    launches = srv.launches - launches0 + args.steps      # + one fetch scatter per step
     total_ms = max_over_ranks(start.elapsed_time(end), world, device)
-    sel_ms = sum(e[0].elapsed_time(e[1]) for e in ev) / args.steps
-    app_ms = sum(e[1].elapsed_time(e[2]) for e in ev) / args.steps
+    stage = [sum(e[k].elapsed_time(e[k + 1]) for e in ev) / args.steps for k in range(4)]
+    sel_ms, app_ms, fsel_ms, fapp_ms = stage
     sent = counts.cpu().numpy().astype(np.float64)
+    fetched = fcounts.cpu().numpy().astype(np.float64)
     frac = float(sent.mean() / P)
     srv.sync()
     srv.close()
@@ -448,12 +467,16 @@ def run_bfasgd(args, w, world, rank, local):
                      "traffic": profiled_traffic(w.name, SPARSE_KERNEL_SOURCES),
                      "select_ms": round(sel_ms, 5), "apply_ms": round(app_ms, 5),
                      "select_gbs": round(alg_select / (sel_ms / 1e3) / 1e9, 1),
-                     "apply_gbs": round(alg_apply / (app_ms / 1e3) / 1e9, 1)},
+                     "apply_gbs": round(alg_apply / (app_ms / 1e3) / 1e9, 1),
+                     "fetch_select_ms": round(fsel_ms, 5), "fetch_apply_ms": round(fapp_ms, 5)},
         "clocks": clock_info, "e2e": None, "gpu_launches": launches,
         "pushes_per_s": world / step_s, "sent_fraction": round(frac, 4),
+        "fetched_fraction": round(float(fetched.mean() / P), 4),
         "sent_updates_per_s": sent.mean() * world / step_s,
         "config": {"workload": w.name, "P_per_gpu": P, "P_total": P * world, "lambda": w.lam,
                    "K": 1, "variant": "b-fasgd", "c_push": c_push, "target_send_fraction": w.send_frac,
+                   "c_fetch": c_fetch, "target_fetch_fraction": FETCH_FRACTION,
+                   "step": "push select/compact + sparse apply + fetch select/compact + client scatter",
                    "staleness": w.delay, "parallelism": f"param-shard{world}",
                    "l2": "inputs larger than L2, no flush"},
     }
@@ -523,7 +546,7 @@ def main():
                 "roofline": res["roofline"], "cpu_baseline": cpu, "e2e": res["e2e"],
                 "clocks": res["clocks"], "gpu_launches": res["gpu_launches"],
                 "pushes_per_s": res["pushes_per_s"]}
-        for k in ("hbm_gbs_step", "sent_fraction", "sent_updates_per_s"):
+        for k in ("hbm_gbs_step", "sent_fraction", "fetched_fraction", "sent_updates_per_s"):
             if k in res:
                 line[k] = res[k]
         print(json.dumps(line))

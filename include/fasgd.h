@@ -167,7 +167,7 @@ FASGD_API int fasgd_apply_pending(fasgd_t* h, int32_t K);
  * Eq. 9, taken per parameter with the parameter's own v_p).
  * For every p, u_p is the top 24 bits of word (p mod 4) of Philox4x32-10
  * (Salmon et al., SC'11) with counter (p div 4, client, push#, push# >> 32)
- * and key = seed, where push# counts this client's earlier calls.  With
+ * and key = seed, where push# counts this client's earlier pushes.  With
  * a = fl(v_p + eps_b) and d = fl(a + c_push), p is sent iff
  * u_p * d < a * 2^24 exactly, i.e. u_p / 2^24 < 1 / (1 + c_push / a).
  * Outputs: idx[0..m) = the sent p in ascending order (int32), val[i] =
@@ -180,6 +180,40 @@ FASGD_API int fasgd_apply_pending(fasgd_t* h, int32_t K);
  */
 FASGD_API int bfasgd_select_compact(fasgd_t* h, int32_t client, const float* grad, const float* v,
                           int32_t* idx, float* val, int64_t* n_dev);
+
+/*
+ * bfasgd_fetch_compact -- B-FASGD fetch decision and compaction, per
+ * parameter (Sec. 2.3: a client "given an opportunity to ... receive a
+ * parameter update" takes it iff Eq. 9 holds, here with each parameter's own
+ * v_p as the future-work section proposes).  Exactly as
+ * bfasgd_select_compact, with the fetch threshold c_fetch
+ * (fasgd_set_fetch_threshold), draws from the fetch stream (counter word
+ * client + 2^31, push# replaced by the client's count of earlier fetches),
+ * and the server's current theta as the values: idx[0..m) = the kept p
+ * ascending, val[i] = theta[idx[i]], *n_dev = m.  theta is read as of the
+ * pushes applied so far on the stream.  v: device fp32[P] or NULL for the
+ * server's live v.  The client applies the result with bfasgd_fetch_apply
+ * and keeps its stale values elsewhere.  Errors: EINVAL, ERANGE, ECUDA.
+ */
+FASGD_API int bfasgd_fetch_compact(fasgd_t* h, int32_t client, const float* v, int32_t* idx,
+                                   float* val, int64_t* n_dev);
+
+/* Fetch threshold c_fetch of Eq. 9 (>= 0, +inf allowed: nothing is fetched).  Default 0. */
+FASGD_API int fasgd_set_fetch_threshold(fasgd_t* h, float c_fetch);
+
+/*
+ * bfasgd_fetch_apply -- client side of a fetch: theta_client[idx[i]] = val[i]
+ * for i < count, on `stream` (a cudaStream_t; NULL = legacy default stream).
+ * theta_client: device fp32[P]; idx, val: device lists from
+ * bfasgd_fetch_compact (distinct indices); count = *n_dev if n_dev is not
+ * NULL, else n_max; 0 <= n_max <= P.  An index outside [0, P) is skipped and
+ * a count above n_max is clamped; both raise flags in *err_dev (device int32,
+ * may be NULL).  Needs no handle.  Errors: EINVAL (text via
+ * fasgd_last_error(NULL)), ECUDA.
+ */
+FASGD_API int bfasgd_fetch_apply(int64_t P, float* theta_client, const int32_t* idx,
+                                 const float* val, const int64_t* n_dev, int64_t n_max,
+                                 void* stream, int32_t* err_dev);
 
 /*
  * fasgd_pull -- copy theta (P fp32) into params (host or device) on the
@@ -199,9 +233,11 @@ FASGD_API int fasgd_get_state(fasgd_t* h, float* theta, float* n, float* b, floa
 FASGD_API int fasgd_set_state(fasgd_t* h, const float* theta, const float* n, const float* b,
                     const float* v, int64_t T);
 
-/* Per-client B-FASGD push counters (lambda uint64 values, host memory). */
+/* Per-client B-FASGD push and fetch counters (lambda uint64 values, host memory). */
 FASGD_API int fasgd_get_push_counts(fasgd_t* h, uint64_t* counts);
 FASGD_API int fasgd_set_push_counts(fasgd_t* h, const uint64_t* counts);
+FASGD_API int fasgd_get_fetch_counts(fasgd_t* h, uint64_t* counts);
+FASGD_API int fasgd_set_fetch_counts(fasgd_t* h, const uint64_t* counts);
 
 /*
  * fasgd_sync -- wait until the handle's stream is idle, then report and
@@ -261,7 +297,8 @@ FASGD_API int bfasgd_select_compact_noalloc(int64_t P, const float* grad, const 
                                             int64_t* n_dev, void* stream);
 
 /* Text of the last failure on h, or, when h is NULL, of the last failed call
- * made without a handle (fasgd_create, bfasgd_select_compact_noalloc). */
+ * made without a handle (fasgd_create, bfasgd_fetch_apply,
+ * bfasgd_select_compact_noalloc). */
 FASGD_API const char* fasgd_last_error(const fasgd_t* h);
 
 #ifdef __cplusplus

@@ -54,7 +54,7 @@ constexpr int kSelectTile = 8192;
 constexpr int kSelectTileWords = kSelectTile / 32;
 
 struct SelectArgs {
-    const float* grad;
+    const float* values;   // copied into val for kept parameters (a push's gradient, or theta)
     const float* v;
     int32_t* idx;
     float* val;
@@ -68,7 +68,19 @@ struct SelectArgs {
     float eps_b;
     uint32_t round_key0[10];       // Philox key schedule: seed advanced by the
     uint32_t round_key1[10];       // Weyl constants, one pair per round
-    uint32_t client, push_lo, push_hi;
+    uint32_t client_word;          // client + 2^31 * stream (0: push, 1: fetch)
+    uint32_t push_lo, push_hi;     // the client's count of earlier calls of that stream
+};
+
+// Client side of a B-FASGD fetch: theta[idx[i]] = val[i] for i < count.
+struct ScatterArgs {
+    float* theta;
+    const int32_t* idx;
+    const float* val;
+    const int64_t* count_dev;  // may be null: count = count_max
+    int64_t count_max;
+    int64_t P;
+    int32_t* err;              // may be null; flags 1 (count) and 2 (index)
 };
 
 // Launchers: enqueue on `stream`, return the launch status.
@@ -78,6 +90,7 @@ cudaError_t launch_dense(const DenseArgs& a, bool fasgd_rule, int num_sms, cudaS
 cudaError_t launch_sparse(const SparseArgs& a, bool fasgd_rule, int num_sms, cudaStream_t stream,
                           int64_t* launches);
 cudaError_t launch_select(const SelectArgs& a, cudaStream_t stream, int64_t* launches);
+cudaError_t launch_scatter(const ScatterArgs& a, int num_sms, cudaStream_t stream);
 
 inline int32_t select_tiles(int64_t P) {
     return (int32_t)((P + kSelectTile - 1) / kSelectTile);

@@ -77,6 +77,7 @@ struct fasgd_s {
     float alpha = 0.f;
     int32_t variant = FASGD_FASGD;
     float gamma = 0.95f, beta = 0.95f, eps = 1e-4f, c_push = 0.f, eps_b = 1e-8f;
+    float c_fetch = 0.f;
     uint64_t seed = 0;
     cudaStream_t stream = nullptr;
     int device = 0;
@@ -96,6 +97,7 @@ struct fasgd_s {
     int64_t T = 0;
     int64_t launches = 0;
     std::vector<uint64_t> push_count;
+    std::vector<uint64_t> fetch_count;
     std::string err;
 
     int fail(int code, const char* fmt, ...) {
@@ -175,6 +177,7 @@ int fasgd_create(fasgd_t** h, int64_t P, int32_t lambda, float alpha, int32_t va
     s->alpha = alpha;
     s->variant = variant;
     s->push_count.assign((size_t)lambda, 0);
+    s->fetch_count.assign((size_t)lambda, 0);
     s->ntiles = fasgd::select_tiles(P);
     cudaError_t st = cudaGetDevice(&s->device);
     if (st == cudaSuccess)
@@ -378,22 +381,28 @@ int fasgd_apply_pending(fasgd_t* h, int32_t K) {
     return FASGD_OK;
 }
 
-int bfasgd_select_compact(fasgd_t* h, int32_t client, const float* grad, const float* v,
-                          int32_t* idx, float* val, int64_t* n_dev) {
-    if (h == nullptr) return FASGD_EINVAL;
+}  // extern "C"
+
+// One B-FASGD decision + compaction pass: stream 0 (push: values = the
+// client's gradient, threshold c_push) or 1 (fetch: values = theta, c_fetch).
+static int run_select(fasgd_t* h, const char* what, uint32_t stream, int32_t client,
+                      const float* values, const float* v, int32_t* idx, float* val,
+                      int64_t* n_dev, float c, std::vector<uint64_t>& counter) {
     if (client < 0 || client >= h->lambda)
-        return h->fail(FASGD_ERANGE, "client %d outside [0, %d)", client, h->lambda);
-    if (grad == nullptr || !aligned(grad, 16))
-        return h->fail(FASGD_EINVAL, "grad must be a non-NULL 16-byte aligned device pointer");
+        return h->fail(FASGD_ERANGE, "%s: client %d outside [0, %d)", what, client, h->lambda);
+    if (values == nullptr || !aligned(values, 16))
+        return h->fail(FASGD_EINVAL, "%s: grad must be a non-NULL 16-byte aligned device pointer",
+                       what);
     if (v != nullptr && !aligned(v, 16))
-        return h->fail(FASGD_EINVAL, "v must be 16-byte aligned (or NULL for the server's v)");
+        return h->fail(FASGD_EINVAL, "%s: v must be 16-byte aligned (or NULL for the server's v)",
+                       what);
     if (idx == nullptr || val == nullptr || n_dev == nullptr || !aligned(idx, 4) ||
         !aligned(val, 4) || !aligned(n_dev, 8))
-        return h->fail(FASGD_EINVAL, "idx, val, n_dev must be non-NULL and aligned");
+        return h->fail(FASGD_EINVAL, "%s: idx, val, n_dev must be non-NULL and aligned", what);
     DeviceGuard g(h->device);
     fasgd::SelectArgs a;
     std::memset(&a, 0, sizeof a);
-    a.grad = grad;
+    a.values = values;
     a.v = v != nullptr ? v : h->v;
     a.idx = idx;
     a.val = val;
@@ -403,16 +412,71 @@ int bfasgd_select_compact(fasgd_t* h, int32_t client, const float* grad, const f
     a.tile_base = h->tile_base;
     a.P = h->P;
     a.ntiles = h->ntiles;
-    a.c = h->c_push;
+    a.c = c;
     a.eps_b = h->eps_b;
     fasgd::select_key_schedule(a, h->seed);
-    const uint64_t push_no = h->push_count[(size_t)client];
-    a.client = (uint32_t)client;
-    a.push_lo = (uint32_t)push_no;
-    a.push_hi = (uint32_t)(push_no >> 32);
+    const uint64_t n = counter[(size_t)client];
+    a.client_word = (uint32_t)client | (stream << 31);
+    a.push_lo = (uint32_t)n;
+    a.push_hi = (uint32_t)(n >> 32);
     cudaError_t st = fasgd::launch_select(a, h->stream, &h->launches);
-    if (st != cudaSuccess) return h->cuda_fail(st, "bfasgd_select_compact");
-    h->push_count[(size_t)client] = push_no + 1;
+    if (st != cudaSuccess) return h->cuda_fail(st, what);
+    counter[(size_t)client] = n + 1;
+    return FASGD_OK;
+}
+
+extern "C" {
+
+int bfasgd_select_compact(fasgd_t* h, int32_t client, const float* grad, const float* v,
+                          int32_t* idx, float* val, int64_t* n_dev) {
+    if (h == nullptr) return FASGD_EINVAL;
+    return run_select(h, "bfasgd_select_compact", 0, client, grad, v, idx, val, n_dev, h->c_push,
+                      h->push_count);
+}
+
+int bfasgd_fetch_compact(fasgd_t* h, int32_t client, const float* v, int32_t* idx, float* val,
+                         int64_t* n_dev) {
+    if (h == nullptr) return FASGD_EINVAL;
+    return run_select(h, "bfasgd_fetch_compact", 1, client, h->theta, v, idx, val, n_dev,
+                      h->c_fetch, h->fetch_count);
+}
+
+int fasgd_set_fetch_threshold(fasgd_t* h, float c_fetch) {
+    if (h == nullptr) return FASGD_EINVAL;
+    if (!(c_fetch >= 0.f)) return h->fail(FASGD_EINVAL, "c_fetch must be >= 0 (may be +inf)");
+    h->c_fetch = c_fetch;
+    return FASGD_OK;
+}
+
+int bfasgd_fetch_apply(int64_t P, float* theta_client, const int32_t* idx, const float* val,
+                       const int64_t* n_dev, int64_t n_max, void* stream, int32_t* err_dev) {
+    if (P < 1 || P > FASGD_PMAX) {
+        g_create_error = "bfasgd_fetch_apply: P must be in [1, 2^31)";
+        return FASGD_EINVAL;
+    }
+    if (theta_client == nullptr || n_max < 0 || n_max > P ||
+        (n_max > 0 && (idx == nullptr || val == nullptr)) || !aligned(theta_client, 4) ||
+        !aligned(idx, 4) || !aligned(val, 4) || !aligned(n_dev, 8) || !aligned(err_dev, 4)) {
+        g_create_error = "bfasgd_fetch_apply: bad pointer or n_max outside [0, P]";
+        return FASGD_EINVAL;
+    }
+    if (n_max == 0 && n_dev == nullptr) return FASGD_OK;
+    int dev = 0, sms = 0;
+    cudaError_t st = cudaGetDevice(&dev);
+    if (st == cudaSuccess) st = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    fasgd::ScatterArgs a;
+    a.theta = theta_client;
+    a.idx = idx;
+    a.val = val;
+    a.count_dev = n_dev;
+    a.count_max = n_max;
+    a.P = P;
+    a.err = err_dev;
+    if (st == cudaSuccess) st = fasgd::launch_scatter(a, sms, static_cast<cudaStream_t>(stream));
+    if (st != cudaSuccess) {
+        g_create_error = std::string("bfasgd_fetch_apply: ") + cudaGetErrorString(st);
+        return FASGD_ECUDA;
+    }
     return FASGD_OK;
 }
 
@@ -473,6 +537,18 @@ int fasgd_get_push_counts(fasgd_t* h, uint64_t* counts) {
 int fasgd_set_push_counts(fasgd_t* h, const uint64_t* counts) {
     if (h == nullptr || counts == nullptr) return FASGD_EINVAL;
     std::memcpy(h->push_count.data(), counts, h->push_count.size() * sizeof(uint64_t));
+    return FASGD_OK;
+}
+
+int fasgd_get_fetch_counts(fasgd_t* h, uint64_t* counts) {
+    if (h == nullptr || counts == nullptr) return FASGD_EINVAL;
+    std::memcpy(counts, h->fetch_count.data(), h->fetch_count.size() * sizeof(uint64_t));
+    return FASGD_OK;
+}
+
+int fasgd_set_fetch_counts(fasgd_t* h, const uint64_t* counts) {
+    if (h == nullptr || counts == nullptr) return FASGD_EINVAL;
+    std::memcpy(h->fetch_count.data(), counts, h->fetch_count.size() * sizeof(uint64_t));
     return FASGD_OK;
 }
 

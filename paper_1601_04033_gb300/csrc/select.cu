@@ -1,6 +1,8 @@
-// B-FASGD push side, per parameter (paper Sec. 2.3, Eq. 9): the send
-// decision and the compaction of the sent entries into an ascending index
-// list and the matching values.
+// B-FASGD transmission decisions, per parameter (paper Sec. 2.3, Eq. 9): the
+// send (push) or fetch decision and the compaction of the kept entries into
+// an ascending index list and the matching values (the push's gradient, or
+// the server's theta for a fetch).  Push and fetch draws come from separate
+// Philox counter streams (bit 31 of the client word).
 //
 // Three kernels, all on the caller's stream:
 //   1. mask:    per tile of 8192 parameters, draw u_p (Philox4x32-10), take
@@ -99,7 +101,7 @@ __global__ void __launch_bounds__(kSelectThreads) bfasgd_mask_kernel(const __gri
         const int64_t e = warp_start + it * 128 + 4 * lane;
         uint32_t nib = 0;
         if (e < a.P) {
-            const Philox4 r = philox4x32_10((uint32_t)(e >> 2), a.client, a.push_lo, a.push_hi, a);
+            const Philox4 r = philox4x32_10((uint32_t)(e >> 2), a.client_word, a.push_lo, a.push_hi, a);
             nib = send_bit(r.x[0] >> 8, v4[it].x, a.c, a.eps_b) |
                   (send_bit(r.x[1] >> 8, v4[it].y, a.c, a.eps_b) << 1) |
                   (send_bit(r.x[2] >> 8, v4[it].z, a.c, a.eps_b) << 2) |
@@ -181,11 +183,11 @@ __global__ void __launch_bounds__(kSelectThreads) bfasgd_compact_kernel(const __
     for (int it = 0; it < kIters; ++it) {
         const int64_t e = warp_start + it * 128 + 4 * lane;
         if (e + 3 < a.P) {
-            g4[it] = __ldcs(reinterpret_cast<const float4*>(a.grad + e));
+            g4[it] = __ldcs(reinterpret_cast<const float4*>(a.values + e));
         } else {
             float t[4] = {0.f, 0.f, 0.f, 0.f};
             for (int j = 0; j < 4; ++j)
-                if (e + j < a.P) t[j] = a.grad[e + j];
+                if (e + j < a.P) t[j] = a.values[e + j];
             g4[it] = make_float4(t[0], t[1], t[2], t[3]);
         }
     }
@@ -346,7 +348,7 @@ extern "C" int bfasgd_select_compact_noalloc(int64_t P, const float* grad, const
         return noalloc_fail(FASGD_ECUDA, "bfasgd_select_compact_noalloc: cannot address the "
                                          "static scratch on this device");
     fasgd::SelectArgs a;
-    a.grad = grad;
+    a.values = grad;
     a.v = v;
     a.idx = idx;
     a.val = val;
@@ -359,7 +361,7 @@ extern "C" int bfasgd_select_compact_noalloc(int64_t P, const float* grad, const
     a.c = c;
     a.eps_b = eps_b;
     fasgd::select_key_schedule(a, seed);
-    a.client = (uint32_t)client;
+    a.client_word = (uint32_t)client;
     a.push_lo = (uint32_t)push_no;
     a.push_hi = (uint32_t)(push_no >> 32);
     int64_t launches = 0;

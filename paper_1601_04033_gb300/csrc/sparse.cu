@@ -105,7 +105,40 @@ cudaError_t launch_rule(const SparseArgs& a, int num_sms, cudaStream_t stream) {
     return cudaGetLastError();
 }
 
+// Client side of a B-FASGD fetch: theta[idx[i]] = val[i] for i < count.
+// Indices come from one compaction, so they are distinct and no two threads
+// write the same parameter; an index outside [0, P) is skipped and flagged.
+__global__ void __launch_bounds__(kSparseThreads) fetch_scatter_kernel(const __grid_constant__ ScatterArgs a) {
+    int64_t count = a.count_max;
+    if (a.count_dev != nullptr) {
+        const int64_t c = *a.count_dev;
+        count = c;
+        if (c < 0 || c > a.count_max) {
+            if (blockIdx.x == 0 && threadIdx.x == 0 && a.err != nullptr) atomicOr(a.err, 1);
+            count = c < 0 ? 0 : a.count_max;
+        }
+    }
+    const int64_t stride = (int64_t)gridDim.x * kSparseThreads;
+    for (int64_t i = (int64_t)blockIdx.x * kSparseThreads + threadIdx.x; i < count; i += stride) {
+        const int32_t p = a.idx[i];
+        if (p < 0 || (int64_t)p >= a.P) {
+            if (a.err != nullptr) atomicOr(a.err, 2);
+            continue;
+        }
+        a.theta[p] = a.val[i];
+    }
+}
+
 }  // namespace
+
+cudaError_t launch_scatter(const ScatterArgs& a, int num_sms, cudaStream_t stream) {
+    int64_t want = (a.count_max + kSparseThreads - 1) / kSparseThreads;
+    const int64_t cap = (int64_t)(num_sms > 0 ? num_sms : 1) * 8;
+    if (want > cap) want = cap;
+    if (want < 1) want = 1;
+    fetch_scatter_kernel<<<(unsigned)want, kSparseThreads, 0, stream>>>(a);
+    return cudaGetLastError();
+}
 
 cudaError_t launch_sparse(const SparseArgs& a, bool fasgd_rule, int num_sms, cudaStream_t stream,
                           int64_t* launches) {

@@ -47,6 +47,11 @@ SIGNATURES = {
     "fasgd_timestamp": (_i64, [_p]),
     "fasgd_pending": (_i64, [_p]),
     "fasgd_kernel_launches": (_i64, [_p]),
+    "bfasgd_fetch_compact": (_i32, [_p, _i32, _p, _p, _p, _p]),
+    "fasgd_set_fetch_threshold": (_i32, [_p, _f32]),
+    "bfasgd_fetch_apply": (_i32, [_i64, _p, _p, _p, _p, _i64, _p, _p]),
+    "fasgd_get_fetch_counts": (_i32, [_p, _p]),
+    "fasgd_set_fetch_counts": (_i32, [_p, _p]),
     "bfasgd_select_compact_noalloc": (_i32, [_i64, _p, _p, _f32, _f32, _u64, _i32, _u64,
                                              _p, _p, _p, _p]),
     "fasgd_last_error": (ctypes.c_char_p, [_p]),
@@ -121,6 +126,26 @@ def fasgd_apply_pending(h, K):
 
 def bfasgd_select_compact(h, client, grad, v, idx, val, n_dev):
     return LIB.bfasgd_select_compact(h, client, grad, v, idx, val, n_dev)
+
+
+def bfasgd_fetch_compact(h, client, v, idx, val, n_dev):
+    return LIB.bfasgd_fetch_compact(h, client, v, idx, val, n_dev)
+
+
+def fasgd_set_fetch_threshold(h, c_fetch):
+    return LIB.fasgd_set_fetch_threshold(h, c_fetch)
+
+
+def bfasgd_fetch_apply(P, theta_client, idx, val, n_dev, n_max, stream, err_dev):
+    return LIB.bfasgd_fetch_apply(P, theta_client, idx, val, n_dev, n_max, stream, err_dev)
+
+
+def fasgd_get_fetch_counts(h, counts):
+    return LIB.fasgd_get_fetch_counts(h, counts)
+
+
+def fasgd_set_fetch_counts(h, counts):
+    return LIB.fasgd_set_fetch_counts(h, counts)
 
 
 def fasgd_pull(h, params):
@@ -199,6 +224,18 @@ def aligned_vectors(data, device="cuda"):
     return buf, [buf[r, :P] for r in range(R)]
 
 
+def fetch_apply(theta_client, idx, val, n_dev=None, n_max=None, err_dev=None, stream=None):
+    """Client side of a B-FASGD fetch (bfasgd_fetch_apply) on torch tensors."""
+    import torch
+    if n_max is None:
+        n_max = idx.numel()
+    s = stream if stream is not None else torch.cuda.current_stream()
+    rc = bfasgd_fetch_apply(theta_client.numel(), _ptr(theta_client), _ptr(idx), _ptr(val),
+                            _ptr(n_dev), n_max, s.cuda_stream, _ptr(err_dev))
+    if rc != OK:
+        raise FasgdError(rc, fasgd_last_error(None))
+
+
 class Server:
     """One FASGD parameter server on the current CUDA device.
 
@@ -262,6 +299,19 @@ class Server:
     def select_compact(self, client: int, grad, idx, val, n_dev, v=None):
         self._check(bfasgd_select_compact(self.h, client, _ptr(grad), _ptr(v), _ptr(idx),
                                           _ptr(val), _ptr(n_dev)))
+
+    def set_fetch_threshold(self, c_fetch: float):
+        self._check(fasgd_set_fetch_threshold(self.h, c_fetch))
+
+    def fetch_compact(self, client: int, idx, val, n_dev, v=None):
+        self._check(bfasgd_fetch_compact(self.h, client, _ptr(v), _ptr(idx), _ptr(val),
+                                         _ptr(n_dev)))
+
+    def fetch_counts(self):
+        import numpy as np
+        out = np.zeros(self.lam, dtype=np.uint64)
+        self._check(fasgd_get_fetch_counts(self.h, out.ctypes.data))
+        return out
 
     def pull(self, params=None) -> int:
         rc, T = fasgd_pull(self.h, _ptr(params))
