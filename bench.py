@@ -301,7 +301,8 @@ def run_dense(args, w, world, rank, local):
         host_slots = [host_pool[r] for r in range(host_pool.shape[0])]
         out = torch.empty(P, dtype=torch.float32).pin_memory()
         T0 = srv.T
-        e2e_ps = streams.push_stream(w, (args.e2e_steps + 2) * K, K)
+        e2e_warm = 4    # enough steps for the staging pool to reach its steady size
+        e2e_ps = streams.push_stream(w, (args.e2e_steps + e2e_warm) * K, K)
 
         def e2e_step(b):
             cl, js, sl = e2e_ps.batch(b)
@@ -311,7 +312,7 @@ def run_dense(args, w, world, rank, local):
             srv.apply_pending(K)
             srv.pull(out)
 
-        for b in range(2):
+        for b in range(e2e_warm):
             e2e_step(b)
         torch.cuda.synchronize()
         barrier(world)
@@ -319,7 +320,7 @@ def run_dense(args, w, world, rank, local):
         e_start, e_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         e_start.record(stream)
         for b in range(args.e2e_steps):
-            e2e_step(2 + b)
+            e2e_step(e2e_warm + b)
         e_end.record(stream)
         torch.cuda.synchronize()
         wall = time.perf_counter() - t0

@@ -125,11 +125,14 @@ FASGD_API int fasgd_push(fasgd_t* h, int32_t client, int64_t timestamp, const fl
 
 /*
  * fasgd_push_host -- as fasgd_push, for a gradient in host memory: the P
- * values are copied (asynchronously, on the stream) into a device staging
- * slot owned by the handle, so the host buffer must stay unchanged until
- * the stream reaches the copy (pinned memory makes the copy asynchronous).
- * At most FASGD_KMAX host pushes may be pending; the first use of each
- * staging slot allocates it.  Errors: EINVAL, ERANGE, EAGAIN, ENOMEM, ECUDA.
+ * values are copied asynchronously into a device staging slot owned by the
+ * handle, on an internal copy stream so that the copies of later pushes
+ * overlap the pass that consumes earlier ones (the pass waits for its
+ * copies).  The host buffer must stay unchanged until the apply that
+ * consumes the push has completed on the handle's stream (pinned memory
+ * keeps the copy asynchronous).  At most FASGD_KMAX host pushes may be
+ * pending; staging slots (P floats each, at most FASGD_KMAX) are allocated on
+ * first need.  Errors: EINVAL, ERANGE, EAGAIN, ENOMEM, ECUDA.
  */
 FASGD_API int fasgd_push_host(fasgd_t* h, int32_t client, int64_t timestamp, const float* grad_host);
 
@@ -216,9 +219,12 @@ FASGD_API int bfasgd_fetch_apply(int64_t P, float* theta_client, const int32_t* 
                                  void* stream, int32_t* err_dev);
 
 /*
- * fasgd_pull -- copy theta (P fp32) into params (host or device) on the
- * stream and return the server timestamp T in *T (Sec. 2.1 protocol step 3:
- * the parameters handed back to a client).  Pending pushes are not applied.
+ * fasgd_pull -- copy theta (P fp32) into params (host or device) and return
+ * the server timestamp T in *T (Sec. 2.1 protocol step 3: the parameters
+ * handed back to a client).  The copy is ordered after earlier work on the
+ * handle's stream and later work on that stream waits for it (it runs on an
+ * internal stream beside pending host-push copies).  Pending pushes are not
+ * applied.
  * Either output may be NULL.  Errors: EINVAL, ECUDA.
  */
 FASGD_API int fasgd_pull(fasgd_t* h, float* params, int64_t* T);

@@ -91,8 +91,17 @@ struct fasgd_s {
     int64_t* tile_base = nullptr;
     int32_t* dev_err = nullptr;
     int32_t ntiles = 0;
+    // Host pushes: device staging slots filled on copy_stream, so the copies
+    // of the next pushes overlap the pass that consumes the previous ones.
     std::vector<float*> stage;
-    std::vector<char> stage_busy;
+    std::vector<char> stage_busy;       // held by a queued push
+    std::vector<char> stage_used;       // slot_free has been recorded
+    std::vector<cudaEvent_t> slot_ready;  // the copy into the slot is done
+    std::vector<cudaEvent_t> slot_free;   // the last pass reading the slot is done
+    cudaStream_t copy_stream = nullptr;
+    cudaStream_t pull_stream = nullptr;   // pulls run beside the next host copies
+    cudaEvent_t order_ev = nullptr;
+    cudaEvent_t pull_done_ev = nullptr;
     std::deque<Push> fifo;
     int64_t T = 0;
     int64_t launches = 0;
@@ -110,6 +119,19 @@ struct fasgd_s {
     int cuda_fail(cudaError_t st, const char* what) {
         return fail(st == cudaErrorMemoryAllocation ? FASGD_ENOMEM : FASGD_ECUDA, "%s: %s", what,
                     cudaGetErrorString(st));
+    }
+    // Streams and events for host copies and pulls, created on first use.
+    cudaError_t ensure_aux() {
+        cudaError_t st = cudaSuccess;
+        if (copy_stream == nullptr)
+            st = cudaStreamCreateWithFlags(&copy_stream, cudaStreamNonBlocking);
+        if (st == cudaSuccess && pull_stream == nullptr)
+            st = cudaStreamCreateWithFlags(&pull_stream, cudaStreamNonBlocking);
+        if (st == cudaSuccess && order_ev == nullptr)
+            st = cudaEventCreateWithFlags(&order_ev, cudaEventDisableTiming);
+        if (st == cudaSuccess && pull_done_ev == nullptr)
+            st = cudaEventCreateWithFlags(&pull_done_ev, cudaEventDisableTiming);
+        return st;
     }
     fasgd::StatParams stat_params() const {
         fasgd::StatParams sp;
@@ -134,6 +156,16 @@ struct fasgd_s {
         cudaFree(tile_base);
         cudaFree(dev_err);
         for (float* s : stage) cudaFree(s);
+        for (cudaEvent_t e : slot_ready) cudaEventDestroy(e);
+        for (cudaEvent_t e : slot_free) cudaEventDestroy(e);
+        slot_ready.clear();
+        slot_free.clear();
+        if (order_ev) cudaEventDestroy(order_ev);
+        if (pull_done_ev) cudaEventDestroy(pull_done_ev);
+        if (copy_stream) cudaStreamDestroy(copy_stream);
+        if (pull_stream) cudaStreamDestroy(pull_stream);
+        order_ev = pull_done_ev = nullptr;
+        copy_stream = pull_stream = nullptr;
         theta = n = b = v = nullptr;
         mask = nullptr;
         tile_count = nullptr;
@@ -212,6 +244,8 @@ void fasgd_destroy(fasgd_t* h) {
     if (h == nullptr) return;
     DeviceGuard g(h->device);
     cudaStreamSynchronize(h->stream);
+    if (h->copy_stream) cudaStreamSynchronize(h->copy_stream);
+    if (h->pull_stream) cudaStreamSynchronize(h->pull_stream);
     h->free_all();
     delete h;
 }
@@ -278,28 +312,48 @@ int fasgd_push_host(fasgd_t* h, int32_t client, int64_t timestamp, const float* 
     if (grad_host == nullptr) return h->fail(FASGD_EINVAL, "grad_host is NULL");
     int rc = check_push(h, client, timestamp);
     if (rc != FASGD_OK) return rc;
-    int slot = -1;
-    for (size_t s = 0; s < h->stage.size(); ++s)
-        if (!h->stage_busy[s]) {
+    DeviceGuard g(h->device);
+    cudaError_t st = h->ensure_aux();
+    if (st != cudaSuccess) return h->cuda_fail(st, "fasgd_push_host: streams");
+    // Prefer a free slot no pass is still reading; else grow the pool; else
+    // take any free slot (its copy then waits for the pass that read it).
+    int slot = -1, waiting = -1;
+    for (size_t s = 0; s < h->stage.size(); ++s) {
+        if (h->stage_busy[s]) continue;
+        if (!h->stage_used[s] || cudaEventQuery(h->slot_free[s]) == cudaSuccess) {
             slot = (int)s;
             break;
         }
-    DeviceGuard g(h->device);
-    if (slot < 0) {
-        if ((int)h->stage.size() >= FASGD_KMAX)
-            return h->fail(FASGD_EAGAIN, "%d host pushes already pending", FASGD_KMAX);
+        if (waiting < 0) waiting = (int)s;
+    }
+    if (slot < 0 && (int)h->stage.size() < FASGD_KMAX) {
         float* p = nullptr;
-        cudaError_t st = cudaMalloc(reinterpret_cast<void**>(&p), (size_t)h->P * sizeof(float));
-        if (st != cudaSuccess) return h->cuda_fail(st, "fasgd_push_host: staging slot");
+        cudaEvent_t ready = nullptr, freed = nullptr;
+        st = cudaMalloc(reinterpret_cast<void**>(&p), (size_t)h->P * sizeof(float));
+        if (st == cudaSuccess) st = cudaEventCreateWithFlags(&ready, cudaEventDisableTiming);
+        if (st == cudaSuccess) st = cudaEventCreateWithFlags(&freed, cudaEventDisableTiming);
+        if (st != cudaSuccess) {
+            cudaFree(p);
+            if (ready) cudaEventDestroy(ready);
+            return h->cuda_fail(st, "fasgd_push_host: staging slot");
+        }
         h->stage.push_back(p);
         h->stage_busy.push_back(0);
+        h->stage_used.push_back(0);
+        h->slot_ready.push_back(ready);
+        h->slot_free.push_back(freed);
         slot = (int)h->stage.size() - 1;
     }
-    cudaError_t st = cudaMemcpyAsync(h->stage[slot], grad_host, (size_t)h->P * sizeof(float),
-                                     cudaMemcpyDefault, h->stream);
+    if (slot < 0) slot = waiting;
+    if (slot < 0) return h->fail(FASGD_EAGAIN, "%d host pushes already pending", FASGD_KMAX);
+    if (h->stage_used[(size_t)slot]) st = cudaStreamWaitEvent(h->copy_stream, h->slot_free[(size_t)slot], 0);
+    if (st == cudaSuccess)
+        st = cudaMemcpyAsync(h->stage[(size_t)slot], grad_host, (size_t)h->P * sizeof(float),
+                             cudaMemcpyDefault, h->copy_stream);
+    if (st == cudaSuccess) st = cudaEventRecord(h->slot_ready[(size_t)slot], h->copy_stream);
     if (st != cudaSuccess) return h->cuda_fail(st, "fasgd_push_host: copy");
-    h->stage_busy[slot] = 1;
-    h->fifo.push_back(Push{false, client, timestamp, h->stage[slot], nullptr, nullptr, nullptr, 0, slot});
+    h->stage_busy[(size_t)slot] = 1;
+    h->fifo.push_back(Push{false, client, timestamp, h->stage[(size_t)slot], nullptr, nullptr, nullptr, 0, slot});
     return FASGD_OK;
 }
 
@@ -347,7 +401,19 @@ int fasgd_apply_pending(fasgd_t* h, int32_t K) {
                 ++r;
             }
             a.K = r;
-            cudaError_t st = fasgd::launch_dense(a, fas, h->num_sms, h->stream, &h->launches);
+            cudaError_t st = cudaSuccess;
+            for (int i = 0; i < r && st == cudaSuccess; ++i) {  // staged host copies landed
+                const int slot = h->fifo[(size_t)(k + i)].stage;
+                if (slot >= 0) st = cudaStreamWaitEvent(h->stream, h->slot_ready[(size_t)slot], 0);
+            }
+            if (st == cudaSuccess) st = fasgd::launch_dense(a, fas, h->num_sms, h->stream, &h->launches);
+            for (int i = 0; i < r && st == cudaSuccess; ++i) {  // the slots may be refilled after this
+                const int slot = h->fifo[(size_t)(k + i)].stage;
+                if (slot >= 0) {
+                    st = cudaEventRecord(h->slot_free[(size_t)slot], h->stream);
+                    h->stage_used[(size_t)slot] = 1;
+                }
+            }
             if (st != cudaSuccess) return h->cuda_fail(st, "fasgd_apply_pending: dense pass");
             k += r;
         } else {
@@ -483,9 +549,18 @@ int bfasgd_fetch_apply(int64_t P, float* theta_client, const int32_t* idx, const
 int fasgd_pull(fasgd_t* h, float* params, int64_t* T) {
     if (h == nullptr) return FASGD_EINVAL;
     if (params != nullptr) {
+        // The copy runs on its own stream (so it overlaps host-push copies of
+        // the next pushes) and the handle's stream waits for it: later work on
+        // the stream, and a caller synchronising it, see the pull complete.
         DeviceGuard g(h->device);
-        cudaError_t st = cudaMemcpyAsync(params, h->theta, (size_t)h->P * sizeof(float),
-                                         cudaMemcpyDefault, h->stream);
+        cudaError_t st = h->ensure_aux();
+        if (st == cudaSuccess) st = cudaEventRecord(h->order_ev, h->stream);
+        if (st == cudaSuccess) st = cudaStreamWaitEvent(h->pull_stream, h->order_ev, 0);
+        if (st == cudaSuccess)
+            st = cudaMemcpyAsync(params, h->theta, (size_t)h->P * sizeof(float), cudaMemcpyDefault,
+                                 h->pull_stream);
+        if (st == cudaSuccess) st = cudaEventRecord(h->pull_done_ev, h->pull_stream);
+        if (st == cudaSuccess) st = cudaStreamWaitEvent(h->stream, h->pull_done_ev, 0);
         if (st != cudaSuccess) return h->cuda_fail(st, "fasgd_pull");
     }
     if (T != nullptr) *T = h->T;
