@@ -84,6 +84,10 @@ def load_library(path: str, real: str) -> ctypes.CDLL:
                                      P, P]
     lib.ora_fetch_apply.restype = None
     lib.ora_fetch_apply.argtypes = [P, i64, P, P]
+    lib.ora_mean_v.restype = ctypes.c_float
+    lib.ora_mean_v.argtypes = [i64, P]
+    lib.ora_draw_message.restype = u32
+    lib.ora_draw_message.argtypes = [u64, u32, u32, u64]
     assert lib.ora_real_bytes() == (4 if real == "f32" else 8)
     return lib
 
@@ -169,6 +173,17 @@ def fetch_apply(theta_client: np.ndarray, idx: np.ndarray, val: np.ndarray, lib=
     (lib or _load("f32")).ora_fetch_apply(_ptr(theta_client), i.shape[0], _ptr(i), _ptr(x))
 
 
+def mean_v(v: np.ndarray, real: str = "f32", lib=None) -> float:
+    """The per-message statistic of Sec. 2.3: mean of v over all parameters (fp32)."""
+    vv = np.ascontiguousarray(v, dtype=_dtype(real))
+    return float((lib or _load(real)).ora_mean_v(vv.shape[0], _ptr(vv)))
+
+
+def draw_message(seed: int, stream: int, client: int, n: int, lib=None) -> int:
+    """24-bit draw of a client's n-th push (stream 0) or fetch (stream 1) message."""
+    return int((lib or _load("f32")).ora_draw_message(seed, stream, client, n))
+
+
 class OracleError(Exception):
     pass
 
@@ -198,6 +213,8 @@ class OracleServer:
         self.push_count = [0] * lam
         self.fetch_count = [0] * lam
         self.c_fetch = 0.0
+        self.cache: dict = {}          # client -> most recent sent gradient (message pushes)
+        self.message_log: list = []    # decisions of applied message pushes, in order
         self.set_hparams(gamma, beta, eps, c_push, eps_b, seed)
 
     def set_hparams(self, gamma, beta, eps, c_push, eps_b, seed):
@@ -212,6 +229,27 @@ class OracleServer:
     def push(self, client: int, j: int, g: np.ndarray):
         self._check(client, j)
         self.fifo.append(("dense", int(client), int(j), np.asarray(g, dtype=np.float32)))
+
+    def push_message(self, client: int, j: int, g: np.ndarray):
+        """Literal B-FASGD push (Sec. 2.3): decided when applied, against the
+        mean of v at that moment; a dropped push re-applies the client's most
+        recent sent gradient (zeros if it has none)."""
+        self._check(client, j)
+        self.fifo.append(("message", int(client), int(j), np.asarray(g, dtype=np.float32)))
+
+    def fetch_message(self, client: int, theta_client: np.ndarray) -> bool:
+        """Literal B-FASGD fetch: one decision with c_fetch against the mean of
+        v; on success the client's copy becomes theta.  Returns the decision."""
+        if not 0 <= client < self.lam:
+            raise OracleError("client out of range")
+        n = self.fetch_count[client]
+        self.fetch_count[client] += 1
+        u = draw_message(self.seed, 1, client, n)
+        vbar = mean_v(self.v, self.real)
+        ok = decide(u, vbar, self.c_fetch, self.eps_b)
+        if ok:
+            theta_client[:] = self.theta.astype(np.float32)
+        return ok
 
     def push_sparse(self, client: int, j: int, idx: np.ndarray, val: np.ndarray):
         self._check(client, j)
@@ -232,6 +270,17 @@ class OracleServer:
             kind, client, j, payload = self.fifo.pop(0)
             tau = self.T - j
             c = self.lib.ora_coef(self.variant, self.alpha, tau)
+            if kind == "message":
+                n = self.push_count[client]
+                self.push_count[client] += 1
+                u = draw_message(self.seed, 0, client, n)
+                vbar = mean_v(self.v, self.real)
+                sent = decide(u, vbar, self.c_push, self.eps_b)
+                self.message_log.append(sent)
+                if sent:
+                    self.cache[client] = payload.copy()
+                kind = "dense"
+                payload = self.cache.get(client, np.zeros(self.P, np.float32))
             if kind == "dense":
                 g = np.ascontiguousarray(payload, dtype=np.float32)
                 self.lib.ora_apply_dense(self.variant, self.P, _ptr(self.theta), _ptr(self.n),

@@ -253,3 +253,30 @@ void ora_fetch_apply(float *theta_client, int64_t count, const int32_t *idx, con
     for (int64_t i = 0; i < count; i++)
         theta_client[idx[i]] = val[i];
 }
+
+/*
+ * The paper's literal B-FASGD (Sec. 2.3): one decision per transmission
+ * opportunity, with v the mean over all parameters of the server's moving
+ * averages.  ora_mean_v returns that mean, summed in fp64 in index order and
+ * rounded once to fp32; the decision is Eq. 9 in fp32 (ora_decide) with a
+ * draw from the message domain: word 0 of Philox4x32-10 at counter
+ * (2^32 - 1, client + 2^31 * stream, n low, n high), top 24 bits (the
+ * per-parameter draws never reach that first counter word, since
+ * p div 4 < 2^29).
+ */
+float ora_mean_v(int64_t P, const REAL *v)
+{
+    double s = 0.0;
+    for (int64_t p = 0; p < P; p++)
+        s += (double)v[p];
+    return (float)(s / (double)P);
+}
+
+uint32_t ora_draw_message(uint64_t seed, uint32_t stream, uint32_t client, uint64_t n)
+{
+    uint32_t ctr[4] = {0xFFFFFFFFu, client | (stream << 31), (uint32_t)n, (uint32_t)(n >> 32)};
+    uint32_t key[2] = {(uint32_t)seed, (uint32_t)(seed >> 32)};
+    uint32_t out[4];
+    ora_philox4x32_10(ctr, key, out);
+    return out[0] >> 8;
+}

@@ -469,6 +469,93 @@ def check_server_fetch_counters(libs: Libs):
     assert np.array_equal(a[0], b[0])
 
 
+def check_message_path(libs: Libs):
+    """The paper's literal B-FASGD (Sec. 2.3): one Eq. 9 decision per message
+    against the mean of v; dropped pushes re-apply the client's cached
+    gradient; dropped fetches leave the client's copy as it is."""
+    rng = np.random.default_rng(41)
+    # The statistic is the exact mean of v, rounded once to fp32.
+    for real in ("f32", "f64"):
+        for P in (1, 7, 1000, 4099):
+            v = (10 ** rng.uniform(-2, 3, P)).astype(np.float32)
+            exact = Fraction(math.fsum(v.astype(np.float64))) / P
+            got = oracle.mean_v(v, real, lib=libs.lib(real))
+            assert got == float(np.float32(float(exact))), (real, P)
+    # Message draws are their own domain (not the per-parameter draws).
+    seed = 99
+    same = sum(oracle.draw_message(seed, 0, 2, n, lib=libs.f32) ==
+               oracle.draw_stream(seed, 0, 2, n, 0, lib=libs.f32) for n in range(300))
+    assert same < 3
+    assert sum(oracle.draw_message(seed, 0, 2, n, lib=libs.f32) ==
+               oracle.draw_message(seed, 1, 2, n, lib=libs.f32) for n in range(300)) < 3
+    P, lam = 37, 3
+    grads = [(rng.standard_normal(P) * 0.1).astype(np.float32) for _ in range(30)]
+    theta0 = (rng.standard_normal(P) * 0.01).astype(np.float32)
+
+    def run(c_push, variant=FASGD):
+        s = _server(libs, "f32", P, variant, lam=lam, c_push=c_push, seed=seed)
+        s.set_params(theta0)
+        for t, g in enumerate(grads):
+            s.push_message(t % lam, s.T - min(t % 2, s.T), g)
+            s.apply_pending(1)
+        return s
+
+    def dense(seq, variant=FASGD):
+        s = _server(libs, "f32", P, variant, lam=lam)
+        s.set_params(theta0)
+        for t, g in enumerate(seq):
+            s.push(t % lam, s.T - min(t % 2, s.T), g)
+            s.apply_pending(1)
+        return s
+
+    # c = 0: every push is sent -> plain FASGD.
+    a, b = run(0.0), dense(grads)
+    assert all(a.message_log)
+    for x, y in zip(a.state()[:4], b.state()[:4]):
+        assert np.array_equal(x.view(np.uint32), y.view(np.uint32))
+    # c = inf: nothing is sent, nothing is cached -> zero gradients.
+    a, b = run(float("inf")), dense([np.zeros(P, np.float32)] * len(grads))
+    assert not any(a.message_log)
+    for x, y in zip(a.state()[:4], b.state()[:4]):
+        assert np.array_equal(x.view(np.uint32), y.view(np.uint32))
+    # Moderate c: the run equals plain FASGD on the sequence where each dropped
+    # push is replaced by its client's last sent gradient.
+    a = run(30.0)
+    assert 0 < sum(a.message_log) < len(grads)
+    last, seq = {}, []
+    for t, (g, sent) in enumerate(zip(grads, a.message_log)):
+        c = t % lam
+        if sent:
+            last[c] = g
+        seq.append(last.get(c, np.zeros(P, np.float32)))
+    b = dense(seq)
+    for x, y in zip(a.state()[:4], b.state()[:4]):
+        assert np.array_equal(x.view(np.uint32), y.view(np.uint32))
+    # Decisions are Eq. 9 against the mean of v, with the message draw; the
+    # send fraction at fixed v matches 1 / (1 + c / v).
+    s = _server(libs, "f32", P, ASGD, lam=1, c_push=4.0, seed=seed)
+    s.v[:] = 4.0                     # ASGD never changes v
+    for t in range(3000):
+        s.push_message(0, s.T, grads[t % len(grads)])
+        s.apply_pending(1)
+    for n in range(50):
+        u = oracle.draw_message(seed, 0, 0, n, lib=libs.f32)
+        assert s.message_log[n] == _exact_decide(u, 4.0, 4.0, s.eps_b)
+    frac = sum(s.message_log) / 3000
+    assert abs(frac - 0.5) < 5 * math.sqrt(0.25 / 3000), frac
+    # Fetch messages: c_fetch = 0 always fetches, inf never.
+    s = _server(libs, "f32", P, FASGD, lam=2, seed=seed)
+    s.push(0, 0, grads[0])
+    s.apply_pending(1)
+    copy = np.full(P, 3.0, np.float32)
+    s.set_fetch_threshold(float("inf"))
+    assert s.fetch_message(1, copy) is False and np.all(copy == 3.0)
+    s.set_fetch_threshold(0.0)
+    assert s.fetch_message(1, copy) is True
+    assert np.array_equal(copy.view(np.uint32), s.theta.view(np.uint32))
+    assert s.fetch_count == [0, 2]
+
+
 def check_protocol_errors(libs: Libs):
     s = _server(libs, "f32", 4, FASGD, lam=2)
     g = np.zeros(4, np.float32)
@@ -509,5 +596,6 @@ ALL_CHECKS = [
     check_sparse_leaves_unsent_untouched,
     check_fetch_path,
     check_server_fetch_counters,
+    check_message_path,
     check_protocol_errors,
 ]

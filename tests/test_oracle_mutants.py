@@ -45,6 +45,10 @@ MUTANTS = {
     "fetch_uses_push_stream": ("return ora_select_stream(P, theta, v, c, eps_b, seed, 1,",
                                "return ora_select_stream(P, theta, v, c, eps_b, seed, 0,"),
     "fetch_apply_wrong_slot": ("theta_client[idx[i]] = val[i];", "theta_client[i] = val[i];"),
+    "mean_v_wrong_divisor": ("return (float)(s / (double)P);", "return (float)(s / (double)(P + 1));"),
+    "mean_v_first_only": ("s += (double)v[p];", "s = (double)v[p];"),
+    "message_draw_collides": ("uint32_t ctr[4] = {0xFFFFFFFFu,", "uint32_t ctr[4] = {0u,"),
+    "message_draw_ignores_stream": ("{0xFFFFFFFFu, client | (stream << 31),", "{0xFFFFFFFFu, client,"),
     "decide_not_strict": ("prod == A && err < 0.0f", "prod == A && err <= 0.0f"),
     "decide_ignores_err": ("if (prod == A && err < 0.0f)\n        return 1;\n", ""),
     "decide_drops_eps": ("float a = v + eps_b;", "float a = v;"),
