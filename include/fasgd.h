@@ -219,6 +219,39 @@ FASGD_API int bfasgd_fetch_apply(int64_t P, float* theta_client, const int32_t* 
                                  void* stream, int32_t* err_dev);
 
 /*
+ * bfasgd_push_message -- the paper's literal B-FASGD push (Sec. 2.3): one
+ * decision for the whole message.  When the push is applied (in arrival
+ * order, by fasgd_apply_pending), the server forms vbar = the mean of v over
+ * all P parameters (fp64 sum in a fixed order, rounded once to fp32), draws u
+ * (Philox4x32-10 word 0 at counter (2^32-1, client, n, n >> 32), key = seed,
+ * n = the client's push count, which then advances) and transmits iff Eq. 9
+ * holds: u / 2^24 < 1 / (1 + c_push / (vbar + eps_b)), decided exactly in
+ * fp32.  A transmitted push replaces the client's slot of the server's
+ * gradient cache; either way the server applies the slot, so a dropped push
+ * re-applies the client's most recent transmitted gradient (zeros if it has
+ * none yet) -- the paper's choice.  The first call allocates the cache:
+ * lambda x P floats.  grad: device fp32[P], 16-byte aligned, borrowed until
+ * the apply completes.  sent_dev: device int32 receiving 1 (transmitted) or 0
+ * (dropped) when the push is applied, or NULL.  Such a push is applied as its
+ * own pass (it does not fuse with neighbours).
+ * Errors: EINVAL, ERANGE, EAGAIN, ENOMEM, ECUDA.
+ */
+FASGD_API int bfasgd_push_message(fasgd_t* h, int32_t client, int64_t timestamp,
+                                  const float* grad, int32_t* sent_dev);
+
+/*
+ * bfasgd_fetch_message -- the paper's literal B-FASGD fetch (Sec. 2.3): one
+ * decision, as for a message push but with c_fetch and counter word
+ * client + 2^31 (n = the client's fetch count, which advances), taken on the
+ * stream against the current server state; if transmitted, theta is copied
+ * into theta_client (device fp32[P], 16-byte aligned), otherwise the client
+ * keeps its copy.  fetched_dev: device int32 receiving 1 or 0, or NULL.
+ * Errors: EINVAL, ERANGE, ENOMEM, ECUDA.
+ */
+FASGD_API int bfasgd_fetch_message(fasgd_t* h, int32_t client, float* theta_client,
+                                   int32_t* fetched_dev);
+
+/*
  * fasgd_pull -- copy theta (P fp32) into params (host or device) and return
  * the server timestamp T in *T (Sec. 2.1 protocol step 3: the parameters
  * handed back to a client).  The copy is ordered after earlier work on the

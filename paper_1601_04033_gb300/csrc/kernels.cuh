@@ -83,6 +83,28 @@ struct ScatterArgs {
     int32_t* err;              // may be null; flags 1 (count) and 2 (index)
 };
 
+// One per-message B-FASGD decision (push or fetch) and, when the message is
+// transmitted, the copy src -> dst (P floats, both 16-byte aligned).
+constexpr int kMessageMaxBlocks = 1024;
+
+struct MessageArgs {
+    const float* v;            // the server's statistic, fp32[P]
+    int64_t P;
+    double* partial;           // scratch: nblocks partial sums
+    int32_t nblocks;           // message_partial_blocks(P)
+    float c;                   // c_push or c_fetch
+    float eps_b;
+    uint32_t round_key0[10];
+    uint32_t round_key1[10];
+    uint32_t client_word;      // client + 2^31 * stream (0: push, 1: fetch)
+    uint32_t n_lo, n_hi;       // the client's count of earlier messages of that stream
+    const float* src;          // may be null: decide only
+    float* dst;
+    int32_t* flag_out;         // may be null: 1 transmitted, 0 dropped
+};
+
+int32_t message_partial_blocks(int64_t P);
+
 // Launchers: enqueue on `stream`, return the launch status.
 // `launches` is incremented by the number of kernels enqueued.
 cudaError_t launch_dense(const DenseArgs& a, bool fasgd_rule, int num_sms, cudaStream_t stream,
@@ -91,6 +113,8 @@ cudaError_t launch_sparse(const SparseArgs& a, bool fasgd_rule, int num_sms, cud
                           int64_t* launches);
 cudaError_t launch_select(const SelectArgs& a, cudaStream_t stream, int64_t* launches);
 cudaError_t launch_scatter(const ScatterArgs& a, int num_sms, cudaStream_t stream);
+cudaError_t launch_message(const MessageArgs& a, int num_sms, cudaStream_t stream,
+                           int64_t* launches);
 
 inline int32_t select_tiles(int64_t P) {
     return (int32_t)((P + kSelectTile - 1) / kSelectTile);

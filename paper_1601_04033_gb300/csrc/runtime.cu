@@ -21,6 +21,7 @@
 #include <string>
 #include <vector>
 
+#include "eq9.cuh"
 #include "fasgd.h"
 #include "kernels.cuh"
 
@@ -31,8 +32,10 @@ constexpr int32_t kMaxLambda = int32_t(1) << 20;
 
 thread_local std::string g_create_error;
 
+enum PushKind { kDense = 0, kSparse = 1, kMessage = 2 };
+
 struct Push {
-    bool sparse;
+    int kind;              // PushKind
     int32_t client;
     int64_t j;
     const float* grad;     // dense
@@ -41,6 +44,7 @@ struct Push {
     const int64_t* n_dev;
     int64_t n_max;
     int stage;             // staging slot of a host push, -1 otherwise
+    int32_t* flag;         // message push: where to report the decision (may be null)
 };
 
 bool aligned(const void* p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) & (a - 1)) == 0; }
@@ -120,6 +124,55 @@ struct fasgd_s {
         return fail(st == cudaErrorMemoryAllocation ? FASGD_ENOMEM : FASGD_ECUDA, "%s: %s", what,
                     cudaGetErrorString(st));
     }
+    // Per-message B-FASGD: the gradient cache (lambda slots of cache_stride
+    // floats, allocated by the first message push) and the partial sums.
+    float* grad_cache = nullptr;
+    int64_t cache_stride = 0;
+    double* msg_partial = nullptr;
+
+    cudaError_t ensure_message_scratch(bool cache) {
+        cudaError_t st = cudaSuccess;
+        if (msg_partial == nullptr)
+            st = cudaMalloc(reinterpret_cast<void**>(&msg_partial),
+                            fasgd::kMessageMaxBlocks * sizeof(double));
+        if (st == cudaSuccess && cache && grad_cache == nullptr) {
+            cache_stride = (P + 63) / 64 * 64;   // 256-byte aligned slots
+            const size_t bytes = (size_t)lambda * (size_t)cache_stride * sizeof(float);
+            st = cudaMalloc(reinterpret_cast<void**>(&grad_cache), bytes);
+            if (st == cudaSuccess) st = cudaMemsetAsync(grad_cache, 0, bytes, stream);
+            if (st != cudaSuccess && grad_cache != nullptr) {
+                cudaFree(grad_cache);
+                grad_cache = nullptr;
+            }
+        }
+        return st;
+    }
+
+    // One per-message decision of `stream_id` for `client` (advancing its
+    // counter), copying src -> dst if transmitted.
+    cudaError_t launch_message(uint32_t stream_id, int32_t client, const float* src, float* dst,
+                               int32_t* flag, float c, std::vector<uint64_t>& counter) {
+        fasgd::MessageArgs a;
+        std::memset(&a, 0, sizeof a);
+        a.v = v;
+        a.P = P;
+        a.partial = msg_partial;
+        a.nblocks = fasgd::message_partial_blocks(P);
+        a.c = c;
+        a.eps_b = eps_b;
+        fasgd::philox_key_schedule(seed, a.round_key0, a.round_key1);
+        const uint64_t n = counter[(size_t)client];
+        a.client_word = (uint32_t)client | (stream_id << 31);
+        a.n_lo = (uint32_t)n;
+        a.n_hi = (uint32_t)(n >> 32);
+        a.src = src;
+        a.dst = dst;
+        a.flag_out = flag;
+        cudaError_t st = fasgd::launch_message(a, num_sms, stream, &launches);
+        if (st == cudaSuccess) counter[(size_t)client] = n + 1;
+        return st;
+    }
+
     // Streams and events for host copies and pulls, created on first use.
     cudaError_t ensure_aux() {
         cudaError_t st = cudaSuccess;
@@ -155,6 +208,10 @@ struct fasgd_s {
         cudaFree(tile_count);
         cudaFree(tile_base);
         cudaFree(dev_err);
+        cudaFree(grad_cache);
+        cudaFree(msg_partial);
+        grad_cache = nullptr;
+        msg_partial = nullptr;
         for (float* s : stage) cudaFree(s);
         for (cudaEvent_t e : slot_ready) cudaEventDestroy(e);
         for (cudaEvent_t e : slot_free) cudaEventDestroy(e);
@@ -303,7 +360,7 @@ int fasgd_push(fasgd_t* h, int32_t client, int64_t timestamp, const float* grad)
         return h->fail(FASGD_EINVAL, "grad must be a non-NULL 16-byte aligned device pointer");
     int rc = check_push(h, client, timestamp);
     if (rc != FASGD_OK) return rc;
-    h->fifo.push_back(Push{false, client, timestamp, grad, nullptr, nullptr, nullptr, 0, -1});
+    h->fifo.push_back(Push{kDense, client, timestamp, grad, nullptr, nullptr, nullptr, 0, -1, nullptr});
     return FASGD_OK;
 }
 
@@ -353,7 +410,38 @@ int fasgd_push_host(fasgd_t* h, int32_t client, int64_t timestamp, const float* 
     if (st == cudaSuccess) st = cudaEventRecord(h->slot_ready[(size_t)slot], h->copy_stream);
     if (st != cudaSuccess) return h->cuda_fail(st, "fasgd_push_host: copy");
     h->stage_busy[(size_t)slot] = 1;
-    h->fifo.push_back(Push{false, client, timestamp, h->stage[(size_t)slot], nullptr, nullptr, nullptr, 0, slot});
+    h->fifo.push_back(Push{kDense, client, timestamp, h->stage[(size_t)slot], nullptr, nullptr, nullptr, 0, slot, nullptr});
+    return FASGD_OK;
+}
+
+int bfasgd_push_message(fasgd_t* h, int32_t client, int64_t timestamp, const float* grad,
+                        int32_t* sent_dev) {
+    if (h == nullptr) return FASGD_EINVAL;
+    if (grad == nullptr || !aligned(grad, 16))
+        return h->fail(FASGD_EINVAL, "grad must be a non-NULL 16-byte aligned device pointer");
+    if (!aligned(sent_dev, 4)) return h->fail(FASGD_EINVAL, "sent_dev must be 4-byte aligned");
+    int rc = check_push(h, client, timestamp);
+    if (rc != FASGD_OK) return rc;
+    DeviceGuard g(h->device);
+    cudaError_t st = h->ensure_message_scratch(true);
+    if (st != cudaSuccess) return h->cuda_fail(st, "bfasgd_push_message: gradient cache");
+    h->fifo.push_back(Push{kMessage, client, timestamp, grad, nullptr, nullptr, nullptr, 0, -1, sent_dev});
+    return FASGD_OK;
+}
+
+int bfasgd_fetch_message(fasgd_t* h, int32_t client, float* theta_client, int32_t* fetched_dev) {
+    if (h == nullptr) return FASGD_EINVAL;
+    if (client < 0 || client >= h->lambda)
+        return h->fail(FASGD_ERANGE, "client %d outside [0, %d)", client, h->lambda);
+    if (theta_client == nullptr || !aligned(theta_client, 16) || !aligned(fetched_dev, 4))
+        return h->fail(FASGD_EINVAL, "theta_client must be a non-NULL 16-byte aligned device "
+                                     "pointer (fetched_dev 4-byte aligned)");
+    DeviceGuard g(h->device);
+    cudaError_t st = h->ensure_message_scratch(false);
+    if (st == cudaSuccess)
+        st = h->launch_message(1, client, h->theta, theta_client, fetched_dev, h->c_fetch,
+                               h->fetch_count);
+    if (st != cudaSuccess) return h->cuda_fail(st, "bfasgd_fetch_message");
     return FASGD_OK;
 }
 
@@ -367,7 +455,7 @@ int fasgd_push_sparse(fasgd_t* h, int32_t client, int64_t timestamp, const int32
         return h->fail(FASGD_EINVAL, "idx, val must be 4-byte and n_dev 8-byte aligned");
     int rc = check_push(h, client, timestamp);
     if (rc != FASGD_OK) return rc;
-    h->fifo.push_back(Push{true, client, timestamp, nullptr, idx, val, n_dev, n_max, -1});
+    h->fifo.push_back(Push{kSparse, client, timestamp, nullptr, idx, val, n_dev, n_max, -1, nullptr});
     return FASGD_OK;
 }
 
@@ -382,7 +470,7 @@ int fasgd_apply_pending(fasgd_t* h, int32_t K) {
     int k = 0;
     while (k < K) {
         const Push& first = h->fifo[(size_t)k];
-        if (!first.sparse) {
+        if (first.kind == kDense) {
             // Fuse the run of consecutive dense pushes into one pass.
             fasgd::DenseArgs a;
             std::memset(&a, 0, sizeof a);
@@ -394,7 +482,7 @@ int fasgd_apply_pending(fasgd_t* h, int32_t K) {
             a.sp = sp;
             a.err = h->dev_err;
             int r = 0;
-            while (k + r < K && !h->fifo[(size_t)(k + r)].sparse) {
+            while (k + r < K && h->fifo[(size_t)(k + r)].kind == kDense) {
                 const Push& p = h->fifo[(size_t)(k + r)];
                 a.grad[r] = p.grad;
                 a.coef[r] = h->coef(h->T + k + r - p.j);
@@ -416,6 +504,29 @@ int fasgd_apply_pending(fasgd_t* h, int32_t K) {
             }
             if (st != cudaSuccess) return h->cuda_fail(st, "fasgd_apply_pending: dense pass");
             k += r;
+        } else if (first.kind == kMessage) {
+            // Decide against the mean of v now, refresh the client's cache
+            // slot if the push is transmitted, then apply the slot.
+            float* slot = h->grad_cache + (size_t)first.client * (size_t)h->cache_stride;
+            cudaError_t st = h->launch_message(0, first.client, first.grad, slot, first.flag,
+                                               h->c_push, h->push_count);
+            if (st == cudaSuccess) {
+                fasgd::DenseArgs a;
+                std::memset(&a, 0, sizeof a);
+                a.theta = h->theta;
+                a.n = h->n;
+                a.b = h->b;
+                a.v = h->v;
+                a.P = h->P;
+                a.sp = sp;
+                a.err = h->dev_err;
+                a.grad[0] = slot;
+                a.coef[0] = h->coef(h->T + k - first.j);
+                a.K = 1;
+                st = fasgd::launch_dense(a, fas, h->num_sms, h->stream, &h->launches);
+            }
+            if (st != cudaSuccess) return h->cuda_fail(st, "fasgd_apply_pending: message push");
+            k += 1;
         } else {
             fasgd::SparseArgs a;
             std::memset(&a, 0, sizeof a);

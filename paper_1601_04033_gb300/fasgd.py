@@ -52,6 +52,8 @@ SIGNATURES = {
     "bfasgd_fetch_apply": (_i32, [_i64, _p, _p, _p, _p, _i64, _p, _p]),
     "fasgd_get_fetch_counts": (_i32, [_p, _p]),
     "fasgd_set_fetch_counts": (_i32, [_p, _p]),
+    "bfasgd_push_message": (_i32, [_p, _i32, _i64, _p, _p]),
+    "bfasgd_fetch_message": (_i32, [_p, _i32, _p, _p]),
     "bfasgd_select_compact_noalloc": (_i32, [_i64, _p, _p, _f32, _f32, _u64, _i32, _u64,
                                              _p, _p, _p, _p]),
     "fasgd_last_error": (ctypes.c_char_p, [_p]),
@@ -146,6 +148,14 @@ def fasgd_get_fetch_counts(h, counts):
 
 def fasgd_set_fetch_counts(h, counts):
     return LIB.fasgd_set_fetch_counts(h, counts)
+
+
+def bfasgd_push_message(h, client, timestamp, grad, sent_dev):
+    return LIB.bfasgd_push_message(h, client, timestamp, grad, sent_dev)
+
+
+def bfasgd_fetch_message(h, client, theta_client, fetched_dev):
+    return LIB.bfasgd_fetch_message(h, client, theta_client, fetched_dev)
 
 
 def fasgd_pull(h, params):
@@ -306,6 +316,12 @@ class Server:
     def fetch_compact(self, client: int, idx, val, n_dev, v=None):
         self._check(bfasgd_fetch_compact(self.h, client, _ptr(v), _ptr(idx), _ptr(val),
                                          _ptr(n_dev)))
+
+    def push_message(self, client: int, timestamp: int, grad, sent_dev=None):
+        self._check(bfasgd_push_message(self.h, client, timestamp, _ptr(grad), _ptr(sent_dev)))
+
+    def fetch_message(self, client: int, theta_client, fetched_dev=None):
+        self._check(bfasgd_fetch_message(self.h, client, _ptr(theta_client), _ptr(fetched_dev)))
 
     def fetch_counts(self):
         import numpy as np

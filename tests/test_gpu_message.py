@@ -1,0 +1,99 @@
+"""CUDA path of the paper's literal per-message B-FASGD (mean-v decision,
+server gradient cache) against the oracle."""
+
+import numpy as np
+import pytest
+
+import oracle
+from gpu_util import GpuRun, OracleRun, assert_bitwise, compare_states
+from paper_1601_04033_gb300 import streams
+
+pytestmark = pytest.mark.gpu
+
+SEED = 0x3E55A6E
+
+
+def _run_pair(P, n_push, c_push, lam=3, variant=oracle.FASGD):
+    import torch
+    w = streams.WORKLOADS["fasgd-1.29m"].replace(lam=lam, R=8)
+    pool = streams.gradient_pool(w, P)
+    th0 = streams.theta0(w, P)
+    ps = streams.push_stream(w, n_push, 1)
+    g = GpuRun(w, variant, P, pool, th0, c_push=c_push, seed=SEED)
+    o = OracleRun(w, variant, P, pool, th0, c_push=c_push, seed=SEED)
+    flags = torch.full((n_push,), -1, dtype=torch.int32, device="cuda")
+    for t in range(n_push):
+        cl, js, sl = ps.batch(t)
+        c, j, s = int(cl[0]), int(js[0]), int(sl[0])
+        g.srv.push_message(c, j, g.pool[s], sent_dev=flags[t:t + 1])
+        g.srv.apply_pending(1)
+        o.srv.push_message(c, j, pool[s])
+        o.srv.apply_pending(1)
+        if (t + 1) % 100 == 0:
+            compare_states(g.state(), o.state(), variant, f"message T={t + 1}")
+    got = flags.cpu().numpy()
+    assert np.array_equal(got, np.array(o.srv.message_log, dtype=np.int32)), "decisions differ"
+    return g, o, got
+
+
+@pytest.mark.parametrize("P", [5, 8192, 70_001])
+def test_message_pushes_against_oracle(P):
+    # c chosen so that roughly half the pushes are transmitted once v settles
+    _, _, flags = _run_pair(P, 200, 40.0)
+    assert 0 < flags.sum() < flags.size
+
+
+def test_message_c0_equals_dense_and_cinf_applies_zeros():
+    import torch
+    w = streams.WORKLOADS["fasgd-1.29m"].replace(lam=2, R=4)
+    P = 10_007
+    pool = streams.gradient_pool(w, P)
+    th0 = streams.theta0(w, P)
+    ps = streams.push_stream(w, 30, 1)
+    a = GpuRun(w, oracle.FASGD, P, pool, th0, c_push=0.0, seed=SEED)
+    b = GpuRun(w, oracle.FASGD, P, pool, th0)
+    z = GpuRun(w, oracle.FASGD, P, pool, th0, c_push=float("inf"), seed=SEED)
+    zb = GpuRun(w, oracle.FASGD, P, np.zeros_like(pool), th0)
+    for t in range(30):
+        cl, js, sl = ps.batch(t)
+        c, j, s = int(cl[0]), int(js[0]), int(sl[0])
+        a.srv.push_message(c, j, a.pool[s])
+        a.srv.apply_pending(1)
+        b.push_batch(cl, js, sl)
+        z.srv.push_message(c, j, z.pool[s])
+        z.srv.apply_pending(1)
+        zb.push_batch(cl, js, sl)
+    for x, y in zip(a.state()[:4], b.state()[:4]):
+        assert_bitwise(x, y, "c=0")
+    for x, y in zip(z.state()[:4], zb.state()[:4]):
+        assert_bitwise(x, y, "c=inf")
+    assert a.srv.launches == 30 * 3 and b.srv.launches == 30
+
+
+def test_fetch_messages_against_oracle():
+    import torch
+    from paper_1601_04033_gb300 import fasgd
+    P = 33_333
+    rng = np.random.default_rng(12)
+    theta = (rng.standard_normal(P) * 0.01).astype(np.float32)
+    n = np.zeros(P, np.float32)
+    b = np.zeros(P, np.float32)
+    v = (10 ** rng.uniform(0, 2, P)).astype(np.float32)
+    srv = fasgd.Server(P, 3, 0.001, fasgd.FASGD, seed=SEED)
+    srv.set_state(*[torch.from_numpy(x).cuda() for x in (theta, n, b, v)], 5)
+    o = oracle.OracleServer(P, 3, 0.001, oracle.FASGD, seed=SEED)
+    o.theta[:], o.n[:], o.b[:], o.v[:] = theta, n, b, v
+    vbar = oracle.mean_v(v)
+    for c in (0.0, vbar, float("inf")):            # always, about half, never
+        srv.set_fetch_threshold(c)
+        o.set_fetch_threshold(c)
+        for k in range(40):
+            client = k % 3
+            gcopy = torch.full((P,), 7.0, device="cuda")
+            flag = torch.full((1,), -1, dtype=torch.int32, device="cuda")
+            srv.fetch_message(client, gcopy, fetched_dev=flag)
+            ocopy = np.full(P, 7.0, np.float32)
+            ok = o.fetch_message(client, ocopy)
+            assert int(flag.item()) == int(ok), (c, k)
+            assert_bitwise(gcopy.cpu().numpy(), ocopy, f"fetched copy c={c} k={k}")
+    assert list(srv.fetch_counts()) == o.fetch_count
