@@ -483,6 +483,112 @@ def run_bfasgd(args, w, world, rank, local):
     }
 
 
+def run_message(args, w, world, rank, local):
+    """The paper's literal B-FASGD exchange per step: a message push (mean-v
+    decision, gradient-cache refresh, dense pass over the cache slot) and a
+    message fetch (decision, copy of theta to the client's copy)."""
+    import torch
+    from paper_1601_04033_gb300 import fasgd
+
+    device = torch.device("cuda", local)
+    torch.cuda.set_device(device)
+    P = args.P or w.P
+    wr = shard_workload(w, rank)
+    R = min(w.R, 8)
+    pool = streams.gradient_pool(wr, P, R)
+    th0 = streams.theta0(wr, P)
+    n_steps = args.warmup + args.steps + w.lam
+    ps = streams.push_stream(w.replace(R=R), n_steps, 1)
+    pool_t, slots = fasgd.aligned_vectors(pool, device)
+    stream = torch.cuda.current_stream()
+    srv = fasgd.Server(P, w.lam, w.alpha, streams.FASGD, stream=stream, seed=w.seed)
+    srv.set_params(torch.from_numpy(th0).to(device))
+    t = 0
+    for _ in range(w.lam):          # dense warm-up so that v is settled
+        cl, js, sl = ps.batch(t)
+        srv.push(int(cl[0]), int(js[0]), slots[int(sl[0])])
+        srv.apply_pending(1)
+        t += 1
+    v_now = torch.empty(P, device=device)
+    srv.get_state(None, None, None, v_now)
+    vbar = float(v_now.double().mean().item())
+    c_push = vbar * (1.0 / w.send_frac - 1.0)        # P(send) = vbar / (vbar + c)
+    c_fetch = vbar * (1.0 / FETCH_FRACTION - 1.0)
+    srv.set_hparams(0.95, 0.95, 1e-4, c_push, 1e-8, w.seed)
+    srv.set_fetch_threshold(c_fetch)
+    client_theta = torch.empty((w.lam, (P + 3) // 4 * 4), device=device)
+    client_theta[:, :P].copy_(torch.from_numpy(th0).to(device))
+    sent = torch.zeros(args.steps, dtype=torch.int32, device=device)
+    fetched = torch.zeros(args.steps, dtype=torch.int32, device=device)
+
+    def step(t, ev=None, i=None):
+        cl, js, sl = ps.batch(t)
+        c = int(cl[0])
+        if ev is not None:
+            ev[0].record(stream)
+        srv.push_message(c, int(js[0]), slots[int(sl[0])],
+                         sent_dev=sent[i:i + 1] if i is not None else None)
+        srv.apply_pending(1)
+        if ev is not None:
+            ev[1].record(stream)
+        srv.fetch_message(c, client_theta[c, :P], fetched_dev=fetched[i:i + 1] if i is not None else None)
+        if ev is not None:
+            ev[2].record(stream)
+
+    for _ in range(args.warmup):
+        step(t)
+        t += 1
+    torch.cuda.synchronize()
+    clocks = ClockSampler(gpu_identifier(torch))
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    launches0 = srv.launches
+    barrier(world)
+    torch.cuda.synchronize()
+    clocks.start()
+    time.sleep(0.3)
+    start.record(stream)
+    for i in range(args.steps):
+        step(t, ev[i], i)
+        t += 1
+    end.record(stream)
+    torch.cuda.synchronize()
+    clock_info = clocks.stop()
+    barrier(world)
+    launches = srv.launches - launches0
+    total_ms = max_over_ranks(start.elapsed_time(end), world, device)
+    push_ms = sum(e[0].elapsed_time(e[1]) for e in ev) / args.steps
+    fetch_ms = sum(e[1].elapsed_time(e[2]) for e in ev) / args.steps
+    s_frac = float(sent.float().mean().item())
+    f_frac = float(fetched.float().mean().item())
+    srv.sync()
+    srv.close()
+    step_s = total_ms / 1e3 / args.steps
+    peak, peak_kind = peaks()
+    # A push: vbar read (4 B), the cache refresh when sent (8 B), the dense
+    # K=1 pass over the cache slot (36 B); per parameter.
+    push_bytes = P * (4 + 8 * s_frac + 36)
+    achieved = push_bytes / (push_ms / 1e3) / 1e9
+    return {
+        "value": P * world / step_s, "ms_per_step": total_ms / args.steps,
+        "roofline": {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
+                     "frac": round(achieved / peak, 4), "peak_source": peak_kind,
+                     "kernel": "message push (vbar + cache refresh + dense pass)",
+                     "bytes_per_launch": push_bytes, "launch_ms": round(push_ms, 5),
+                     "traffic": None, "fetch_ms": round(fetch_ms, 5)},
+        "clocks": clock_info, "e2e": None, "gpu_launches": launches,
+        "pushes_per_s": world / step_s, "sent_fraction": round(s_frac, 4),
+        "fetched_fraction": round(f_frac, 4),
+        "config": {"workload": w.name, "P_per_gpu": P, "P_total": P * world, "lambda": w.lam,
+                   "K": 1, "variant": "b-fasgd per message", "c_push": c_push, "c_fetch": c_fetch,
+                   "vbar_after_warmup": vbar, "target_send_fraction": w.send_frac,
+                   "target_fetch_fraction": FETCH_FRACTION,
+                   "step": "message push (decision, cache refresh, dense pass) + message fetch",
+                   "staleness": w.delay, "parallelism": f"param-shard{world}",
+                   "l2": "inputs larger than L2, no flush"},
+    }
+
+
 # ---------------------------------------------------------------------------
 def main():
     ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
@@ -500,7 +606,9 @@ def main():
         ap.error("--warmup must be >= 3")
     world, rank, local = dist_env()
     w = streams.WORKLOADS[args.workload]
-    if w.send_frac is not None and args.workload == "bfasgd-25m":
+    if args.workload == "bfasgd-message-25m":
+        mode = "message"
+    elif w.send_frac is not None and args.workload == "bfasgd-25m":
         mode = "bfasgd"
     else:
         mode = "dense"
@@ -528,6 +636,8 @@ def main():
     init_dist(world, backend)
     if mode == "dense":
         res = run_dense(args, w, world, rank, local)
+    elif mode == "message":
+        res = run_message(args, w, world, rank, local)
     else:
         res = run_bfasgd(args, w, world, rank, local)
 

@@ -4,9 +4,9 @@
 //
 // Two kernels per decision:
 //   1. vbar_partial: fixed partition of the parameters into contiguous
-//      chunks, one per block; each block sums its chunk of v in fp64 (fixed
-//      order: per thread in index order, then a fixed shuffle tree) into one
-//      partial;
+//      chunks, one per block; each block sums its chunk of v (fixed order: per
+//      thread in index order as an fp32 sum plus its exact rounding errors,
+//      then a fixed fp64 shuffle tree) into one fp64 partial;
 //   2. message_resolve: every block adds the partials in the same fixed order,
 //      forms vbar = fl32(sum / P), draws u (Philox4x32-10, word 0 at counter
 //      (2^32-1, client + 2^31 * stream, n)), takes the exact Eq. 9 decision,
@@ -27,6 +27,19 @@ namespace {
 constexpr int kMsgThreads = 256;
 constexpr unsigned kFull = 0xffffffffu;
 
+// hi + lo += x, with the rounding error of the fp32 addition recovered
+// exactly (TwoSum: six operations, no branch, no contraction).  lo collects
+// the errors in fp32 and is itself rounded, which bounds the pair's error by
+// a few ulp of lo -- far below one ulp of the fp64 total.
+__device__ __forceinline__ void two_sum_acc(float& hi, float& lo, float x) {
+    const float t = __fadd_rn(hi, x);
+    const float xp = __fsub_rn(t, hi);
+    const float hp = __fsub_rn(t, xp);
+    const float err = __fadd_rn(__fsub_rn(hi, hp), __fsub_rn(x, xp));
+    lo = __fadd_rn(lo, err);
+    hi = t;
+}
+
 __device__ __forceinline__ double block_sum(double s, double* smem) {
 #pragma unroll
     for (int off = 16; off > 0; off >>= 1) s += __shfl_xor_sync(kFull, s, off);
@@ -45,16 +58,19 @@ __global__ void __launch_bounds__(kMsgThreads) vbar_partial_kernel(const __grid_
     const int64_t chunk = (nq + a.nblocks - 1) / a.nblocks;
     const int64_t q0 = (int64_t)blockIdx.x * chunk;
     const int64_t q1 = q0 + chunk < nq ? q0 + chunk : nq;
-    double s = 0.0;
+    // Per thread: an fp32 sum with its exact rounding error carried alongside
+    // (Knuth's TwoSum), so the pair is the exact sum of the values added;
+    // only the per-thread and per-block combines use the (slow) fp64 pipe.
+    float hi = 0.f, lo = 0.f;
     for (int64_t q = q0 + threadIdx.x; q < q1; q += kMsgThreads) {
         const float4 x = __ldcs(reinterpret_cast<const float4*>(a.v + 4 * q));
-        s += (double)x.x;
-        s += (double)x.y;
-        s += (double)x.z;
-        s += (double)x.w;
+        two_sum_acc(hi, lo, x.x);
+        two_sum_acc(hi, lo, x.y);
+        two_sum_acc(hi, lo, x.z);
+        two_sum_acc(hi, lo, x.w);
     }
-    if (blockIdx.x == 0 && threadIdx.x < (int)(a.P & 3)) s += (double)a.v[4 * nq + threadIdx.x];
-    const double t = block_sum(s, smem);
+    if (blockIdx.x == 0 && threadIdx.x < (int)(a.P & 3)) two_sum_acc(hi, lo, a.v[4 * nq + threadIdx.x]);
+    const double t = block_sum((double)hi + (double)lo, smem);
     if (threadIdx.x == 0) a.partial[blockIdx.x] = t;
 }
 

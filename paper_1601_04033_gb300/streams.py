@@ -74,6 +74,9 @@ WORKLOADS = {
                              (FASGD,), "geometric0.05", 2),
     "bfasgd-25m": Workload("bfasgd-25m", 25_000_000, 64, 10_000, 0.001, 1,
                            (FASGD,), "poisson8", 3, send_frac=0.20),
+    # The paper's literal B-FASGD (one decision per message) on the 25M shape.
+    "bfasgd-message-25m": Workload("bfasgd-message-25m", 25_000_000, 64, 10_000, 0.001, 1,
+                                   (FASGD,), "poisson8", 3, send_frac=0.20),
     "fasgd-268m-k16": Workload("fasgd-268m-k16", 268_435_456, 256, 2_000, 0.001, 16,
                                (FASGD,), "pareto1.5", 4, s_lo=1e-5, s_hi=1.0, R=32,
                                send_frac=0.20),
