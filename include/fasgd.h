@@ -55,8 +55,12 @@ typedef struct fasgd_s fasgd_t;
 enum fasgd_variant {
     FASGD_ASGD = 0,   /* theta -= alpha * g                       (Sec. 2.1, protocol step 2) */
     FASGD_SASGD = 1,  /* theta -= alpha / max(tau,1) * g           (Eq. 1-2) */
-    FASGD_FASGD = 2   /* n, b, v moving averages, then
+    FASGD_FASGD = 2,  /* n, b, v moving averages, then
                          theta -= alpha / (v * max(tau,1)) * g     (Eq. 4-8) */
+    FASGD_FASGD_STD = 3  /* as FASGD, but v averages the std sqrt(n - b^2 + eps)
+                            itself, so the step is divided by the std: the
+                            reading of Sec. 2.2's prose ("dividing the learning
+                            rate by the standard deviation") */
 };
 
 enum fasgd_status {

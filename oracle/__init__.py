@@ -25,7 +25,7 @@ import threading
 
 import numpy as np
 
-ASGD, SASGD, FASGD = 0, 1, 2
+ASGD, SASGD, FASGD, FASGD_STD = 0, 1, 2, 3
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
 _SRC = os.path.join(_HERE, "fasgd_oracle.c")

@@ -38,6 +38,7 @@
 #define ORA_ASGD 0
 #define ORA_SASGD 1
 #define ORA_FASGD 2
+#define ORA_FASGD_STD 3
 
 /* Size of REAL, so the Python side can check which build it loaded. */
 int ora_real_bytes(void) { return (int)sizeof(REAL); }
@@ -81,6 +82,16 @@ static void ora_update_one(int variant, REAL *theta, REAL *n, REAL *b, REAL *v,
         REAL r = 1 / ora_sqrt(var + eps);
         *v = beta * *v + (1 - beta) * r;                  /* Eq. 6 */
         *theta = *theta - coef * g / *v;                  /* Eq. 7-8 */
+    } else if (variant == ORA_FASGD_STD) {
+        /* The prose reading of Sec. 2.2 ("dividing the learning rate by the
+         * standard deviation"): v averages the std itself, and Eq. 7 divides
+         * by it. */
+        *n = gamma * *n + (1 - gamma) * (g * g);
+        *b = gamma * *b + (1 - gamma) * g;
+        REAL var = ora_max0(*n - *b * *b);
+        REAL r = ora_sqrt(var + eps);
+        *v = beta * *v + (1 - beta) * r;
+        *theta = *theta - coef * g / *v;
     } else {
         *theta = *theta - coef * g;                       /* Eq. 1-2 */
     }

@@ -9,6 +9,11 @@
 
 namespace fasgd {
 
+// Per-element update rule of a pass: ASGD/SASGD (Eq. 1-2), FASGD (Eq. 4-8),
+// or FASGD with v averaging the std and the step divided by it (the prose
+// reading of Sec. 2.2).
+enum : int { kRuleSgd = 0, kRuleFasgd = 1, kRuleFasgdStd = 2 };
+
 // Hyper-parameters of Eq. 4-6 as the kernels consume them.  one_m_gamma and
 // one_m_beta are formed once on the host in fp32 (1 - gamma, 1 - beta).
 struct StatParams {
@@ -107,9 +112,9 @@ int32_t message_partial_blocks(int64_t P);
 
 // Launchers: enqueue on `stream`, return the launch status.
 // `launches` is incremented by the number of kernels enqueued.
-cudaError_t launch_dense(const DenseArgs& a, bool fasgd_rule, int num_sms, cudaStream_t stream,
+cudaError_t launch_dense(const DenseArgs& a, int rule, int num_sms, cudaStream_t stream,
                          int64_t* launches);
-cudaError_t launch_sparse(const SparseArgs& a, bool fasgd_rule, int num_sms, cudaStream_t stream,
+cudaError_t launch_sparse(const SparseArgs& a, int rule, int num_sms, cudaStream_t stream,
                           int64_t* launches);
 cudaError_t launch_select(const SelectArgs& a, cudaStream_t stream, int64_t* launches);
 cudaError_t launch_scatter(const ScatterArgs& a, int num_sms, cudaStream_t stream);

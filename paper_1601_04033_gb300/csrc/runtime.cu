@@ -252,7 +252,8 @@ int fasgd_create(fasgd_t** h, int64_t P, int32_t lambda, float alpha, int32_t va
         g_create_error = "fasgd_create: alpha must be finite";
         return FASGD_EINVAL;
     }
-    if (variant != FASGD_ASGD && variant != FASGD_SASGD && variant != FASGD_FASGD) {
+    if (variant != FASGD_ASGD && variant != FASGD_SASGD && variant != FASGD_FASGD &&
+        variant != FASGD_FASGD_STD) {
         g_create_error = "fasgd_create: unknown variant";
         return FASGD_EINVAL;
     }
@@ -465,7 +466,9 @@ int fasgd_apply_pending(fasgd_t* h, int32_t K) {
     if ((int64_t)h->fifo.size() < K)
         return h->fail(FASGD_EAGAIN, "K=%d but only %zu pushes pending", K, h->fifo.size());
     DeviceGuard g(h->device);
-    const bool fas = h->variant == FASGD_FASGD;
+    const int rule = h->variant == FASGD_FASGD       ? fasgd::kRuleFasgd
+                     : h->variant == FASGD_FASGD_STD ? fasgd::kRuleFasgdStd
+                                                     : fasgd::kRuleSgd;
     const fasgd::StatParams sp = h->stat_params();
     int k = 0;
     while (k < K) {
@@ -494,7 +497,7 @@ int fasgd_apply_pending(fasgd_t* h, int32_t K) {
                 const int slot = h->fifo[(size_t)(k + i)].stage;
                 if (slot >= 0) st = cudaStreamWaitEvent(h->stream, h->slot_ready[(size_t)slot], 0);
             }
-            if (st == cudaSuccess) st = fasgd::launch_dense(a, fas, h->num_sms, h->stream, &h->launches);
+            if (st == cudaSuccess) st = fasgd::launch_dense(a, rule, h->num_sms, h->stream, &h->launches);
             for (int i = 0; i < r && st == cudaSuccess; ++i) {  // the slots may be refilled after this
                 const int slot = h->fifo[(size_t)(k + i)].stage;
                 if (slot >= 0) {
@@ -523,7 +526,7 @@ int fasgd_apply_pending(fasgd_t* h, int32_t K) {
                 a.grad[0] = slot;
                 a.coef[0] = h->coef(h->T + k - first.j);
                 a.K = 1;
-                st = fasgd::launch_dense(a, fas, h->num_sms, h->stream, &h->launches);
+                st = fasgd::launch_dense(a, rule, h->num_sms, h->stream, &h->launches);
             }
             if (st != cudaSuccess) return h->cuda_fail(st, "fasgd_apply_pending: message push");
             k += 1;
@@ -543,7 +546,7 @@ int fasgd_apply_pending(fasgd_t* h, int32_t K) {
             a.sp = sp;
             a.err = h->dev_err;
             if (first.n_max > 0 || first.n_dev != nullptr) {
-                cudaError_t st = fasgd::launch_sparse(a, fas, h->num_sms, h->stream, &h->launches);
+                cudaError_t st = fasgd::launch_sparse(a, rule, h->num_sms, h->stream, &h->launches);
                 if (st != cudaSuccess) return h->cuda_fail(st, "fasgd_apply_pending: sparse pass");
             }
             k += 1;

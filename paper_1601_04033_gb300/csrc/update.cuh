@@ -33,6 +33,16 @@ __device__ __forceinline__ float rcp_approx(float x) {
     return y;
 }
 
+template <bool FTZ>
+__device__ __forceinline__ float sqrt_approx(float x) {
+    float y;
+    if (FTZ)
+        asm("sqrt.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    else
+        asm("sqrt.approx.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+
 // Smallest eps for which the flush-to-zero forms are exact substitutes.
 constexpr float kFtzSafeEps = 1.17549435e-38f;  // 2^-126
 
@@ -54,13 +64,18 @@ __device__ __forceinline__ void sgd_update(float& theta, float g, float coef) {
 // v and theta updates differ from a once-rounded sequence by a few ulp; v is
 // a positive weighted mean, so that difference does not grow, and theta only
 // accumulates it relative to the size of each step.
-template <bool FTZ = false>
+// STD selects the prose reading of Sec. 2.2: v averages the std itself
+// (r = sqrt(max(n - b^2, 0) + eps)) and the step divides by it.  With
+// eps >= 2^-126 the std is >= 2^-63 and v >= 2^-87, so the flush-to-zero
+// forms stay exact substitutes there too.
+template <bool FTZ = false, bool STD = false>
 __device__ __forceinline__ void fasgd_update(float& theta, float& n, float& b, float& v,
                                              float g, float coef, const StatParams& sp) {
     n = __fadd_rn(__fmul_rn(sp.gamma, n), __fmul_rn(sp.one_m_gamma, __fmul_rn(g, g)));
     b = __fadd_rn(__fmul_rn(sp.gamma, b), __fmul_rn(sp.one_m_gamma, g));
     const float var = fmaxf(__fsub_rn(n, __fmul_rn(b, b)), 0.0f);
-    const float r = rsqrt_approx<FTZ>(__fadd_rn(var, sp.eps));
+    const float rad = __fadd_rn(var, sp.eps);
+    const float r = STD ? sqrt_approx<FTZ>(rad) : rsqrt_approx<FTZ>(rad);
     v = fmaf(sp.beta, v, sp.one_m_beta * r);
     theta = fmaf(-(coef * g), rcp_approx<FTZ>(v), theta);
 }

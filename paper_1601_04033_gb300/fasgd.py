@@ -17,7 +17,7 @@ import os
 
 from . import build as _build
 
-ASGD, SASGD, FASGD = 0, 1, 2
+ASGD, SASGD, FASGD, FASGD_STD = 0, 1, 2, 3
 OK, EINVAL, ERANGE, EAGAIN, ENOMEM, ECUDA, EDEVICE = 0, -1, -2, -3, -4, -5, -6
 KMAX = 32
 STATUS_NAMES = {OK: "OK", EINVAL: "EINVAL", ERANGE: "ERANGE", EAGAIN: "EAGAIN",

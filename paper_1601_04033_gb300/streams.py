@@ -30,8 +30,8 @@ import math
 
 import numpy as np
 
-ASGD, SASGD, FASGD = 0, 1, 2
-VARIANT_NAMES = {ASGD: "asgd", SASGD: "sasgd", FASGD: "fasgd"}
+ASGD, SASGD, FASGD, FASGD_STD = 0, 1, 2, 3
+VARIANT_NAMES = {ASGD: "asgd", SASGD: "sasgd", FASGD: "fasgd", FASGD_STD: "fasgd-std"}
 
 # Sub-stream tags: each component gets its own PCG64 stream keyed by
 # (seed, tag[, slot]) so that any one can be regenerated alone.

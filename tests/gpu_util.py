@@ -103,7 +103,7 @@ class OracleRun:
 def compare_states(gs, os_, variant, where):
     names = ("theta", "n", "b", "v")
     assert gs[4] == os_[4], f"{where}: timestamps differ {gs[4]} vs {os_[4]}"
-    if variant != oracle.FASGD:
+    if variant in (oracle.ASGD, oracle.SASGD):
         assert_bitwise(gs[0], os_[0].astype(np.float32), f"{where} theta")
         return
     # n and b are formed with the same once-rounded fp32 sequence on both sides.

@@ -22,7 +22,7 @@ from fractions import Fraction
 import numpy as np
 
 import oracle
-from oracle import ASGD, FASGD, SASGD
+from oracle import ASGD, FASGD, FASGD_STD, SASGD
 
 GOLDEN = os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden")
 
@@ -79,6 +79,39 @@ def check_hand_trace(libs: Libs):
 # --------------------------------------------------------------------------
 # Constant gradient: closed-form geometric series (Eq. 4-8)
 # --------------------------------------------------------------------------
+def check_std_variant_closed_form(libs: Libs):
+    """Divide-by-std reading: under a constant gradient, v averages
+    sqrt(gamma^k (1 - gamma^k) g^2 + eps) and theta moves by coef g / v."""
+    gvals = np.array([0.8, -0.25, 3e-3, 0.0], dtype=np.float32)
+    P = gvals.shape[0]
+    gamma, beta, eps, alpha = 0.9, 0.85, 1e-4, 0.02
+    theta0 = np.array([0.01, -0.02, 0.0, 0.03], np.float32)
+    for real, steps, tol in (("f32", 30, 2e-5), ("f64", 50, 1e-11)):
+        s = _server(libs, real, P, FASGD_STD, alpha=alpha, gamma=gamma, beta=beta, eps=eps)
+        s.set_params(theta0)
+        G, B = float(np.float32(gamma)), float(np.float32(beta))
+        E, A = float(np.float32(eps)), float(np.float32(alpha))
+        g64 = gvals.astype(np.float64)
+        theta_ref = theta0.astype(np.float64).copy()
+        stds = []
+        for i in range(1, steps + 1):
+            s.push(0, s.T, gvals)
+            s.apply_pending(1)
+            gi = G ** i
+            stds.append(np.sqrt(gi * (1 - gi) * g64 ** 2 + E))
+            v_ref = (1 - B) * sum(B ** (i - k) * stds[k - 1] for k in range(1, i + 1))
+            theta_ref = theta_ref - A * g64 / v_ref
+            assert _rel(s.v, v_ref) <= tol, (real, i, "v")
+            assert np.max(np.abs(s.theta - theta_ref)) <= tol * (np.max(np.abs(theta_ref)) + 1e-3)
+    # The two readings differ (v is an average of std in one, of 1/std in the other).
+    a = _server(libs, "f32", P, FASGD)
+    b = _server(libs, "f32", P, FASGD_STD)
+    for s in (a, b):
+        s.push(0, 0, gvals)
+        s.apply_pending(1)
+    assert not np.array_equal(a.v, b.v)
+
+
 def check_constant_gradient_closed_form(libs: Libs):
     gvals = np.array([1.0, -0.5, 0.03125, -2e-3, 0.3, 7e-5, -1.25, 0.0], dtype=np.float32)
     P = gvals.shape[0]
@@ -130,10 +163,11 @@ def _series_reference(variant, theta0, events, alpha, gamma, beta, eps):
         for i in range(1, len(hist) + 1):
             tau_i, g_i = hist[i - 1]
             c_i = alpha if variant == ASGD else alpha / max(tau_i, 1)
-            if variant == FASGD:
+            if variant in (FASGD, FASGD_STD):
                 n_i = sum((1 - gamma) * gamma ** (i - k) * hist[k - 1][1] ** 2 for k in range(1, i + 1))
                 b_i = sum((1 - gamma) * gamma ** (i - k) * hist[k - 1][1] for k in range(1, i + 1))
-                rs.append(1 / math.sqrt(max(n_i - b_i ** 2, 0.0) + eps))
+                std = math.sqrt(max(n_i - b_i ** 2, 0.0) + eps)
+                rs.append(1 / std if variant == FASGD else std)
                 v_i = sum((1 - beta) * beta ** (i - k) * rs[k - 1] for k in range(1, i + 1))
                 step_sum += c_i * g_i / v_i
                 n[p], b[p], v[p] = n_i, b_i, v_i
@@ -161,7 +195,7 @@ def check_series_bruteforce(libs: Libs):
         else:
             plan.append(("dense", j, None, g))
         T += 1
-    for variant in (ASGD, SASGD, FASGD):
+    for variant in (ASGD, SASGD, FASGD, FASGD_STD):
         events = []
         for T, (kind, j, idx, g) in enumerate(plan):
             tau = T - j
@@ -585,6 +619,7 @@ def check_protocol_errors(libs: Libs):
 ALL_CHECKS = [
     check_hand_trace,
     check_constant_gradient_closed_form,
+    check_std_variant_closed_form,
     check_series_bruteforce,
     check_variant_invariants,
     check_dense_equals_full_sparse,

@@ -56,7 +56,7 @@ def test_host_side_argument_checks(binding):
     for P, lam, alpha, var in ((0, 4, 0.1, 2), (-5, 4, 0.1, 2), (1 << 31, 4, 0.1, 2),
                                (10, 0, 0.1, 2), (10, 1 << 21, 0.1, 2),
                                (10, 4, float("nan"), 2), (10, 4, float("inf"), 0),
-                               (10, 4, 0.1, 3), (10, 4, 0.1, -1)):
+                               (10, 4, 0.1, 4), (10, 4, 0.1, -1)):
         rc, h = f.fasgd_create(P, lam, alpha, var)
         assert rc == f.EINVAL and h is None, (P, lam, alpha, var)
         assert f.fasgd_last_error(None)

@@ -294,3 +294,25 @@ def test_select_at_the_threshold_bit_exact():
     assert 0.2 * P < m < 0.8 * P          # the decisions really are split
     assert_bitwise(gi, oi, "idx at threshold")
     assert_bitwise(gv, ov, "val at threshold")
+
+
+def test_sparse_apply_divide_by_std_matches_dense_at_c0():
+    import torch
+    w = W["bfasgd-25m"]
+    P = 20_011
+    pool = streams.gradient_pool(w, P, 4)
+    th0 = streams.theta0(w, P)
+    ps = streams.push_stream(w.replace(R=4), 25, 1)
+    a = GpuRun(w, oracle.FASGD_STD, P, pool, th0)
+    b = GpuRun(w, oracle.FASGD_STD, P, pool, th0, c_push=0.0, seed=SEED)
+    o = OracleRun(w, oracle.FASGD_STD, P, pool, th0)
+    for t in range(25):
+        cl, js, sl = ps.batch(t)
+        a.push_batch(cl, js, sl)
+        o.push_batch(cl, js, sl)
+        _, _, m, (idx, val, n) = _select_gpu(b.srv, int(cl[0]), b.pool[int(sl[0])])
+        b.srv.push_sparse(int(cl[0]), int(js[0]), idx, val, n_dev=n, n_max=P)
+        b.srv.apply_pending(1)
+    for x, y, name in zip(a.state()[:4], b.state()[:4], ("theta", "n", "b", "v")):
+        assert_bitwise(x, y, name)
+    compare_states(a.state(), o.state(), oracle.FASGD_STD, "std variant")

@@ -173,3 +173,22 @@ def test_eps_at_ftz_threshold():
     """eps = 2^-126 exactly (the smallest eps on the flush-to-zero path)."""
     w = W["fasgd-7850"]
     run_parity(w, oracle.FASGD, w.P, 200, 4, eps=float(np.float32(2.0 ** -126)))
+
+
+@pytest.mark.parametrize("K,eps", [(1, 1e-4), (8, 1e-4), (13, 1e-4), (8, 0.0)])
+def test_divide_by_std_variant(K, eps):
+    """The prose reading of Eq. 7 (v averages the std, the step divides by it)."""
+    w = W["fasgd-25m-k8"].replace(R=max(2 * K, 16))
+    n = 100 * K // np.gcd(100, K)
+    run_parity(w, oracle.FASGD_STD, 30_007, n, K, eps=eps)
+
+
+def test_divide_by_std_full_stream_7850():
+    """The full 200-push stream of the 7,850-parameter workload.  Dividing by
+    the std (~1e-2 and below) instead of multiplying by it makes steps four
+    orders of magnitude larger at the same alpha, so theta swings through
+    values near 1 and ends near 1e-3 -- fp32 rounding of those swings alone
+    exceeds the bound; the variant is run at alpha / 1000, the scale at which
+    its steps match FASGD's."""
+    w = W["fasgd-7850"]
+    run_parity(w.replace(alpha=w.alpha * 1e-3), oracle.FASGD_STD, w.P, w.pushes, 1)

@@ -49,6 +49,7 @@ MUTANTS = {
     "mean_v_first_only": ("s += (double)v[p];", "s = (double)v[p];"),
     "message_draw_collides": ("uint32_t ctr[4] = {0xFFFFFFFFu,", "uint32_t ctr[4] = {0u,"),
     "message_draw_ignores_stream": ("{0xFFFFFFFFu, client | (stream << 31),", "{0xFFFFFFFFu, client,"),
+    "std_variant_inverts": ("REAL r = ora_sqrt(var + eps);\n        *v = beta", "REAL r = 1 / ora_sqrt(var + eps);\n        *v = beta"),
     "decide_not_strict": ("prod == A && err < 0.0f", "prod == A && err <= 0.0f"),
     "decide_ignores_err": ("if (prod == A && err < 0.0f)\n        return 1;\n", ""),
     "decide_drops_eps": ("float a = v + eps_b;", "float a = v;"),
