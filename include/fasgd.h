@@ -106,6 +106,19 @@ FASGD_API void fasgd_destroy(fasgd_t* h);
 FASGD_API int fasgd_set_hparams(fasgd_t* h, float gamma, float beta, float eps, float c_push,
                       float eps_b, uint64_t seed);
 
+/*
+ * fasgd_set_exact -- choose the arithmetic of the FASGD update (Eq. 4-8):
+ * 0 (default) uses the hardware inverse square root / reciprocal and fused
+ * multiply-adds for v and theta (n and b are exact either way; v and theta
+ * stay within a few ulp per step of the exact sequence, 1e-5 relative over
+ * thousands of pushes); 1 computes every operation correctly rounded and
+ * unfused -- the exact fp32 sequence, bit for bit what an IEEE CPU computes,
+ * for runs that must reproduce exactly (e.g. closed-loop simulations, where
+ * feedback can amplify ulp-level differences).  ASGD/SASGD are exact in both
+ * modes.  Errors: EINVAL, EAGAIN (pushes pending).
+ */
+FASGD_API int fasgd_set_exact(fasgd_t* h, int32_t exact);
+
 /* Stream every later call is enqueued on (a cudaStream_t; NULL = legacy default stream). */
 FASGD_API int fasgd_set_stream(fasgd_t* h, void* stream);
 
@@ -339,8 +352,31 @@ FASGD_API int bfasgd_select_compact_noalloc(int64_t P, const float* grad, const 
                                             uint64_t push_no, int32_t* idx, float* val,
                                             int64_t* n_dev, void* stream);
 
+/*
+ * Closed-loop simulation support (the paper's FRED simulator, Sec. 3, with a
+ * synthetic objective in place of its MNIST model; no handle needed).
+ *
+ * fasgd_sim_quadratic_grad -- a client's stochastic gradient of
+ * f(theta) = 1/2 sum_p h_p (theta_p - star_p)^2 at its copy theta:
+ * grad_p = fl(fl(h_p (theta_p - star_p)) + fl(sigma_p xi_p)), xi_p uniform
+ * with unit variance, xi_p = fl(((u + 1/2) 2^-23 - 1/2) * fl(sqrt 12)), u the
+ * top 23 bits of word (p mod 4) of Philox4x32-10 at counter
+ * (p div 4, client + 2^30, n, n >> 32), key = seed (n: the client's gradient
+ * count).  All pointers device fp32[P], 16-byte aligned; 0 <= client < 2^30.
+ * fasgd_sim_quadratic_loss -- *loss (device double) = f(theta), terms in
+ * fp32 summed in a fixed order (reproducible); scratch: device, >= 1024
+ * doubles.  Both run on `stream` (cudaStream_t, NULL = legacy default).
+ * Errors: EINVAL (text via fasgd_last_error(NULL)), ECUDA.
+ */
+FASGD_API int fasgd_sim_quadratic_grad(int64_t P, const float* theta, const float* h,
+                                       const float* star, const float* sigma, uint64_t seed,
+                                       int32_t client, uint64_t n, float* grad, void* stream);
+FASGD_API int fasgd_sim_quadratic_loss(int64_t P, const float* theta, const float* h,
+                                       const float* star, double* scratch, double* loss,
+                                       void* stream);
+
 /* Text of the last failure on h, or, when h is NULL, of the last failed call
- * made without a handle (fasgd_create, bfasgd_fetch_apply,
+ * made without a handle (fasgd_create, bfasgd_fetch_apply, fasgd_sim_*,
  * bfasgd_select_compact_noalloc). */
 FASGD_API const char* fasgd_last_error(const fasgd_t* h);
 

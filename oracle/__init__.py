@@ -88,6 +88,10 @@ def load_library(path: str, real: str) -> ctypes.CDLL:
     lib.ora_mean_v.argtypes = [i64, P]
     lib.ora_draw_message.restype = u32
     lib.ora_draw_message.argtypes = [u64, u32, u32, u64]
+    lib.ora_sim_grad.restype = None
+    lib.ora_sim_grad.argtypes = [i64, P, P, P, P, u64, u32, u64, P]
+    lib.ora_sim_loss.restype = ctypes.c_double
+    lib.ora_sim_loss.argtypes = [i64, P, P, P]
     assert lib.ora_real_bytes() == (4 if real == "f32" else 8)
     return lib
 
@@ -182,6 +186,21 @@ def mean_v(v: np.ndarray, real: str = "f32", lib=None) -> float:
 def draw_message(seed: int, stream: int, client: int, n: int, lib=None) -> int:
     """24-bit draw of a client's n-th push (stream 0) or fetch (stream 1) message."""
     return int((lib or _load("f32")).ora_draw_message(seed, stream, client, n))
+
+
+def sim_grad(theta, h, star, sigma, seed: int, client: int, n: int, lib=None) -> np.ndarray:
+    """Stochastic gradient of the synthetic quadratic at theta (fp32[P])."""
+    arrs = [np.ascontiguousarray(x, dtype=np.float32) for x in (theta, h, star, sigma)]
+    g = np.empty_like(arrs[0])
+    (lib or _load("f32")).ora_sim_grad(arrs[0].shape[0], *[_ptr(x) for x in arrs], seed, client,
+                                       n, _ptr(g))
+    return g
+
+
+def sim_loss(theta, h, star, lib=None) -> float:
+    """f(theta) = 1/2 sum h (theta - star)^2 (terms in fp32, sum in fp64)."""
+    arrs = [np.ascontiguousarray(x, dtype=np.float32) for x in (theta, h, star)]
+    return float((lib or _load("f32")).ora_sim_loss(arrs[0].shape[0], *[_ptr(x) for x in arrs]))
 
 
 class OracleError(Exception):

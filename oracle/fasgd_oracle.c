@@ -291,3 +291,46 @@ uint32_t ora_draw_message(uint64_t seed, uint32_t stream, uint32_t client, uint6
     ora_philox4x32_10(ctr, key, out);
     return out[0] >> 8;
 }
+
+/*
+ * Closed-loop simulation (in the spirit of the paper's FRED simulator,
+ * Sec. 3): clients compute stochastic gradients of a synthetic separable
+ * quadratic f(theta) = 1/2 sum_p h_p (theta_p - star_p)^2 on their own
+ * (stale) copies.  The gradient noise is uniform with variance sigma_p^2,
+ * built from a 23-bit draw so that every operation is exact or rounded once
+ * in fp32:
+ *   u  = Philox word (p mod 4) at counter (p div 4, client + 2^30, n, n >> 32),
+ *        top 23 bits (n = the client's gradient count);
+ *   x  = (u + 1/2) 2^-23 - 1/2            (exact, in (-1/2, 1/2))
+ *   xi = fl(x * fl(sqrt(12)))             (unit variance)
+ *   g  = fl( fl(h (theta - star)) + fl(sigma xi) ).
+ */
+void ora_sim_grad(int64_t P, const float *theta, const float *h, const float *star,
+                  const float *sigma, uint64_t seed, uint32_t client, uint64_t n, float *g)
+{
+    const float root12 = 3.46410161513775458705f;
+    uint32_t key[2] = {(uint32_t)seed, (uint32_t)(seed >> 32)};
+    for (int64_t p = 0; p < P; p++) {
+        uint32_t ctr[4] = {(uint32_t)(p >> 2), client | (1u << 30), (uint32_t)n,
+                           (uint32_t)(n >> 32)};
+        uint32_t out[4];
+        ora_philox4x32_10(ctr, key, out);
+        uint32_t u = out[p & 3] >> 9;
+        float x = ((float)u + 0.5f) * (1.0f / 8388608.0f) - 0.5f;
+        float xi = x * root12;
+        float d = theta[p] - star[p];
+        g[p] = h[p] * d + sigma[p] * xi;
+    }
+}
+
+/* f(theta) = 1/2 sum_p h_p (theta_p - star_p)^2, each term in fp32, summed in fp64. */
+double ora_sim_loss(int64_t P, const float *theta, const float *h, const float *star)
+{
+    double s = 0.0;
+    for (int64_t p = 0; p < P; p++) {
+        float d = theta[p] - star[p];
+        float t = h[p] * (d * d);
+        s += (double)t;
+    }
+    return 0.5 * s;
+}

@@ -105,15 +105,15 @@ __device__ __forceinline__ void bulk_load(void* dst, const void* src, uint32_t b
 }
 
 // ---- the element update on four consecutive parameters --------------------
-template <int RULE, bool FTZ>
+template <int RULE, int ARITH>
 __device__ __forceinline__ void update4(float4& th, float4& n, float4& b, float4& v, const float4& g,
                                         float coef, const StatParams& sp) {
     constexpr bool STD = RULE == kRuleFasgdStd;
     if (RULE != kRuleSgd) {
-        fasgd_update<FTZ, STD>(th.x, n.x, b.x, v.x, g.x, coef, sp);
-        fasgd_update<FTZ, STD>(th.y, n.y, b.y, v.y, g.y, coef, sp);
-        fasgd_update<FTZ, STD>(th.z, n.z, b.z, v.z, g.z, coef, sp);
-        fasgd_update<FTZ, STD>(th.w, n.w, b.w, v.w, g.w, coef, sp);
+        rule_update<ARITH, STD>(th.x, n.x, b.x, v.x, g.x, coef, sp);
+        rule_update<ARITH, STD>(th.y, n.y, b.y, v.y, g.y, coef, sp);
+        rule_update<ARITH, STD>(th.z, n.z, b.z, v.z, g.z, coef, sp);
+        rule_update<ARITH, STD>(th.w, n.w, b.w, v.w, g.w, coef, sp);
     } else {
         sgd_update(th.x, g.x, coef);
         sgd_update(th.y, g.y, coef);
@@ -124,7 +124,7 @@ __device__ __forceinline__ void update4(float4& th, float4& n, float4& b, float4
 
 // Parameters [begin, P) with plain loads, by the consumer threads of one
 // block; begin is a multiple of 4.
-template <int RULE, bool FTZ>
+template <int RULE, int ARITH>
 __device__ void apply_range_direct(const DenseArgs& a, int64_t begin, int tid) {
     constexpr bool FAS = RULE != kRuleSgd;
     const int64_t end_q = a.P & ~int64_t(3);
@@ -138,7 +138,7 @@ __device__ void apply_range_direct(const DenseArgs& a, int64_t begin, int tid) {
         }
         for (int k = 0; k < a.K; ++k) {
             const float4 g = __ldcs(reinterpret_cast<const float4*>(a.grad[k] + e));
-            update4<RULE, FTZ>(th, n, b, v, g, a.coef[k], a.sp);
+            update4<RULE, ARITH>(th, n, b, v, g, a.coef[k], a.sp);
         }
         *reinterpret_cast<float4*>(a.theta + e) = th;
         if (FAS) {
@@ -158,7 +158,7 @@ __device__ void apply_range_direct(const DenseArgs& a, int64_t begin, int tid) {
         for (int k = 0; k < a.K; ++k) {
             const float g = __ldcs(a.grad[k] + p);
             if (FAS)
-                fasgd_update<FTZ, RULE == kRuleFasgdStd>(th, n, b, v, g, a.coef[k], a.sp);
+                rule_update<ARITH, RULE == kRuleFasgdStd>(th, n, b, v, g, a.coef[k], a.sp);
             else
                 sgd_update(th, g, a.coef[k]);
         }
@@ -177,9 +177,9 @@ struct Ring {
     int chunks;     // stages per tile: ceil(K / CH)
 };
 
-// RULE: kRuleSgd / kRuleFasgd / kRuleFasgdStd; FTZ: flush-to-zero MUFU forms
-// (see update.cuh); CH: gradient slices per stage.
-template <int RULE, bool FTZ, int CH>
+// RULE: kRuleSgd / kRuleFasgd / kRuleFasgdStd; ARITH: kArithApprox /
+// kArithApproxFtz / kArithExact (see update.cuh); CH: gradient slices per stage.
+template <int RULE, int ARITH, int CH>
 __global__ void __launch_bounds__(kThreads, 1)
 fasgd_dense_kernel(const __grid_constant__ DenseArgs a, const Ring ring, const int64_t ntiles) {
     constexpr bool FAS = RULE != kRuleSgd;
@@ -273,7 +273,7 @@ fasgd_dense_kernel(const __grid_constant__ DenseArgs a, const Ring ring, const i
                 __syncwarp();
                 if (lane == 0) mbar_arrive(&empty[s]);  // inputs are in registers
 #pragma unroll
-                for (int j = 0; j < CH; ++j) update4<RULE, FTZ>(th, n, b, v, g[j], a.coef[k0 + j], a.sp);
+                for (int j = 0; j < CH; ++j) update4<RULE, ARITH>(th, n, b, v, g[j], a.coef[k0 + j], a.sp);
             } else {               // the last, partial chunk
                 const int ng = a.K - k0;
 #pragma unroll
@@ -283,7 +283,7 @@ fasgd_dense_kernel(const __grid_constant__ DenseArgs a, const Ring ring, const i
                 if (lane == 0) mbar_arrive(&empty[s]);
 #pragma unroll
                 for (int j = 0; j < CH; ++j)
-                    if (j < ng) update4<RULE, FTZ>(th, n, b, v, g[j], a.coef[k0 + j], a.sp);
+                    if (j < ng) update4<RULE, ARITH>(th, n, b, v, g[j], a.coef[k0 + j], a.sp);
             }
             if (++s == ring.stages) {
                 s = 0;
@@ -300,10 +300,10 @@ fasgd_dense_kernel(const __grid_constant__ DenseArgs a, const Ring ring, const i
         }
     }
     // Parameters after the last full tile.
-    if (ok && blockIdx.x == gridDim.x - 1) apply_range_direct<RULE, FTZ>(a, ntiles * kTile, tid);
+    if (ok && blockIdx.x == gridDim.x - 1) apply_range_direct<RULE, ARITH>(a, ntiles * kTile, tid);
 }
 
-template <int RULE, bool FTZ, int CH>
+template <int RULE, int ARITH, int CH>
 cudaError_t launch_ch(const DenseArgs& a, int num_sms, cudaStream_t stream) {
     constexpr int kState = RULE != kRuleSgd ? 4 : 1;
     constexpr int kStageBytes = (kState + CH) * kTile * 4;
@@ -314,7 +314,7 @@ cudaError_t launch_ch(const DenseArgs& a, int num_sms, cudaStream_t stream) {
     const size_t smem = (size_t)ring.stages * kStageBytes + 2 * ring.stages * sizeof(uint64_t);
     static bool configured = false;  // per instantiation
     if (!configured) {
-        cudaError_t st = cudaFuncSetAttribute(fasgd_dense_kernel<RULE, FTZ, CH>,
+        cudaError_t st = cudaFuncSetAttribute(fasgd_dense_kernel<RULE, ARITH, CH>,
                                               cudaFuncAttributeMaxDynamicSharedMemorySize,
                                               kSmemBudget);
         if (st != cudaSuccess) return st;
@@ -323,33 +323,35 @@ cudaError_t launch_ch(const DenseArgs& a, int num_sms, cudaStream_t stream) {
     const int64_t ntiles = a.P / kTile;
     int64_t grid = ntiles < num_sms ? ntiles : num_sms;  // one block per SM (shared-memory bound)
     if (grid < 1) grid = 1;
-    fasgd_dense_kernel<RULE, FTZ, CH><<<(unsigned)grid, kThreads, smem, stream>>>(a, ring, ntiles);
+    fasgd_dense_kernel<RULE, ARITH, CH><<<(unsigned)grid, kThreads, smem, stream>>>(a, ring, ntiles);
     return cudaGetLastError();
 }
 
-template <int RULE, bool FTZ>
+template <int RULE, int ARITH>
 cudaError_t launch_rule(const DenseArgs& a, int num_sms, cudaStream_t stream) {
     // Gradient slices per stage: K rounded up to a power of two, at most 8.
-    if (a.K > 4) return launch_ch<RULE, FTZ, 8>(a, num_sms, stream);
-    if (a.K > 2) return launch_ch<RULE, FTZ, 4>(a, num_sms, stream);
-    if (a.K > 1) return launch_ch<RULE, FTZ, 2>(a, num_sms, stream);
-    return launch_ch<RULE, FTZ, 1>(a, num_sms, stream);
+    if (a.K > 4) return launch_ch<RULE, ARITH, 8>(a, num_sms, stream);
+    if (a.K > 2) return launch_ch<RULE, ARITH, 4>(a, num_sms, stream);
+    if (a.K > 1) return launch_ch<RULE, ARITH, 2>(a, num_sms, stream);
+    return launch_ch<RULE, ARITH, 1>(a, num_sms, stream);
 }
 
 }  // namespace
 
-cudaError_t launch_dense(const DenseArgs& a, int rule, int num_sms, cudaStream_t stream,
-                         int64_t* launches) {
+cudaError_t launch_dense(const DenseArgs& a, int rule, bool exact, int num_sms,
+                         cudaStream_t stream, int64_t* launches) {
     const bool ftz = a.sp.eps >= kFtzSafeEps;
     cudaError_t st;
     if (rule == kRuleSgd)
-        st = launch_rule<kRuleSgd, false>(a, num_sms, stream);
+        st = launch_rule<kRuleSgd, kArithApprox>(a, num_sms, stream);  // exact in every mode
     else if (rule == kRuleFasgd)
-        st = ftz ? launch_rule<kRuleFasgd, true>(a, num_sms, stream)
-                 : launch_rule<kRuleFasgd, false>(a, num_sms, stream);
+        st = exact ? launch_rule<kRuleFasgd, kArithExact>(a, num_sms, stream)
+             : ftz ? launch_rule<kRuleFasgd, kArithApproxFtz>(a, num_sms, stream)
+                   : launch_rule<kRuleFasgd, kArithApprox>(a, num_sms, stream);
     else
-        st = ftz ? launch_rule<kRuleFasgdStd, true>(a, num_sms, stream)
-                 : launch_rule<kRuleFasgdStd, false>(a, num_sms, stream);
+        st = exact ? launch_rule<kRuleFasgdStd, kArithExact>(a, num_sms, stream)
+             : ftz ? launch_rule<kRuleFasgdStd, kArithApproxFtz>(a, num_sms, stream)
+                   : launch_rule<kRuleFasgdStd, kArithApprox>(a, num_sms, stream);
     if (st == cudaSuccess) ++*launches;
     return st;
 }

@@ -110,16 +110,43 @@ struct MessageArgs {
 
 int32_t message_partial_blocks(int64_t P);
 
+// Closed-loop simulation: stochastic gradient and loss of the synthetic
+// quadratic objective (sim.cu).
+struct SimGradArgs {
+    const float* theta;   // the client's copy, fp32[P], 16-byte aligned
+    const float* h;       // curvatures
+    const float* star;    // minimiser
+    const float* sigma;   // noise scales
+    float* grad;          // output
+    int64_t P;
+    uint32_t round_key0[10];
+    uint32_t round_key1[10];
+    uint32_t client, n_lo, n_hi;
+};
+
+constexpr int kSimLossScratch = 1024;   // doubles of scratch the loss needs
+
+struct SimLossArgs {
+    const float* theta;
+    const float* h;
+    const float* star;
+    int64_t P;
+    double* partial;      // kSimLossScratch doubles
+    double* loss;         // output (device)
+};
+
 // Launchers: enqueue on `stream`, return the launch status.
 // `launches` is incremented by the number of kernels enqueued.
-cudaError_t launch_dense(const DenseArgs& a, int rule, int num_sms, cudaStream_t stream,
+cudaError_t launch_dense(const DenseArgs& a, int rule, bool exact, int num_sms, cudaStream_t stream,
                          int64_t* launches);
-cudaError_t launch_sparse(const SparseArgs& a, int rule, int num_sms, cudaStream_t stream,
+cudaError_t launch_sparse(const SparseArgs& a, int rule, bool exact, int num_sms, cudaStream_t stream,
                           int64_t* launches);
 cudaError_t launch_select(const SelectArgs& a, cudaStream_t stream, int64_t* launches);
 cudaError_t launch_scatter(const ScatterArgs& a, int num_sms, cudaStream_t stream);
 cudaError_t launch_message(const MessageArgs& a, int num_sms, cudaStream_t stream,
                            int64_t* launches);
+cudaError_t launch_sim_grad(const SimGradArgs& a, int num_sms, cudaStream_t stream);
+cudaError_t launch_sim_loss(const SimLossArgs& a, cudaStream_t stream);
 
 inline int32_t select_tiles(int64_t P) {
     return (int32_t)((P + kSelectTile - 1) / kSelectTile);

@@ -82,6 +82,7 @@ struct fasgd_s {
     int32_t variant = FASGD_FASGD;
     float gamma = 0.95f, beta = 0.95f, eps = 1e-4f, c_push = 0.f, eps_b = 1e-8f;
     float c_fetch = 0.f;
+    bool exact = false;     // exact fp32 arithmetic instead of the fast forms
     uint64_t seed = 0;
     cudaStream_t stream = nullptr;
     int device = 0;
@@ -327,6 +328,13 @@ int fasgd_set_hparams(fasgd_t* h, float gamma, float beta, float eps, float c_pu
     return FASGD_OK;
 }
 
+int fasgd_set_exact(fasgd_t* h, int32_t exact) {
+    if (h == nullptr) return FASGD_EINVAL;
+    if (!h->fifo.empty()) return h->fail(FASGD_EAGAIN, "pushes are pending");
+    h->exact = exact != 0;
+    return FASGD_OK;
+}
+
 int fasgd_set_stream(fasgd_t* h, void* stream) {
     if (h == nullptr) return FASGD_EINVAL;
     if (!h->fifo.empty()) return h->fail(FASGD_EAGAIN, "pushes are pending");
@@ -497,7 +505,7 @@ int fasgd_apply_pending(fasgd_t* h, int32_t K) {
                 const int slot = h->fifo[(size_t)(k + i)].stage;
                 if (slot >= 0) st = cudaStreamWaitEvent(h->stream, h->slot_ready[(size_t)slot], 0);
             }
-            if (st == cudaSuccess) st = fasgd::launch_dense(a, rule, h->num_sms, h->stream, &h->launches);
+            if (st == cudaSuccess) st = fasgd::launch_dense(a, rule, h->exact, h->num_sms, h->stream, &h->launches);
             for (int i = 0; i < r && st == cudaSuccess; ++i) {  // the slots may be refilled after this
                 const int slot = h->fifo[(size_t)(k + i)].stage;
                 if (slot >= 0) {
@@ -526,7 +534,7 @@ int fasgd_apply_pending(fasgd_t* h, int32_t K) {
                 a.grad[0] = slot;
                 a.coef[0] = h->coef(h->T + k - first.j);
                 a.K = 1;
-                st = fasgd::launch_dense(a, rule, h->num_sms, h->stream, &h->launches);
+                st = fasgd::launch_dense(a, rule, h->exact, h->num_sms, h->stream, &h->launches);
             }
             if (st != cudaSuccess) return h->cuda_fail(st, "fasgd_apply_pending: message push");
             k += 1;
@@ -546,7 +554,7 @@ int fasgd_apply_pending(fasgd_t* h, int32_t K) {
             a.sp = sp;
             a.err = h->dev_err;
             if (first.n_max > 0 || first.n_dev != nullptr) {
-                cudaError_t st = fasgd::launch_sparse(a, rule, h->num_sms, h->stream, &h->launches);
+                cudaError_t st = fasgd::launch_sparse(a, rule, h->exact, h->num_sms, h->stream, &h->launches);
                 if (st != cudaSuccess) return h->cuda_fail(st, "fasgd_apply_pending: sparse pass");
             }
             k += 1;
@@ -655,6 +663,63 @@ int bfasgd_fetch_apply(int64_t P, float* theta_client, const int32_t* idx, const
     if (st == cudaSuccess) st = fasgd::launch_scatter(a, sms, static_cast<cudaStream_t>(stream));
     if (st != cudaSuccess) {
         g_create_error = std::string("bfasgd_fetch_apply: ") + cudaGetErrorString(st);
+        return FASGD_ECUDA;
+    }
+    return FASGD_OK;
+}
+
+int fasgd_sim_quadratic_grad(int64_t P, const float* theta, const float* hcurv, const float* star,
+                             const float* sigma, uint64_t seed, int32_t client, uint64_t n,
+                             float* grad, void* stream) {
+    if (P < 1 || P > FASGD_PMAX || client < 0 || client >= (1 << 30)) {
+        g_create_error = "fasgd_sim_quadratic_grad: P or client out of range";
+        return FASGD_EINVAL;
+    }
+    const void* ptrs[] = {theta, hcurv, star, sigma, grad};
+    for (const void* q : ptrs)
+        if (q == nullptr || !aligned(q, 16)) {
+            g_create_error = "fasgd_sim_quadratic_grad: pointers must be non-NULL, 16-byte aligned";
+            return FASGD_EINVAL;
+        }
+    int dev = 0, sms = 0;
+    cudaError_t st = cudaGetDevice(&dev);
+    if (st == cudaSuccess) st = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    fasgd::SimGradArgs a;
+    a.theta = theta;
+    a.h = hcurv;
+    a.star = star;
+    a.sigma = sigma;
+    a.grad = grad;
+    a.P = P;
+    fasgd::philox_key_schedule(seed, a.round_key0, a.round_key1);
+    a.client = (uint32_t)client;
+    a.n_lo = (uint32_t)n;
+    a.n_hi = (uint32_t)(n >> 32);
+    if (st == cudaSuccess) st = fasgd::launch_sim_grad(a, sms, static_cast<cudaStream_t>(stream));
+    if (st != cudaSuccess) {
+        g_create_error = std::string("fasgd_sim_quadratic_grad: ") + cudaGetErrorString(st);
+        return FASGD_ECUDA;
+    }
+    return FASGD_OK;
+}
+
+int fasgd_sim_quadratic_loss(int64_t P, const float* theta, const float* hcurv, const float* star,
+                             double* scratch, double* loss, void* stream) {
+    if (P < 1 || P > FASGD_PMAX || theta == nullptr || hcurv == nullptr || star == nullptr ||
+        scratch == nullptr || loss == nullptr || !aligned(scratch, 8) || !aligned(loss, 8)) {
+        g_create_error = "fasgd_sim_quadratic_loss: bad argument";
+        return FASGD_EINVAL;
+    }
+    fasgd::SimLossArgs a;
+    a.theta = theta;
+    a.h = hcurv;
+    a.star = star;
+    a.P = P;
+    a.partial = scratch;
+    a.loss = loss;
+    cudaError_t st = fasgd::launch_sim_loss(a, static_cast<cudaStream_t>(stream));
+    if (st != cudaSuccess) {
+        g_create_error = std::string("fasgd_sim_quadratic_loss: ") + cudaGetErrorString(st);
         return FASGD_ECUDA;
     }
     return FASGD_OK;

@@ -20,7 +20,7 @@ namespace {
 constexpr int kSparseThreads = 256;
 constexpr int kUnroll = 4;
 
-template <int RULE>
+template <int RULE, bool EXACT>
 __global__ void __launch_bounds__(kSparseThreads) fasgd_sparse_kernel(const __grid_constant__ SparseArgs a) {
     constexpr bool FAS = RULE != kRuleSgd;
     int64_t count = a.count_max;
@@ -74,8 +74,8 @@ __global__ void __launch_bounds__(kSparseThreads) fasgd_sparse_kernel(const __gr
         for (int u = 0; u < kUnroll; ++u) {
             if (ok[u]) {
                 if (FAS) {
-                    fasgd_update<false, RULE == kRuleFasgdStd>(th[u], n[u], b[u], v[u], g[u],
-                                                               a.coef, a.sp);
+                    rule_update<EXACT ? kArithExact : kArithApprox, RULE == kRuleFasgdStd>(
+                        th[u], n[u], b[u], v[u], g[u], a.coef, a.sp);
                     a.n[p[u]] = n[u];
                     a.b[p[u]] = b[u];
                     a.v[p[u]] = v[u];
@@ -88,12 +88,12 @@ __global__ void __launch_bounds__(kSparseThreads) fasgd_sparse_kernel(const __gr
     }
 }
 
-template <int RULE>
+template <int RULE, bool EXACT>
 cudaError_t launch_rule(const SparseArgs& a, int num_sms, cudaStream_t stream) {
     static int blocks_per_sm = 0;
     if (blocks_per_sm == 0) {
         cudaError_t st = cudaOccupancyMaxActiveBlocksPerMultiprocessor(
-            &blocks_per_sm, fasgd_sparse_kernel<RULE>, kSparseThreads, 0);
+            &blocks_per_sm, fasgd_sparse_kernel<RULE, EXACT>, kSparseThreads, 0);
         if (st != cudaSuccess) return st;
         if (blocks_per_sm < 1) blocks_per_sm = 1;
     }
@@ -103,7 +103,7 @@ cudaError_t launch_rule(const SparseArgs& a, int num_sms, cudaStream_t stream) {
     const int64_t cap = (int64_t)num_sms * blocks_per_sm;
     if (want > cap) want = cap;
     if (want < 1) want = 1;
-    fasgd_sparse_kernel<RULE><<<(unsigned)want, kSparseThreads, 0, stream>>>(a);
+    fasgd_sparse_kernel<RULE, EXACT><<<(unsigned)want, kSparseThreads, 0, stream>>>(a);
     return cudaGetLastError();
 }
 
@@ -142,11 +142,17 @@ cudaError_t launch_scatter(const ScatterArgs& a, int num_sms, cudaStream_t strea
     return cudaGetLastError();
 }
 
-cudaError_t launch_sparse(const SparseArgs& a, int rule, int num_sms, cudaStream_t stream,
-                          int64_t* launches) {
-    cudaError_t st = rule == kRuleSgd     ? launch_rule<kRuleSgd>(a, num_sms, stream)
-                     : rule == kRuleFasgd ? launch_rule<kRuleFasgd>(a, num_sms, stream)
-                                          : launch_rule<kRuleFasgdStd>(a, num_sms, stream);
+cudaError_t launch_sparse(const SparseArgs& a, int rule, bool exact, int num_sms,
+                          cudaStream_t stream, int64_t* launches) {
+    cudaError_t st;
+    if (rule == kRuleSgd)
+        st = launch_rule<kRuleSgd, false>(a, num_sms, stream);
+    else if (rule == kRuleFasgd)
+        st = exact ? launch_rule<kRuleFasgd, true>(a, num_sms, stream)
+                   : launch_rule<kRuleFasgd, false>(a, num_sms, stream);
+    else
+        st = exact ? launch_rule<kRuleFasgdStd, true>(a, num_sms, stream)
+                   : launch_rule<kRuleFasgdStd, false>(a, num_sms, stream);
     if (st == cudaSuccess) ++*launches;
     return st;
 }

@@ -80,4 +80,35 @@ __device__ __forceinline__ void fasgd_update(float& theta, float& n, float& b, f
     theta = fmaf(-(coef * g), rcp_approx<FTZ>(v), theta);
 }
 
+// The same rule with every operation correctly rounded and none fused
+// (IEEE square root and division, separate multiplies and adds): the exact
+// fp32 sequence Eq. 4-8 define, bit for bit on any IEEE machine.  Selected
+// per handle (fasgd_set_exact) where results must be reproducible bit for
+// bit, e.g. in closed-loop simulations; it costs a division and a square
+// root per element-push on the pipes the fast form leaves idle.
+template <bool STD = false>
+__device__ __forceinline__ void fasgd_update_exact(float& theta, float& n, float& b, float& v,
+                                                   float g, float coef, const StatParams& sp) {
+    n = __fadd_rn(__fmul_rn(sp.gamma, n), __fmul_rn(sp.one_m_gamma, __fmul_rn(g, g)));
+    b = __fadd_rn(__fmul_rn(sp.gamma, b), __fmul_rn(sp.one_m_gamma, g));
+    const float var = fmaxf(__fsub_rn(n, __fmul_rn(b, b)), 0.0f);
+    const float root = __fsqrt_rn(__fadd_rn(var, sp.eps));
+    const float r = STD ? root : __fdiv_rn(1.0f, root);
+    v = __fadd_rn(__fmul_rn(sp.beta, v), __fmul_rn(sp.one_m_beta, r));
+    theta = __fsub_rn(theta, __fdiv_rn(__fmul_rn(coef, g), v));
+}
+
+// Arithmetic of a pass: hardware approximations (subnormal-preserving or
+// flush-to-zero forms) or the exact sequence.
+enum : int { kArithApprox = 0, kArithApproxFtz = 1, kArithExact = 2 };
+
+template <int ARITH, bool STD>
+__device__ __forceinline__ void rule_update(float& theta, float& n, float& b, float& v, float g,
+                                            float coef, const StatParams& sp) {
+    if (ARITH == kArithExact)
+        fasgd_update_exact<STD>(theta, n, b, v, g, coef, sp);
+    else
+        fasgd_update<ARITH == kArithApproxFtz, STD>(theta, n, b, v, g, coef, sp);
+}
+
 }  // namespace fasgd

@@ -32,6 +32,7 @@ SIGNATURES = {
     "fasgd_destroy": (None, [_p]),
     "fasgd_set_hparams": (_i32, [_p, _f32, _f32, _f32, _f32, _f32, _u64]),
     "fasgd_set_stream": (_i32, [_p, _p]),
+    "fasgd_set_exact": (_i32, [_p, _i32]),
     "fasgd_set_params": (_i32, [_p, _p]),
     "fasgd_push": (_i32, [_p, _i32, _i64, _p]),
     "fasgd_push_host": (_i32, [_p, _i32, _i64, _p]),
@@ -54,6 +55,8 @@ SIGNATURES = {
     "fasgd_set_fetch_counts": (_i32, [_p, _p]),
     "bfasgd_push_message": (_i32, [_p, _i32, _i64, _p, _p]),
     "bfasgd_fetch_message": (_i32, [_p, _i32, _p, _p]),
+    "fasgd_sim_quadratic_grad": (_i32, [_i64, _p, _p, _p, _p, _u64, _i32, _u64, _p, _p]),
+    "fasgd_sim_quadratic_loss": (_i32, [_i64, _p, _p, _p, _p, _p, _p]),
     "bfasgd_select_compact_noalloc": (_i32, [_i64, _p, _p, _f32, _f32, _u64, _i32, _u64,
                                              _p, _p, _p, _p]),
     "fasgd_last_error": (ctypes.c_char_p, [_p]),
@@ -100,6 +103,10 @@ def fasgd_destroy(h):
 
 def fasgd_set_hparams(h, gamma, beta, eps, c_push, eps_b, seed):
     return LIB.fasgd_set_hparams(h, gamma, beta, eps, c_push, eps_b, seed)
+
+
+def fasgd_set_exact(h, exact):
+    return LIB.fasgd_set_exact(h, exact)
 
 
 def fasgd_set_stream(h, stream):
@@ -156,6 +163,14 @@ def bfasgd_push_message(h, client, timestamp, grad, sent_dev):
 
 def bfasgd_fetch_message(h, client, theta_client, fetched_dev):
     return LIB.bfasgd_fetch_message(h, client, theta_client, fetched_dev)
+
+
+def fasgd_sim_quadratic_grad(P, theta, h, star, sigma, seed, client, n, grad, stream):
+    return LIB.fasgd_sim_quadratic_grad(P, theta, h, star, sigma, seed, client, n, grad, stream)
+
+
+def fasgd_sim_quadratic_loss(P, theta, h, star, scratch, loss, stream):
+    return LIB.fasgd_sim_quadratic_loss(P, theta, h, star, scratch, loss, stream)
 
 
 def fasgd_pull(h, params):
@@ -287,6 +302,9 @@ class Server:
     # -- calls ---------------------------------------------------------------
     def set_hparams(self, gamma, beta, eps, c_push, eps_b, seed):
         self._check(fasgd_set_hparams(self.h, gamma, beta, eps, c_push, eps_b, seed))
+
+    def set_exact(self, exact: bool):
+        self._check(fasgd_set_exact(self.h, 1 if exact else 0))
 
     def set_params(self, theta0):
         self._check(fasgd_set_params(self.h, _ptr(theta0)))

@@ -223,3 +223,41 @@ def client_v_snapshot(w: Workload, client: int, P: int | None = None,
     P = w.P if P is None else P
     u = _rng(w.seed, _TAG_VSNAP, client).uniform(math.log(lo), math.log(hi), P)
     return np.exp(u).astype(np.float32)
+
+
+_TAG_OBJ_H, _TAG_OBJ_STAR, _TAG_OBJ_SIGMA, _TAG_DISPATCH = 7, 8, 9, 10
+
+
+def quadratic_objective(seed: int, P: int, h_lo: float = 1e-2, h_hi: float = 10.0,
+                        sigma_lo: float = 1e-3, sigma_hi: float = 1e-1):
+    """A synthetic separable quadratic for the closed-loop simulation:
+    curvatures h_p log-uniform[h_lo, h_hi], minimiser star_p ~ N(0, 0.1^2),
+    gradient-noise scales sigma_p log-uniform[sigma_lo, sigma_hi] (fp32[P] each).
+    The spread of h makes a single learning rate a compromise across
+    parameters, as in a real network."""
+    h = np.exp(_rng(seed, _TAG_OBJ_H).uniform(math.log(h_lo), math.log(h_hi), P)).astype(np.float32)
+    star = (_rng(seed, _TAG_OBJ_STAR).standard_normal(P, dtype=np.float32) * np.float32(0.1))
+    sigma = np.exp(_rng(seed, _TAG_OBJ_SIGMA).uniform(math.log(sigma_lo), math.log(sigma_hi),
+                                                      P)).astype(np.float32)
+    return h, star, sigma
+
+
+def dispatch_schedule(seed: int, lam: int, n_batches: int, K: int = 1, rho: float = 1.0):
+    """Which clients push in each batch of K (distinct within a batch: a client
+    waits for the server's reply before it pushes again, Sec. 3).  Selection
+    weights start at 1; a selected client's weight is multiplied by rho and
+    every other weight by 1/rho, capped at 1 (rho = 1: uniform choice)."""
+    if K > lam:
+        raise ValueError("K clients per batch need lambda >= K")
+    g = _rng(seed, _TAG_DISPATCH)
+    w = np.ones(lam)
+    out = np.empty((n_batches, K), dtype=np.int32)
+    for b in range(n_batches):
+        pick = g.choice(lam, K, replace=False, p=w / w.sum())
+        out[b] = pick
+        if rho != 1.0:
+            mask = np.zeros(lam, bool)
+            mask[pick] = True
+            w[mask] *= rho
+            w[~mask] = np.minimum(1.0, w[~mask] / rho)
+    return out

@@ -63,6 +63,7 @@ class GpuRun:
         self.srv = f.Server(P, w.lam, w.alpha, variant, gamma=h["gamma"], beta=h["beta"],
                             eps=h["eps"], c_push=h.get("c_push", 0.0), eps_b=h["eps_b"],
                             seed=h.get("seed", 0))
+        self.srv.set_exact(bool(h.get("exact", False)))
         self.P = P
         self._pool_buf, self.pool = f.aligned_vectors(pool)
         self.srv.set_params(torch.from_numpy(theta0).cuda())
@@ -88,6 +89,7 @@ class OracleRun:
                                        gamma=h["gamma"], beta=h["beta"], eps=h["eps"],
                                        c_push=h.get("c_push", 0.0), eps_b=h["eps_b"],
                                        seed=h.get("seed", 0))
+        h.pop("exact", None)
         self.srv.set_params(theta0)
         self.pool = pool
 
@@ -100,11 +102,15 @@ class OracleRun:
         return list(self.srv.state())
 
 
-def compare_states(gs, os_, variant, where):
+def compare_states(gs, os_, variant, where, exact=False):
     names = ("theta", "n", "b", "v")
     assert gs[4] == os_[4], f"{where}: timestamps differ {gs[4]} vs {os_[4]}"
     if variant in (oracle.ASGD, oracle.SASGD):
         assert_bitwise(gs[0], os_[0].astype(np.float32), f"{where} theta")
+        return
+    if exact:   # exact arithmetic mode: every array bit for bit
+        for k in range(4):
+            assert_bitwise(gs[k], os_[k].astype(np.float32), f"{where} {names[k]}")
         return
     # n and b are formed with the same once-rounded fp32 sequence on both sides.
     assert_bitwise(gs[1], os_[1].astype(np.float32), f"{where} n")
@@ -128,7 +134,8 @@ def run_parity(w, variant, P, n_pushes, K, check_every=None, real="f32", **hp):
         o.push_batch(cl, js, sl)
         T = (b + 1) * K
         if T % check_every == 0:
-            compare_states(g.state(), o.state(), variant, f"{w.name} var={variant} P={P} K={K} T={T}")
+            compare_states(g.state(), o.state(), variant, f"{w.name} var={variant} P={P} K={K} T={T}",
+                           exact=bool(hp.get("exact", False)))
             checks += 1
     assert checks > 0
     return g, o

@@ -590,6 +590,48 @@ def check_message_path(libs: Libs):
     assert s.fetch_count == [0, 2]
 
 
+def check_sim_objective(libs: Libs):
+    """The closed-loop simulation's objective: the deterministic part of the
+    gradient is h (theta - star) in fp32, the noise is uniform with the stated
+    variance and range, fresh per (client, gradient count), and the loss is
+    1/2 sum h (theta - star)^2; a single client with full fetches reproduces
+    plain stochastic gradient descent step by step."""
+    import oracle.sim as osim
+    rng = np.random.default_rng(51)
+    P = 50_000
+    th = (rng.standard_normal(P) * 0.1).astype(np.float32)
+    h = (10 ** rng.uniform(-2, 1, P)).astype(np.float32)
+    star = (rng.standard_normal(P) * 0.1).astype(np.float32)
+    g = oracle.sim_grad(th, h, star, np.zeros(P, np.float32), 5, 1, 0, lib=libs.f32)
+    assert np.array_equal(g.view(np.uint32), (h * (th - star)).astype(np.float32).view(np.uint32))
+    sig = np.full(P, 0.25, np.float32)
+    noise = oracle.sim_grad(star, h, star, sig, 5, 1, 0, lib=libs.f32).astype(np.float64)
+    assert abs(noise.mean()) < 5 * 0.25 / math.sqrt(P)
+    assert abs(noise.var() - 0.0625) < 0.0625 * 0.03
+    assert np.max(np.abs(noise)) <= 0.25 * math.sqrt(3) * (1 + 1e-6)
+    other = oracle.sim_grad(star, h, star, sig, 5, 2, 0, lib=libs.f32)
+    again = oracle.sim_grad(star, h, star, sig, 5, 1, 0, lib=libs.f32)
+    later = oracle.sim_grad(star, h, star, sig, 5, 1, 1, lib=libs.f32)
+    assert np.array_equal(again, noise.astype(np.float32))
+    assert abs(np.corrcoef(noise, other)[0, 1]) < 0.02 and abs(np.corrcoef(noise, later)[0, 1]) < 0.02
+    terms = (h * ((th - star) * (th - star))).astype(np.float32).astype(np.float64)
+    want = 0.5 * math.fsum(terms)
+    assert abs(oracle.sim_loss(th, h, star, lib=libs.f32) - want) <= 1e-12 * want
+    # One client, full fetches: the simulation is plain SGD at the current point.
+    Ps = 301
+    obj = (h[:Ps], star[:Ps], (10 ** rng.uniform(-3, -1, Ps)).astype(np.float32))
+    th0 = np.zeros(Ps, np.float32)
+    sim = osim.OracleSimulation(Ps, 1, 0.05, ASGD, objective=obj, theta0=th0, seed=3,
+                                lib=libs.f32)
+    sim.run(np.zeros((40, 1), np.int32))
+    ref = th0.copy()
+    a32 = np.float32(0.05)
+    for t in range(40):
+        gt = oracle.sim_grad(ref, *obj, 3, 0, t, lib=libs.f32)
+        ref = (ref - a32 * gt).astype(np.float32)
+    assert np.array_equal(sim.srv.theta.view(np.uint32), ref.view(np.uint32))
+
+
 def check_protocol_errors(libs: Libs):
     s = _server(libs, "f32", 4, FASGD, lam=2)
     g = np.zeros(4, np.float32)
@@ -632,5 +674,6 @@ ALL_CHECKS = [
     check_fetch_path,
     check_server_fetch_counters,
     check_message_path,
+    check_sim_objective,
     check_protocol_errors,
 ]

@@ -192,3 +192,14 @@ def test_divide_by_std_full_stream_7850():
     its steps match FASGD's."""
     w = W["fasgd-7850"]
     run_parity(w.replace(alpha=w.alpha * 1e-3), oracle.FASGD_STD, w.P, w.pushes, 1)
+
+
+@pytest.mark.parametrize("variant", [oracle.FASGD, oracle.FASGD_STD])
+@pytest.mark.parametrize("K,eps", [(1, 1e-4), (8, 1e-4), (13, 1e-4), (8, 0.0)])
+def test_exact_mode_is_bitwise(variant, K, eps):
+    """fasgd_set_exact(1): theta, n, b and v equal the oracle's fp32 sequence bit for bit."""
+    w = W["fasgd-25m-k8"].replace(R=max(2 * K, 16))
+    if variant == oracle.FASGD_STD:
+        w = w.replace(alpha=w.alpha * 1e-3)
+    n = 100 * K // np.gcd(100, K)
+    run_parity(w, variant, 30_011, n, K, eps=eps, exact=True)

@@ -50,6 +50,9 @@ MUTANTS = {
     "message_draw_collides": ("uint32_t ctr[4] = {0xFFFFFFFFu,", "uint32_t ctr[4] = {0u,"),
     "message_draw_ignores_stream": ("{0xFFFFFFFFu, client | (stream << 31),", "{0xFFFFFFFFu, client,"),
     "std_variant_inverts": ("REAL r = ora_sqrt(var + eps);\n        *v = beta", "REAL r = 1 / ora_sqrt(var + eps);\n        *v = beta"),
+    "sim_noise_half_range": ("(1.0f / 8388608.0f) - 0.5f", "(1.0f / 16777216.0f) - 0.5f"),
+    "sim_grad_sign": ("float d = theta[p] - star[p];\n        g[p]", "float d = star[p] - theta[p];\n        g[p]"),
+    "sim_loss_no_half": ("return 0.5 * s;", "return s;"),
     "decide_not_strict": ("prod == A && err < 0.0f", "prod == A && err <= 0.0f"),
     "decide_ignores_err": ("if (prod == A && err < 0.0f)\n        return 1;\n", ""),
     "decide_drops_eps": ("float a = v + eps_b;", "float a = v;"),
