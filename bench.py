@@ -251,6 +251,7 @@ def run_dense(args, w, world, rank, local):
     pool_t, slots = fasgd.aligned_vectors(pool, device)
     stream = torch.cuda.current_stream()
     srv = fasgd.Server(P, w.lam, w.alpha, variant, stream=stream)
+    srv.set_exact(args.exact)
     srv.set_params(torch.from_numpy(th0).to(device))
     batches = [ps.batch(b) for b in range(n_batches)]
     batches = [([int(c) for c in cl], [int(j) for j in js], [int(s) for s in sl])
@@ -351,6 +352,8 @@ def run_dense(args, w, world, rank, local):
                    "K": K, "variant": "fasgd", "alpha": w.alpha, "staleness": w.delay,
                    "gradient_pool_slots": w.R, "pushes_timed": K * args.steps,
                    "parallelism": f"param-shard{world}",
+                   "arithmetic": "exact (IEEE sqrt/div, unfused)" if args.exact else
+                   "fast (hardware rsqrt/rcp, n and b exact)",
                    "l2": "inputs larger than L2 (%.2f GB per step vs 129 MB L2), no flush"
                    % (alg / 1e9) if alg > 4 * L2_BYTES else "working set may be L2-resident"},
     }
@@ -601,6 +604,8 @@ def main():
     ap.add_argument("--e2e-steps", type=int, default=40)
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--exact", action="store_true",
+                    help="dense workloads: time the exact-arithmetic FASGD update")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")

@@ -126,14 +126,16 @@ class Simulation:
         self.srv.close()
 
 
-def compare(P: int, lam: int, n_batches: int, K: int, alphas, seed: int = 0, log_every: int = 0):
+def compare(P: int, lam: int, n_batches: int, K: int, alphas, seed: int = 0, log_every: int = 0,
+            noise: str = "independent"):
     """Final loss of each update rule at each learning rate (same schedule,
     objective and start for all)."""
     sched = streams.dispatch_schedule(seed, lam, n_batches, K)
-    obj = streams.quadratic_objective(seed, P)
+    obj = streams.quadratic_objective(seed, P, noise=noise)
     th0 = np.zeros(P, np.float32)
     init = float(0.5 * np.sum(obj[0].astype(np.float64) * (th0 - obj[1]).astype(np.float64) ** 2))
-    out = {"P": P, "lambda": lam, "K": K, "batches": n_batches, "initial_loss": init, "runs": []}
+    out = {"P": P, "lambda": lam, "K": K, "batches": n_batches, "noise": noise,
+           "initial_loss": init, "runs": []}
     for name, var in (("asgd", fasgd.ASGD), ("sasgd", fasgd.SASGD), ("fasgd", fasgd.FASGD),
                       ("fasgd-std", fasgd.FASGD_STD)):
         for a in alphas[name]:
@@ -157,11 +159,12 @@ def main():
     ap.add_argument("--batches", type=int, default=2000)
     ap.add_argument("--K", type=int, default=1)
     ap.add_argument("--seed", type=int, default=0)
+    ap.add_argument("--noise", choices=["independent", "fisher"], default="independent")
     args = ap.parse_args()
-    grid = [10.0 ** e for e in np.arange(-4.0, 0.01, 0.5)]
+    grid = [10.0 ** e for e in np.arange(-5.0, 1.01, 0.5)]
     alphas = {"asgd": grid, "sasgd": grid, "fasgd": grid, "fasgd-std": [g * 1e-3 for g in grid]}
     res = compare(args.P, args.lam, args.batches, args.K, alphas, args.seed,
-                  log_every=max(1, args.batches // 20))
+                  log_every=max(1, args.batches // 20), noise=args.noise)
     best = {}
     for r in res["runs"]:
         if np.isfinite(r["final_loss"]) and (r["rule"] not in best or
@@ -169,7 +172,9 @@ def main():
             best[r["rule"]] = r
     res["best"] = {k: {"alpha": v["alpha"], "final_loss": v["final_loss"],
                        "curve": v["curve"]} for k, v in best.items()}
-    print(json.dumps(res if args.compare else res["best"]))
+    summary = {"P": res["P"], "lambda": res["lambda"], "K": res["K"], "noise": res["noise"],
+               "batches": res["batches"], "initial_loss": res["initial_loss"], "best": res["best"]}
+    print(json.dumps(res if args.compare else summary))
 
 
 if __name__ == "__main__":
