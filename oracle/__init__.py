@@ -88,6 +88,19 @@ def load_library(path: str, real: str) -> ctypes.CDLL:
     lib.ora_mean_v.argtypes = [i64, P]
     lib.ora_draw_message.restype = u32
     lib.ora_draw_message.argtypes = [u64, u32, u32, u64]
+    lib.ora_tensor_means.restype = None
+    lib.ora_tensor_means.argtypes = [i32, P, P, P]
+    lib.ora_budget_expected.restype = i64
+    lib.ora_budget_expected.argtypes = [i32, P, P, ctypes.c_float, ctypes.c_float]
+    lib.ora_budget_c.restype = ctypes.c_float
+    lib.ora_budget_c.argtypes = [i32, P, P, ctypes.c_float, i64]
+    lib.ora_draw_tensor.restype = u32
+    lib.ora_draw_tensor.argtypes = [u64, u32, u32, u64, i32]
+    lib.ora_tensor_select.restype = i64
+    lib.ora_tensor_select.argtypes = [i32, P, P, ctypes.c_float, ctypes.c_float, u64, u32, u32,
+                                      u64, P]
+    lib.ora_apply_tensors.restype = None
+    lib.ora_apply_tensors.argtypes = [i32, i32, P, P, P, P, P, P, P, R, R, R, R]
     lib.ora_sim_grad.restype = None
     lib.ora_sim_grad.argtypes = [i64, P, P, P, P, u64, u32, u64, P]
     lib.ora_sim_loss.restype = ctypes.c_double
@@ -188,6 +201,53 @@ def draw_message(seed: int, stream: int, client: int, n: int, lib=None) -> int:
     return int((lib or _load("f32")).ora_draw_message(seed, stream, client, n))
 
 
+def _sizes(sizes) -> np.ndarray:
+    s = np.ascontiguousarray(sizes, dtype=np.int64)
+    assert s.ndim == 1 and s.size >= 1 and (s >= 1).all()
+    return s
+
+
+def tensor_means(v: np.ndarray, sizes, real: str = "f32", lib=None) -> np.ndarray:
+    """vbar_t: mean of v over each contiguous tensor (fp64 sum, rounded to fp32)."""
+    s = _sizes(sizes)
+    vv = np.ascontiguousarray(v, dtype=_dtype(real))
+    assert vv.shape[0] == int(s.sum())
+    out = np.empty(s.size, dtype=np.float32)
+    (lib or _load(real)).ora_tensor_means(s.size, _ptr(s), _ptr(vv), _ptr(out))
+    return out
+
+
+def budget_expected(sizes, vbar, eps_b: float, x: float, lib=None) -> int:
+    """E(x) = sum_t floor(s_t fl(a_t / fl(a_t + x)) 2^32), a_t = fl(vbar_t + eps_b)."""
+    s = _sizes(sizes)
+    vb = np.ascontiguousarray(vbar, dtype=np.float32)
+    return int((lib or _load("f32")).ora_budget_expected(s.size, _ptr(s), _ptr(vb), eps_b, x))
+
+
+def budget_c(sizes, vbar, eps_b: float, budget: int, lib=None) -> float:
+    """Smallest threshold c (non-negative float or +inf) with E(c) <= min(B, P) 2^32."""
+    s = _sizes(sizes)
+    vb = np.ascontiguousarray(vbar, dtype=np.float32)
+    return float((lib or _load("f32")).ora_budget_c(s.size, _ptr(s), _ptr(vb), eps_b,
+                                                     int(budget)))
+
+
+def draw_tensor(seed: int, stream: int, client: int, n: int, t: int, lib=None) -> int:
+    """24-bit draw of tensor t for a client's n-th push (stream 0) or fetch (stream 1)."""
+    return int((lib or _load("f32")).ora_draw_tensor(seed, stream, client, n, t))
+
+
+def tensor_select(sizes, vbar, c: float, eps_b: float, seed: int, stream: int, client: int,
+                  n: int, lib=None):
+    """Per-tensor Eq. 9 decisions at threshold c: (sent uint8[T], parameters sent)."""
+    s = _sizes(sizes)
+    vb = np.ascontiguousarray(vbar, dtype=np.float32)
+    sent = np.zeros(s.size, dtype=np.uint8)
+    m = (lib or _load("f32")).ora_tensor_select(s.size, _ptr(s), _ptr(vb), c, eps_b, seed,
+                                                stream, client, n, _ptr(sent))
+    return sent, int(m)
+
+
 def sim_grad(theta, h, star, sigma, seed: int, client: int, n: int, lib=None) -> np.ndarray:
     """Stochastic gradient of the synthetic quadratic at theta (fp32[P])."""
     arrs = [np.ascontiguousarray(x, dtype=np.float32) for x in (theta, h, star, sigma)]
@@ -234,6 +294,8 @@ class OracleServer:
         self.c_fetch = 0.0
         self.cache: dict = {}          # client -> most recent sent gradient (message pushes)
         self.message_log: list = []    # decisions of applied message pushes, in order
+        self.sizes: np.ndarray | None = None   # tensor partition (per-tensor pushes)
+        self.budget_log: list = []     # (sent, c, parameters sent) of applied budget pushes
         self.set_hparams(gamma, beta, eps, c_push, eps_b, seed)
 
     def set_hparams(self, gamma, beta, eps, c_push, eps_b, seed):
@@ -270,6 +332,47 @@ class OracleServer:
             theta_client[:] = self.theta.astype(np.float32)
         return ok
 
+    def set_tensors(self, sizes):
+        """Partition the parameters into contiguous tensors (sizes sum to P)."""
+        s = _sizes(sizes)
+        if int(s.sum()) != self.P:
+            raise OracleError("tensor sizes must sum to P")
+        if self.fifo:
+            raise OracleError("pushes are pending")
+        self.sizes = s
+
+    def _budget_decide(self, stream: int, client: int, n: int, budget: int):
+        vbar = tensor_means(self.v, self.sizes, self.real)
+        c = budget_c(self.sizes, vbar, self.eps_b, budget)
+        sent, m = tensor_select(self.sizes, vbar, c, self.eps_b, self.seed, stream, client, n)
+        return sent, c, m
+
+    def push_budget(self, client: int, j: int, g: np.ndarray, budget: int):
+        """Per-tensor B-FASGD push under a budget of `budget` expected
+        parameters (decided when applied, against the server's v then)."""
+        if self.sizes is None:
+            raise OracleError("no tensor partition")
+        if budget < 0:
+            raise OracleError("budget must be >= 0")
+        self._check(client, j)
+        self.fifo.append(("budget", int(client), int(j),
+                          (np.asarray(g, dtype=np.float32), int(budget))))
+
+    def fetch_budget(self, client: int, theta_client: np.ndarray, budget: int):
+        """Per-tensor B-FASGD fetch under a budget: the transmitted tensors of
+        theta overwrite the client's copy.  Returns (sent, c, parameters sent)."""
+        if self.sizes is None:
+            raise OracleError("no tensor partition")
+        if not 0 <= client < self.lam or budget < 0:
+            raise OracleError("client or budget out of range")
+        n = self.fetch_count[client]
+        self.fetch_count[client] += 1
+        sent, c, m = self._budget_decide(1, client, n, budget)
+        off = np.concatenate([[0], np.cumsum(self.sizes)])
+        for t in np.flatnonzero(sent):
+            theta_client[off[t]:off[t + 1]] = self.theta[off[t]:off[t + 1]].astype(np.float32)
+        return sent, c, m
+
     def push_sparse(self, client: int, j: int, idx: np.ndarray, val: np.ndarray):
         self._check(client, j)
         self.fifo.append(("sparse", int(client), int(j),
@@ -300,7 +403,18 @@ class OracleServer:
                     self.cache[client] = payload.copy()
                 kind = "dense"
                 payload = self.cache.get(client, np.zeros(self.P, np.float32))
-            if kind == "dense":
+            if kind == "budget":
+                g, budget = payload
+                n = self.push_count[client]
+                self.push_count[client] += 1
+                sent, cb, m = self._budget_decide(0, client, n, budget)
+                self.budget_log.append((sent, cb, m))
+                g = np.ascontiguousarray(g, dtype=np.float32)
+                self.lib.ora_apply_tensors(self.variant, self.sizes.size, _ptr(self.sizes),
+                                           _ptr(sent), _ptr(self.theta), _ptr(self.n),
+                                           _ptr(self.b), _ptr(self.v), _ptr(g), c,
+                                           self.gamma, self.beta, self.eps)
+            elif kind == "dense":
                 g = np.ascontiguousarray(payload, dtype=np.float32)
                 self.lib.ora_apply_dense(self.variant, self.P, _ptr(self.theta), _ptr(self.n),
                                          _ptr(self.b), _ptr(self.v), _ptr(g), c,

@@ -30,6 +30,7 @@
  */
 #include <math.h>
 #include <stdint.h>
+#include <string.h>
 
 #ifndef REAL
 #define REAL float
@@ -333,4 +334,156 @@ double ora_sim_loss(int64_t P, const float *theta, const float *h, const float *
         s += (double)t;
     }
     return 0.5 * s;
+}
+
+/*
+ * Per-tensor B-FASGD under a bandwidth budget (Sec. 5, future work: decide
+ * per tensor rather than per message, and spread a fixed bandwidth budget
+ * over the tensors according to their statistics).  The paper gives no
+ * formula; the reading built here:
+ *
+ *   tensors    contiguous ranges [o_t, o_t + s_t) that partition [0, P),
+ *              o_0 = 0, o_{t+1} = o_t + s_t, s_t >= 1;
+ *   statistic  vbar_t = the mean of v over tensor t (fp64 sum in index
+ *              order, rounded once to fp32), as the per-message rule uses
+ *              the mean over all parameters;
+ *   decision   Eq. 9 per tensor: transmit tensor t iff
+ *              u_t / 2^24 < 1 / (1 + c / (vbar_t + eps_b))   (ora_decide);
+ *   budget     c is chosen so that the expected number of parameters
+ *              transmitted does not exceed the budget B:
+ *                  E(x) = sum_t floor(s_t * q_t(x) * 2^32),
+ *                  q_t(x) = fl(a_t / fl(a_t + x)),  a_t = fl(vbar_t + eps_b),
+ *              (q_t = 0 where a_t is not positive and finite), and
+ *                  c = the smallest x among the non-negative floats and +inf
+ *                      with E(x) <= min(B, P) * 2^32.
+ *              Every q_t is non-increasing in x (IEEE rounding is monotone),
+ *              so E is too and c is unique; E(+inf) = 0, so c exists.  The
+ *              terms are integers (fixed point, 2^-32 parameters), so the sum
+ *              is exact in any order.  A tensor with a larger vbar gets a
+ *              larger share: the expected share of tensor t is s_t a_t /
+ *              (a_t + c), the allocation "according to likelihood of
+ *              staleness" of the future-work section.
+ *   draws      u_t = word (t mod 4) of Philox4x32-10 at counter
+ *              (2^31 + t div 4, client + 2^31 * stream, n, n >> 32), top 24
+ *              bits, n = the client's count of earlier pushes (stream 0) or
+ *              fetches (stream 1); the first counter word never meets the
+ *              per-parameter draws (p div 4 < 2^29) or the per-message draw
+ *              (2^32 - 1) for t < 2^31 - 4.
+ *   unsent     a tensor that is not transmitted is not updated (the same
+ *              reading as the per-parameter path).
+ */
+
+/* vbar_t for every tensor: fp64 sum over the tensor in index order, rounded once. */
+void ora_tensor_means(int32_t T, const int64_t *sizes, const REAL *v, float *vbar)
+{
+    int64_t off = 0;
+    for (int32_t t = 0; t < T; t++) {
+        double s = 0.0;
+        for (int64_t p = off; p < off + sizes[t]; p++)
+            s += (double)v[p];
+        vbar[t] = (float)(s / (double)sizes[t]);
+        off += sizes[t];
+    }
+}
+
+/* floor(size * q * 2^32) for q = fl(a / fl(a + x)), exactly, in integers. */
+static int64_t ora_budget_term(int64_t size, float vbar, float eps_b, float x)
+{
+    float a = vbar + eps_b;
+    if (!(a > 0.0f) || isinf(a))
+        return 0;
+    float d = a + x;
+    float q = a / d;
+    if (q == 0.0f)
+        return 0;
+    int e;
+    float m = frexpf(q, &e);                   /* q = m 2^e, 1/2 <= m < 1 */
+    int64_t M = (int64_t)ldexpf(m, 24);        /* integer, exact: at most 24 bits */
+    int64_t prod = size * M;                   /* < 2^31 * 2^24 */
+    int shift = e - 24 + 32;                   /* size * q * 2^32 = prod * 2^shift */
+    if (shift >= 0)
+        return prod << shift;                  /* q <= 1, so at most size * 2^32 */
+    if (shift <= -63)
+        return 0;
+    return prod >> (-shift);
+}
+
+/* E(x): expected parameters sent at threshold x, in units of 2^-32. */
+int64_t ora_budget_expected(int32_t T, const int64_t *sizes, const float *vbar, float eps_b,
+                            float x)
+{
+    int64_t e = 0;
+    for (int32_t t = 0; t < T; t++)
+        e += ora_budget_term(sizes[t], vbar[t], eps_b, x);
+    return e;
+}
+
+static float ora_float_of_bits(uint32_t bits)
+{
+    float f;
+    memcpy(&f, &bits, sizeof f);
+    return f;
+}
+
+/* The budget threshold c (above): bisection over the bit patterns of the
+ * non-negative floats, which are ordered like the values they encode. */
+float ora_budget_c(int32_t T, const int64_t *sizes, const float *vbar, float eps_b,
+                   int64_t budget)
+{
+    int64_t S = 0;
+    for (int32_t t = 0; t < T; t++)
+        S += sizes[t];
+    int64_t B = budget < 0 ? 0 : (budget > S ? S : budget);
+    int64_t limit = B * ((int64_t)1 << 32);
+    if (ora_budget_expected(T, sizes, vbar, eps_b, 0.0f) <= limit)
+        return 0.0f;
+    uint32_t lo = 0, hi = 0x7F800000u;        /* E(lo) > limit >= E(hi) = E(+inf) */
+    while (hi - lo > 1) {
+        uint32_t mid = lo + (hi - lo) / 2;
+        if (ora_budget_expected(T, sizes, vbar, eps_b, ora_float_of_bits(mid)) <= limit)
+            hi = mid;
+        else
+            lo = mid;
+    }
+    return ora_float_of_bits(hi);
+}
+
+uint32_t ora_draw_tensor(uint64_t seed, uint32_t stream, uint32_t client, uint64_t n, int32_t t)
+{
+    uint32_t ctr[4] = {0x80000000u + ((uint32_t)t >> 2), client | (stream << 31), (uint32_t)n,
+                       (uint32_t)(n >> 32)};
+    uint32_t key[2] = {(uint32_t)seed, (uint32_t)(seed >> 32)};
+    uint32_t out[4];
+    ora_philox4x32_10(ctr, key, out);
+    return out[t & 3] >> 8;
+}
+
+/* The per-tensor decisions at threshold c; returns the parameters transmitted. */
+int64_t ora_tensor_select(int32_t T, const int64_t *sizes, const float *vbar, float c,
+                          float eps_b, uint64_t seed, uint32_t stream, uint32_t client,
+                          uint64_t n, uint8_t *sent)
+{
+    int64_t m = 0;
+    for (int32_t t = 0; t < T; t++) {
+        uint32_t u = ora_draw_tensor(seed, stream, client, n, t);
+        sent[t] = (uint8_t)ora_decide(u, vbar[t], c, eps_b);
+        if (sent[t])
+            m += sizes[t];
+    }
+    return m;
+}
+
+/* A per-tensor push: every parameter of a transmitted tensor receives g[p]. */
+void ora_apply_tensors(int variant, int32_t T, const int64_t *sizes, const uint8_t *sent,
+                       REAL *theta, REAL *n, REAL *b, REAL *v, const float *g, REAL coef,
+                       REAL gamma, REAL beta, REAL eps)
+{
+    int64_t off = 0;
+    for (int32_t t = 0; t < T; t++) {
+        if (sent[t])
+            for (int64_t p = off; p < off + sizes[t]; p++)
+                ora_update_one(variant, &theta[p], &n[p], &b[p], &v[p], (REAL)g[p], coef,
+                               gamma, beta, eps);
+        off += sizes[t];
+    }
 }

@@ -656,6 +656,219 @@ def check_protocol_errors(libs: Libs):
         pass
     else:
         raise AssertionError("descending sparse list accepted")
+    t = _server(libs, "f32", 4, FASGD, lam=2)
+    for bad in (lambda: t.push_budget(0, 0, g, 2),          # no partition yet
+                lambda: t.set_tensors([1, 2]),               # sizes do not sum to P
+                lambda: t.set_tensors([4, 0]),               # empty tensor
+                lambda: (t.set_tensors([1, 3]), t.push_budget(0, 0, g, -1))):
+        try:
+            bad()
+        except (oracle.OracleError, AssertionError):
+            pass
+        else:
+            raise AssertionError("bad per-tensor call accepted")
+
+
+# --------------------------------------------------------------------------
+# Per-tensor B-FASGD under a bandwidth budget (future-work section)
+# --------------------------------------------------------------------------
+def _budget_E(sizes, vbar, eps_b, x):
+    """E(x) from its definition, independently: numpy's IEEE fp32 add and
+    divide for q_t, then exact rationals for floor(s_t q_t 2^32)."""
+    tot = 0
+    with np.errstate(over="ignore", invalid="ignore", divide="ignore"):
+        for s, vb in zip(sizes, vbar):
+            a = np.float32(vb) + np.float32(eps_b)
+            if not (a > 0 and np.isfinite(a)):
+                continue
+            q = a / (a + np.float32(x))
+            tot += math.floor(Fraction(float(q)) * int(s) * 2 ** 32)
+    return tot
+
+
+def _f32_prev(x):
+    return float(np.array([np.float32(x).view(np.uint32) - 1], np.uint32).view(np.float32)[0])
+
+
+def _budget_instances(rng, n):
+    for k in range(n):
+        T = int(rng.integers(1, 13))
+        sizes = rng.integers(1, 5000, T)
+        sizes[rng.random(T) < 0.2] = 1
+        vbar = (10 ** rng.uniform(-3, 3, T)).astype(np.float32)
+        eps_b = (0.0, 1e-8, 0.5)[k % 3]
+        if eps_b == 0.0:
+            vbar[rng.random(T) < 0.2] = 0.0       # a_t = 0: never sent, no share
+        S = int(sizes.sum())
+        for B in (0, 1, S // 7, S // 2, S - 1, S, S + 10):
+            yield sizes, vbar, eps_b, max(B, 0)
+
+
+def check_tensor_means(libs: Libs):
+    """vbar_t is the exact mean of v over tensor t, rounded once to fp32."""
+    rng = np.random.default_rng(61)
+    for real in ("f32", "f64"):
+        sizes = np.array([1, 7, 1000, 4099, 2, 333])
+        v = (10 ** rng.uniform(-2, 3, int(sizes.sum()))).astype(np.float32)
+        got = oracle.tensor_means(v, sizes, real, lib=libs.lib(real))
+        off = np.concatenate([[0], np.cumsum(sizes)])
+        for t in range(sizes.size):
+            seg = v[off[t]:off[t + 1]].astype(np.float64)
+            exact = Fraction(math.fsum(seg)) / int(sizes[t])
+            assert got[t] == np.float32(float(exact)), (real, t)
+        assert got[0] == v[0]                          # one-element tensor: v itself
+        const = np.repeat(np.float32([0.3, 7.0, 1e-3]), [5, 11, 3])
+        assert np.array_equal(oracle.tensor_means(const, [5, 11, 3], real, lib=libs.lib(real)),
+                              np.float32([0.3, 7.0, 1e-3]))
+    # One tensor over everything: the per-message statistic.
+    v = (10 ** rng.uniform(-2, 3, 5000)).astype(np.float32)
+    assert oracle.tensor_means(v, [5000], lib=libs.f32)[0] == oracle.mean_v(v, lib=libs.f32)
+
+
+def check_budget_threshold(libs: Libs):
+    """c is the smallest non-negative float (or +inf) with E(c) <= B 2^32,
+    E defined exactly; equal statistics give the closed form a (S/B - 1)."""
+    rng = np.random.default_rng(62)
+    for sizes, vbar, eps_b, B in _budget_instances(rng, 24):
+        S = int(sizes.sum())
+        limit = min(B, S) * 2 ** 32
+        c = oracle.budget_c(sizes, vbar, eps_b, B, lib=libs.f32)
+        assert c >= 0.0
+        e_c = _budget_E(sizes, vbar, eps_b, c)
+        assert oracle.budget_expected(sizes, vbar, eps_b, c, lib=libs.f32) == e_c
+        assert e_c <= limit, (B, c)
+        if c > 0.0:
+            prev = _f32_prev(c)
+            e_prev = _budget_E(sizes, vbar, eps_b, prev)
+            assert oracle.budget_expected(sizes, vbar, eps_b, prev, lib=libs.f32) == e_prev
+            assert e_prev > limit, (B, c, prev)
+        for x in (0.0, 1e-3, 1.0, 123.5, 3e38, float("inf")):
+            assert oracle.budget_expected(sizes, vbar, eps_b, x, lib=libs.f32) == \
+                _budget_E(sizes, vbar, eps_b, x)
+        if B >= S and (vbar.astype(np.float64) + eps_b > 0).all():
+            assert c == 0.0
+    # Non-increasing in the budget.
+    sizes = np.array([100, 2000, 5, 40000])
+    vbar = np.float32([0.5, 3.0, 40.0, 0.01])
+    cs = [oracle.budget_c(sizes, vbar, 0.0, B, lib=libs.f32) for B in range(0, 42106, 1000)]
+    assert all(x >= y for x, y in zip(cs, cs[1:]))
+    # Equal statistics: sum_t s_t a / (a + c) = B  =>  c = a (S / B - 1).
+    for a, B in ((0.7, 2500), (13.0, 9000), (2e-3, 100)):
+        sizes = np.array([1000, 3000, 6000])
+        c = oracle.budget_c(sizes, np.float32([a] * 3), 0.0, B, lib=libs.f32)
+        want = float(np.float32(a)) * (10000 / B - 1)
+        assert abs(c - want) <= 2e-6 * want, (a, B, c, want)
+
+
+def check_tensor_decisions(libs: Libs):
+    """Tensor draws have their own Philox domain and layout; decisions are
+    Eq. 9 per tensor; over many pushes the parameters sent average E(c)."""
+    seed, client = 0xFEED_F00D_1234, 5
+    for stream in (0, 1):
+        for n in (0, 1, (2 << 32) + 9):
+            for t in (0, 1, 2, 3, 4, 4099):
+                block = oracle.philox4x32_10(
+                    [(1 << 31) + (t >> 2), client | (stream << 31), n & 0xFFFFFFFF, n >> 32],
+                    [seed & 0xFFFFFFFF, seed >> 32], lib=libs.f32)
+                assert oracle.draw_tensor(seed, stream, client, n, t, lib=libs.f32) == \
+                    block[t & 3] >> 8
+    same = sum(oracle.draw_tensor(seed, 0, 2, n, 0, lib=libs.f32) ==
+               oracle.draw_stream(seed, 0, 2, n, 0, lib=libs.f32) for n in range(300))
+    assert same < 3
+    sizes = np.array([10, 700, 3000, 1, 64, 20000, 5, 900])
+    vbar = np.float32([0.1, 4.0, 1.0, 50.0, 0.5, 2.0, 0.02, 9.0])
+    eps_b = 1e-8
+    S = int(sizes.sum())
+    B = S // 4
+    c = oracle.budget_c(sizes, vbar, eps_b, B, lib=libs.f32)
+    N = 3000
+    tot = []
+    for n in range(N):
+        sent, m = oracle.tensor_select(sizes, vbar, c, eps_b, seed, 0, client, n, lib=libs.f32)
+        assert m == int((sizes * sent).sum())
+        if n < 40:
+            for t in range(sizes.size):
+                u = oracle.draw_tensor(seed, 0, client, n, t, lib=libs.f32)
+                assert bool(sent[t]) == _exact_decide(u, vbar[t], c, eps_b)
+        tot.append(m)
+    q = np.array([float(np.float32(vb + np.float32(eps_b)) / np.float32(np.float32(vb + np.float32(eps_b)) + np.float32(c)))
+                  for vb in vbar])
+    mu = float((sizes * q).sum())
+    sd = math.sqrt(float((sizes.astype(np.float64) ** 2 * q * (1 - q)).sum()) / N)
+    assert abs(np.mean(tot) - mu) <= 5 * sd + S * 2.0 ** -24, (np.mean(tot), mu, sd)
+    assert abs(mu - B) <= 1.0
+    # c = 0 sends every tensor; c = +inf none.
+    assert oracle.tensor_select(sizes, vbar, 0.0, eps_b, seed, 0, 1, 0, lib=libs.f32)[1] == S
+    assert oracle.tensor_select(sizes, vbar, float("inf"), eps_b, seed, 0, 1, 0,
+                                lib=libs.f32)[1] == 0
+
+
+def check_budget_server(libs: Libs):
+    """Server path: a budget of P or more is plain FASGD; a zero budget
+    changes nothing but T; otherwise the run equals sparse pushes of exactly
+    the transmitted tensors, each decided against the v of that moment."""
+    rng = np.random.default_rng(63)
+    sizes = np.array([40, 3, 17, 1, 60, 9])
+    P, lam, seed = int(sizes.sum()), 3, 2024
+    off = np.concatenate([[0], np.cumsum(sizes)])
+    grads = [(rng.standard_normal(P) * 0.1).astype(np.float32) for _ in range(25)]
+    theta0 = (rng.standard_normal(P) * 0.01).astype(np.float32)
+
+    def run(budget, variant=FASGD):
+        s = _server(libs, "f32", P, variant, lam=lam, seed=seed, eps_b=1e-3)
+        s.set_params(theta0)
+        s.set_tensors(sizes)
+        for t, g in enumerate(grads):
+            s.push_budget(t % lam, s.T - min(t % 2, s.T), g, budget)
+            s.apply_pending(1)
+        return s
+
+    for variant in (FASGD, FASGD_STD, SASGD):
+        a = run(P + 5, variant)
+        assert all(log[0].all() and log[1] == 0.0 and log[2] == P for log in a.budget_log)
+        b = _server(libs, "f32", P, variant, lam=lam)
+        b.set_params(theta0)
+        for t, g in enumerate(grads):
+            b.push(t % lam, b.T - min(t % 2, b.T), g)
+            b.apply_pending(1)
+        for x, y in zip(a.state(), b.state()):
+            assert np.array_equal(np.asarray(x).view(np.uint32) if hasattr(x, "view") else x,
+                                  np.asarray(y).view(np.uint32) if hasattr(y, "view") else y)
+    a = run(0)
+    assert a.T == len(grads) and sum(int(log[0].sum()) for log in a.budget_log) == 0
+    assert np.array_equal(a.theta, theta0) and not a.v.any() and not a.n.any()
+    # Moderate budget, replayed as sparse pushes of the transmitted ranges.
+    a = run(P // 3)
+    ref = _server(libs, "f32", P, FASGD, lam=lam, seed=seed, eps_b=1e-3)
+    ref.set_params(theta0)
+    total = 0
+    for t, (g, (sent, c, m)) in enumerate(zip(grads, a.budget_log)):
+        vbar = oracle.tensor_means(ref.v, sizes, lib=libs.f32)
+        assert c == oracle.budget_c(sizes, vbar, 1e-3, P // 3, lib=libs.f32)
+        idx = np.concatenate([np.arange(off[k], off[k + 1]) for k in np.flatnonzero(sent)]
+                             + [np.zeros(0, np.int64)]).astype(np.int32)
+        assert m == idx.size
+        total += m
+        ref.push_sparse(t % lam, ref.T - min(t % 2, ref.T), idx, g[idx])
+        ref.apply_pending(1)
+    assert 0 < total < P * len(grads)
+    for x, y in zip(a.state()[:4], ref.state()[:4]):
+        assert np.array_equal(x.view(np.uint32), y.view(np.uint32))
+    assert a.push_count == [9, 8, 8]
+    # Fetches: a full budget copies theta, a zero budget copies nothing, and
+    # a partial one copies exactly the transmitted tensors.
+    copy = np.full(P, 5.0, np.float32)
+    assert a.fetch_budget(1, copy, 0)[2] == 0 and np.all(copy == 5.0)
+    sent, c, m = a.fetch_budget(1, copy, P // 2)
+    for k in range(sizes.size):
+        seg = copy[off[k]:off[k + 1]]
+        if sent[k]:
+            assert np.array_equal(seg, a.theta[off[k]:off[k + 1]])
+        else:
+            assert np.all(seg == 5.0)
+    assert m == int((sizes * sent).sum())
+    assert a.fetch_budget(1, copy, P)[2] == P and np.array_equal(copy, a.theta)
+    assert a.fetch_count == [0, 3, 0]
 
 
 ALL_CHECKS = [
@@ -675,5 +888,9 @@ ALL_CHECKS = [
     check_server_fetch_counters,
     check_message_path,
     check_sim_objective,
+    check_tensor_means,
+    check_budget_threshold,
+    check_tensor_decisions,
+    check_budget_server,
     check_protocol_errors,
 ]

@@ -60,6 +60,23 @@ MUTANTS = {
     "select_idx_off_by_one": ("idx[m] = (int32_t)p;", "idx[m] = (int32_t)(p + 1);"),
     "sparse_val_reversed": ("(REAL)val[i], coef,", "(REAL)val[count - 1 - i], coef,"),
     "sparse_no_order_check": ("if (i > 0 && idx[i] <= idx[i - 1])\n            return -1;\n", ""),
+    "tensor_mean_divisor": ("vbar[t] = (float)(s / (double)sizes[t]);",
+                            "vbar[t] = (float)(s / (double)(sizes[t] + 1));"),
+    "tensor_mean_no_offset": ("vbar[t] = (float)(s / (double)sizes[t]);\n        off += sizes[t];",
+                              "vbar[t] = (float)(s / (double)sizes[t]);"),
+    "budget_term_scale": ("int shift = e - 24 + 32;", "int shift = e - 24 + 31;"),
+    "budget_ignores_size": ("int64_t prod = size * M;", "int64_t prod = M;"),
+    "budget_drops_eps": ("float a = vbar + eps_b;\n    if (!(a > 0.0f)",
+                         "float a = vbar;\n    if (!(a > 0.0f)"),
+    "budget_returns_lo": ("    return ora_float_of_bits(hi);\n}", "    return ora_float_of_bits(lo);\n}"),
+    "budget_no_zero_shortcut": ("vbar, eps_b, 0.0f) <= limit)\n        return 0.0f;",
+                                "vbar, eps_b, 0.0f) < limit)\n        return 0.0f;"),
+    "tensor_draw_word": ("return out[t & 3] >> 8;", "return out[(t + 1) & 3] >> 8;"),
+    "tensor_draw_param_domain": ("0x80000000u + ((uint32_t)t >> 2)", "((uint32_t)t >> 2)"),
+    "tensor_select_counts_tensors": ("m += sizes[t];\n    }\n    return m;",
+                                     "m += 1;\n    }\n    return m;"),
+    "apply_tensors_offset": ("gamma, beta, eps);\n        off += sizes[t];",
+                             "gamma, beta, eps);\n        off += sent[t] ? sizes[t] : 0;"),
     "dense_skips_last": ("for (int64_t p = 0; p < P; p++)\n        ora_update_one",
                          "for (int64_t p = 0; p < P - 1; p++)\n        ora_update_one"),
 }
