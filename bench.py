@@ -592,6 +592,119 @@ def run_message(args, w, world, rank, local):
     }
 
 
+def run_tensor(args, w, world, rank, local):
+    """Per-tensor B-FASGD under a bandwidth budget, one exchange per step: a
+    budget push (tensor means of v, budget threshold, per-tensor decisions,
+    Eq. 4-8 over the transmitted tensors) and a budget fetch (the same
+    decision for the client, copy of the transmitted tensors of theta)."""
+    import torch
+    from paper_1601_04033_gb300 import fasgd
+
+    device = torch.device("cuda", local)
+    torch.cuda.set_device(device)
+    P = args.P or w.P
+    wr = shard_workload(w, rank)
+    R = min(w.R, 8)
+    pool = streams.gradient_pool(wr, P, R)
+    th0 = streams.theta0(wr, P)
+    sizes = streams.tensor_sizes(w.seed, P, w.tensors)
+    n_steps = args.warmup + args.steps + w.lam
+    ps = streams.push_stream(w.replace(R=R), n_steps, 1)
+    pool_t, slots = fasgd.aligned_vectors(pool, device)
+    stream = torch.cuda.current_stream()
+    srv = fasgd.Server(P, w.lam, w.alpha, streams.FASGD, stream=stream, seed=w.seed)
+    srv.set_params(torch.from_numpy(th0).to(device))
+    srv.set_tensors(sizes)
+    t = 0
+    for _ in range(w.lam):          # dense warm-up so that v is settled
+        cl, js, sl = ps.batch(t)
+        srv.push(int(cl[0]), int(js[0]), slots[int(sl[0])])
+        srv.apply_pending(1)
+        t += 1
+    push_budget = int(w.send_frac * P)
+    fetch_budget = int(FETCH_FRACTION * P)
+    client_theta = torch.empty((w.lam, (P + 3) // 4 * 4), device=device)
+    client_theta[:, :P].copy_(torch.from_numpy(th0).to(device))
+    sent = torch.zeros(args.steps, dtype=torch.int64, device=device)
+    fetched = torch.zeros(args.steps, dtype=torch.int64, device=device)
+    cvals = torch.zeros(args.steps, dtype=torch.float32, device=device)
+
+    def step(t, ev=None, i=None):
+        cl, js, sl = ps.batch(t)
+        c = int(cl[0])
+        if ev is not None:
+            ev[0].record(stream)
+        srv.push_budget(c, int(js[0]), slots[int(sl[0])], push_budget,
+                        c_dev=cvals[i:i + 1] if i is not None else None,
+                        count_dev=sent[i:i + 1] if i is not None else None)
+        srv.apply_pending(1)
+        if ev is not None:
+            ev[1].record(stream)
+        srv.fetch_budget(c, client_theta[c, :P], fetch_budget,
+                         count_dev=fetched[i:i + 1] if i is not None else None)
+        if ev is not None:
+            ev[2].record(stream)
+
+    for _ in range(args.warmup):
+        step(t)
+        t += 1
+    torch.cuda.synchronize()
+    clocks = ClockSampler(gpu_identifier(torch))
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    launches0 = srv.launches
+    barrier(world)
+    torch.cuda.synchronize()
+    clocks.start()
+    time.sleep(0.3)
+    start.record(stream)
+    for i in range(args.steps):
+        step(t, ev[i], i)
+        t += 1
+    end.record(stream)
+    torch.cuda.synchronize()
+    clock_info = clocks.stop()
+    barrier(world)
+    launches = srv.launches - launches0
+    total_ms = max_over_ranks(start.elapsed_time(end), world, device)
+    push_ms = sum(e[0].elapsed_time(e[1]) for e in ev) / args.steps
+    fetch_ms = sum(e[1].elapsed_time(e[2]) for e in ev) / args.steps
+    s_mean = float(sent.double().mean().item())
+    f_mean = float(fetched.double().mean().item())
+    c_med = float(cvals.median().item())
+    srv.sync()
+    srv.close()
+    step_s = total_ms / 1e3 / args.steps
+    peak, peak_kind = peaks()
+    # A push: the K = 1 update of every transmitted parameter (theta, n, b, v
+    # read and written, gradient read: 36 B); the tensor means come from item
+    # sums the previous apply kept current (8 B per item, no pass over v).
+    # A fetch: 8 B per fetched parameter.
+    push_bytes = 36.0 * s_mean
+    fetch_bytes = 8.0 * f_mean
+    achieved = push_bytes / (push_ms / 1e3) / 1e9
+    return {
+        "value": P * world / step_s, "ms_per_step": total_ms / args.steps,
+        "roofline": {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
+                     "frac": round(achieved / peak, 4), "peak_source": peak_kind,
+                     "kernel": "budget push (decision + ranged apply)",
+                     "bytes_per_launch": push_bytes, "launch_ms": round(push_ms, 5),
+                     "traffic": None, "fetch_ms": round(fetch_ms, 5),
+                     "fetch_gbs": round(fetch_bytes / (fetch_ms / 1e3) / 1e9, 1)},
+        "clocks": clock_info, "e2e": None, "gpu_launches": launches,
+        "pushes_per_s": world / step_s, "sent_fraction": round(s_mean / P, 4),
+        "fetched_fraction": round(f_mean / P, 4),
+        "sent_updates_per_s": s_mean * world / step_s,
+        "config": {"workload": w.name, "P_per_gpu": P, "P_total": P * world, "lambda": w.lam,
+                   "K": 1, "variant": "b-fasgd per tensor, bandwidth budget",
+                   "tensors": int(sizes.size), "push_budget": push_budget,
+                   "fetch_budget": fetch_budget, "c_push_median": c_med,
+                   "step": "budget push (decision + ranged apply) + budget fetch (decision + copy)",
+                   "staleness": w.delay, "parallelism": f"param-shard{world}",
+                   "l2": "inputs larger than L2, no flush"},
+    }
+
+
 # ---------------------------------------------------------------------------
 def main():
     ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
@@ -613,6 +726,8 @@ def main():
     w = streams.WORKLOADS[args.workload]
     if args.workload == "bfasgd-message-25m":
         mode = "message"
+    elif w.tensors:
+        mode = "tensor"
     elif w.send_frac is not None and args.workload == "bfasgd-25m":
         mode = "bfasgd"
     else:
@@ -643,6 +758,8 @@ def main():
         res = run_dense(args, w, world, rank, local)
     elif mode == "message":
         res = run_message(args, w, world, rank, local)
+    elif mode == "tensor":
+        res = run_tensor(args, w, world, rank, local)
     else:
         res = run_bfasgd(args, w, world, rank, local)
 

@@ -269,6 +269,69 @@ FASGD_API int bfasgd_fetch_message(fasgd_t* h, int32_t client, float* theta_clie
                                    int32_t* fetched_dev);
 
 /*
+ * Per-tensor B-FASGD under a bandwidth budget (Sec. 5, future work: decide
+ * per tensor, and spread a fixed bandwidth budget over the tensors by their
+ * statistics).  The paper gives no formula; the reading implemented:
+ *   vbar_t  = mean of the server's v over tensor t (exact sum, rounded once);
+ *   a_t     = fl(vbar_t + eps_b);
+ *   E(x)    = sum_t floor(s_t * fl(a_t / fl(a_t + x)) * 2^32)   (integers;
+ *             a term is 0 where a_t is not positive and finite);
+ *   c       = the smallest non-negative float x (or +inf) with
+ *             E(x) <= min(budget, P) * 2^32: the Eq. 9 threshold at which the
+ *             expected number of parameters transmitted meets the budget;
+ *   u_t     = top 24 bits of word (t mod 4) of Philox4x32-10 at counter
+ *             (2^31 + t div 4, client + 2^31 * stream, n, n >> 32), key = seed
+ *             (n: the client's push count for stream 0, fetch count for
+ *             stream 1, which then advances);
+ *   tensor t is transmitted iff u_t * fl(a_t + c) < a_t * 2^24 (Eq. 9,
+ *             exact).  A tensor that is not transmitted is left as it is.
+ * The expected count of transmitted parameters is E(c) 2^-32 (<= budget) up
+ * to P 2^-24 (the 24-bit draw).  vbar_t is summed in a fixed order with
+ * float-float pairs: it equals the correctly rounded mean unless that mean
+ * lies within about 1e-12 (relative) of a rounding boundary of fp32.
+ */
+#define BFASGD_TMAX 4096                      /* tensors in one partition */
+
+/*
+ * bfasgd_set_tensors -- partition the parameters into T contiguous tensors:
+ * tensor t covers [o_t, o_t + sizes[t]), o_0 = 0, o_{t+1} = o_t + sizes[t].
+ * sizes: host int64[T], each >= 1, summing to P; 1 <= T <= BFASGD_TMAX.
+ * Requires an empty queue; waits for the handle's stream; allocates small
+ * device tables (a few bytes per tensor and per 16,384 parameters).
+ * Errors: EINVAL, EAGAIN, ENOMEM, ECUDA.
+ */
+FASGD_API int bfasgd_set_tensors(fasgd_t* h, int32_t T, const int64_t* sizes);
+
+/*
+ * bfasgd_push_budget -- queue a per-tensor B-FASGD push: when it is applied
+ * (in arrival order, by fasgd_apply_pending, as its own pass) the server
+ * forms vbar_t from its v at that moment, solves for c from `budget`
+ * (expected parameters per push, >= 0; budget >= P sends every tensor),
+ * decides each tensor, and applies Eq. 4-8 (or Eq. 1-2) with the push's
+ * alpha(tau) to every parameter of the transmitted tensors, reading grad
+ * there only.  grad: device fp32[P], 16-byte aligned, borrowed until the
+ * apply completes.  Outputs written on the stream at the apply, each may be
+ * NULL: sent_dev (device uint8[T], 1 = transmitted), c_dev (device float),
+ * count_dev (device int64, parameters transmitted).
+ * Errors: EINVAL (no partition, bad pointer, budget < 0), ERANGE, EAGAIN.
+ */
+FASGD_API int bfasgd_push_budget(fasgd_t* h, int32_t client, int64_t timestamp,
+                                 const float* grad, int64_t budget, uint8_t* sent_dev,
+                                 float* c_dev, int64_t* count_dev);
+
+/*
+ * bfasgd_fetch_budget -- per-tensor B-FASGD fetch, taken on the stream
+ * against the current server state: the same rule with stream 1 and the
+ * client's fetch count; the transmitted tensors of theta are copied into
+ * theta_client (device fp32[P], 16-byte aligned), the rest of the client's
+ * copy is left as it is.  Outputs as for bfasgd_push_budget.
+ * Errors: EINVAL, ERANGE, ECUDA.
+ */
+FASGD_API int bfasgd_fetch_budget(fasgd_t* h, int32_t client, float* theta_client,
+                                  int64_t budget, uint8_t* sent_dev, float* c_dev,
+                                  int64_t* count_dev);
+
+/*
  * fasgd_pull -- copy theta (P fp32) into params (host or device) and return
  * the server timestamp T in *T (Sec. 2.1 protocol step 3: the parameters
  * handed back to a client).  The copy is ordered after earlier work on the

@@ -20,25 +20,13 @@
 
 #include "eq9.cuh"
 #include "kernels.cuh"
+#include "twosum.cuh"
 
 namespace fasgd {
 namespace {
 
 constexpr int kMsgThreads = 256;
 constexpr unsigned kFull = 0xffffffffu;
-
-// hi + lo += x, with the rounding error of the fp32 addition recovered
-// exactly (TwoSum: six operations, no branch, no contraction).  lo collects
-// the errors in fp32 and is itself rounded, which bounds the pair's error by
-// a few ulp of lo -- far below one ulp of the fp64 total.
-__device__ __forceinline__ void two_sum_acc(float& hi, float& lo, float x) {
-    const float t = __fadd_rn(hi, x);
-    const float xp = __fsub_rn(t, hi);
-    const float hp = __fsub_rn(t, xp);
-    const float err = __fadd_rn(__fsub_rn(hi, hp), __fsub_rn(x, xp));
-    lo = __fadd_rn(lo, err);
-    hi = t;
-}
 
 __device__ __forceinline__ double block_sum(double s, double* smem) {
 #pragma unroll

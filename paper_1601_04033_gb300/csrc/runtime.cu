@@ -24,6 +24,7 @@
 #include "eq9.cuh"
 #include "fasgd.h"
 #include "kernels.cuh"
+#include "tensors.cuh"
 
 namespace {
 
@@ -32,7 +33,7 @@ constexpr int32_t kMaxLambda = int32_t(1) << 20;
 
 thread_local std::string g_create_error;
 
-enum PushKind { kDense = 0, kSparse = 1, kMessage = 2 };
+enum PushKind { kDense = 0, kSparse = 1, kMessage = 2, kBudget = 3 };
 
 struct Push {
     int kind;              // PushKind
@@ -45,6 +46,10 @@ struct Push {
     int64_t n_max;
     int stage;             // staging slot of a host push, -1 otherwise
     int32_t* flag;         // message push: where to report the decision (may be null)
+    int64_t budget;        // budget push: expected parameters per push
+    uint8_t* sent_out;     // budget push: caller copies of the decisions (each may be null)
+    float* c_out;
+    int64_t* count_out;
 };
 
 bool aligned(const void* p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) & (a - 1)) == 0; }
@@ -131,6 +136,89 @@ struct fasgd_s {
     int64_t cache_stride = 0;
     double* msg_partial = nullptr;
 
+    // Per-tensor B-FASGD: the partition, its work items on the device, the
+    // item sums of v and the decision of the latest call.
+    std::vector<int64_t> tensor_sizes;
+    fasgd::TensorItem* t_items = nullptr;
+    int32_t t_nitems = 0;
+    int32_t* t_item_begin = nullptr;
+    int32_t* t_sizes = nullptr;
+    float2* t_partial = nullptr;
+    uint8_t* t_sent = nullptr;
+    float* t_c = nullptr;
+    int64_t* t_count = nullptr;
+    bool t_sums_valid = false;   // t_partial holds the item sums of the current v
+
+    void free_tensors() {
+        cudaFree(t_items);
+        cudaFree(t_item_begin);
+        cudaFree(t_sizes);
+        cudaFree(t_partial);
+        cudaFree(t_sent);
+        cudaFree(t_c);
+        cudaFree(t_count);
+        t_items = nullptr;
+        t_item_begin = nullptr;
+        t_sizes = nullptr;
+        t_partial = nullptr;
+        t_sent = nullptr;
+        t_c = nullptr;
+        t_count = nullptr;
+        t_nitems = 0;
+        t_sums_valid = false;
+        tensor_sizes.clear();
+    }
+
+    // One per-tensor decision of `stream_id` for `client` under `budget`
+    // (advancing the client's counter); the decisions land in t_sent.
+    cudaError_t launch_budget(uint32_t stream_id, int32_t client, int64_t budget,
+                              uint8_t* sent_out, float* c_out, int64_t* count_out,
+                              std::vector<uint64_t>& counter) {
+        fasgd::TensorArgs a;
+        std::memset(&a, 0, sizeof a);
+        a.v = v;
+        a.items = t_items;
+        a.n_items = t_nitems;
+        a.item_begin = t_item_begin;
+        a.sizes = t_sizes;
+        a.T = (int32_t)tensor_sizes.size();
+        a.partial = t_partial;
+        a.eps_b = eps_b;
+        const int64_t B = budget < P ? budget : P;
+        a.limit = B * (int64_t(1) << 32);
+        fasgd::philox_key_schedule(seed, a.round_key0, a.round_key1);
+        const uint64_t n = counter[(size_t)client];
+        a.client_word = (uint32_t)client | (stream_id << 31);
+        a.n_lo = (uint32_t)n;
+        a.n_hi = (uint32_t)(n >> 32);
+        a.sent = t_sent;
+        a.c_out = t_c;
+        a.count_out = t_count;
+        a.user_sent = sent_out;
+        a.user_c = c_out;
+        a.user_count = count_out;
+        cudaError_t st = fasgd::launch_tensor_decide(a, t_sums_valid, stream, &launches);
+        if (st == cudaSuccess) {
+            t_sums_valid = true;
+            counter[(size_t)client] = n + 1;
+        }
+        return st;
+    }
+    fasgd::RangeArgs range_args() const {
+        fasgd::RangeArgs r;
+        std::memset(&r, 0, sizeof r);
+        r.theta = theta;
+        r.n = n;
+        r.b = b;
+        r.v = v;
+        r.sp = stat_params();
+        r.items = t_items;
+        r.n_items = t_nitems;
+        r.sent = t_sent;
+        r.partial = t_partial;
+        return r;
+    }
+
     cudaError_t ensure_message_scratch(bool cache) {
         cudaError_t st = cudaSuccess;
         if (msg_partial == nullptr)
@@ -213,6 +301,7 @@ struct fasgd_s {
         cudaFree(msg_partial);
         grad_cache = nullptr;
         msg_partial = nullptr;
+        free_tensors();
         for (float* s : stage) cudaFree(s);
         for (cudaEvent_t e : slot_ready) cudaEventDestroy(e);
         for (cudaEvent_t e : slot_free) cudaEventDestroy(e);
@@ -454,6 +543,100 @@ int bfasgd_fetch_message(fasgd_t* h, int32_t client, float* theta_client, int32_
     return FASGD_OK;
 }
 
+int bfasgd_set_tensors(fasgd_t* h, int32_t T, const int64_t* sizes) {
+    if (h == nullptr) return FASGD_EINVAL;
+    if (T < 1 || T > BFASGD_TMAX || sizes == nullptr)
+        return h->fail(FASGD_EINVAL, "T must be in [1, %d] and sizes non-NULL", BFASGD_TMAX);
+    int64_t total = 0;
+    for (int32_t t = 0; t < T; ++t) {
+        if (sizes[t] < 1 || sizes[t] > h->P)
+            return h->fail(FASGD_EINVAL, "tensor %d has size %lld", t, (long long)sizes[t]);
+        total += sizes[t];
+        if (total > h->P) break;
+    }
+    if (total != h->P) return h->fail(FASGD_EINVAL, "tensor sizes do not sum to P");
+    if (!h->fifo.empty()) return h->fail(FASGD_EAGAIN, "pushes are pending");
+    DeviceGuard g(h->device);
+    // Work items: each tensor cut into pieces of at most `chunk` parameters.
+    const int64_t chunk = fasgd::tensor_chunk(h->P);
+    std::vector<fasgd::TensorItem> items;
+    std::vector<int32_t> begin((size_t)T + 1), sz((size_t)T);
+    int64_t off = 0;
+    for (int32_t t = 0; t < T; ++t) {
+        begin[(size_t)t] = (int32_t)items.size();
+        sz[(size_t)t] = (int32_t)sizes[t];
+        for (int64_t s = 0; s < sizes[t]; s += chunk) {
+            const int64_t len = sizes[t] - s < chunk ? sizes[t] - s : chunk;
+            items.push_back(fasgd::TensorItem{off + s, (int32_t)len, t});
+        }
+        off += sizes[t];
+    }
+    begin[(size_t)T] = (int32_t)items.size();
+    cudaError_t st = cudaStreamSynchronize(h->stream);   // no decision still reads the old tables
+    h->free_tensors();
+    const size_t ni = items.size();
+    if (st == cudaSuccess) st = cudaMalloc(reinterpret_cast<void**>(&h->t_items), ni * sizeof(fasgd::TensorItem));
+    if (st == cudaSuccess) st = cudaMalloc(reinterpret_cast<void**>(&h->t_item_begin), begin.size() * sizeof(int32_t));
+    if (st == cudaSuccess) st = cudaMalloc(reinterpret_cast<void**>(&h->t_sizes), sz.size() * sizeof(int32_t));
+    if (st == cudaSuccess) st = cudaMalloc(reinterpret_cast<void**>(&h->t_partial), ni * sizeof(float2));
+    if (st == cudaSuccess) st = cudaMalloc(reinterpret_cast<void**>(&h->t_sent), (size_t)T);
+    if (st == cudaSuccess) st = cudaMalloc(reinterpret_cast<void**>(&h->t_c), sizeof(float));
+    if (st == cudaSuccess) st = cudaMalloc(reinterpret_cast<void**>(&h->t_count), sizeof(int64_t));
+    if (st == cudaSuccess)
+        st = cudaMemcpy(h->t_items, items.data(), ni * sizeof(fasgd::TensorItem), cudaMemcpyHostToDevice);
+    if (st == cudaSuccess)
+        st = cudaMemcpy(h->t_item_begin, begin.data(), begin.size() * sizeof(int32_t), cudaMemcpyHostToDevice);
+    if (st == cudaSuccess)
+        st = cudaMemcpy(h->t_sizes, sz.data(), sz.size() * sizeof(int32_t), cudaMemcpyHostToDevice);
+    if (st != cudaSuccess) {
+        h->free_tensors();
+        return h->cuda_fail(st, "bfasgd_set_tensors");
+    }
+    h->t_nitems = (int32_t)ni;
+    h->tensor_sizes.assign(sizes, sizes + T);
+    return FASGD_OK;
+}
+
+int bfasgd_push_budget(fasgd_t* h, int32_t client, int64_t timestamp, const float* grad,
+                       int64_t budget, uint8_t* sent_dev, float* c_dev, int64_t* count_dev) {
+    if (h == nullptr) return FASGD_EINVAL;
+    if (h->tensor_sizes.empty()) return h->fail(FASGD_EINVAL, "no tensor partition (bfasgd_set_tensors)");
+    if (grad == nullptr || !aligned(grad, 16))
+        return h->fail(FASGD_EINVAL, "grad must be a non-NULL 16-byte aligned device pointer");
+    if (budget < 0) return h->fail(FASGD_EINVAL, "budget must be >= 0");
+    if (!aligned(c_dev, 4) || !aligned(count_dev, 8))
+        return h->fail(FASGD_EINVAL, "c_dev must be 4-byte and count_dev 8-byte aligned");
+    int rc = check_push(h, client, timestamp);
+    if (rc != FASGD_OK) return rc;
+    Push p{kBudget, client, timestamp, grad, nullptr, nullptr, nullptr, 0, -1, nullptr,
+           budget, sent_dev, c_dev, count_dev};
+    h->fifo.push_back(p);
+    return FASGD_OK;
+}
+
+int bfasgd_fetch_budget(fasgd_t* h, int32_t client, float* theta_client, int64_t budget,
+                        uint8_t* sent_dev, float* c_dev, int64_t* count_dev) {
+    if (h == nullptr) return FASGD_EINVAL;
+    if (h->tensor_sizes.empty()) return h->fail(FASGD_EINVAL, "no tensor partition (bfasgd_set_tensors)");
+    if (client < 0 || client >= h->lambda)
+        return h->fail(FASGD_ERANGE, "client %d outside [0, %d)", client, h->lambda);
+    if (theta_client == nullptr || !aligned(theta_client, 16))
+        return h->fail(FASGD_EINVAL, "theta_client must be a non-NULL 16-byte aligned device pointer");
+    if (budget < 0) return h->fail(FASGD_EINVAL, "budget must be >= 0");
+    if (!aligned(c_dev, 4) || !aligned(count_dev, 8))
+        return h->fail(FASGD_EINVAL, "c_dev must be 4-byte and count_dev 8-byte aligned");
+    DeviceGuard g(h->device);
+    cudaError_t st = h->launch_budget(1, client, budget, sent_dev, c_dev, count_dev, h->fetch_count);
+    if (st == cudaSuccess) {
+        fasgd::RangeArgs r = h->range_args();
+        r.src = h->theta;
+        r.dst = theta_client;
+        st = fasgd::launch_tensor_copy(r, h->stream, &h->launches);
+    }
+    if (st != cudaSuccess) return h->cuda_fail(st, "bfasgd_fetch_budget");
+    return FASGD_OK;
+}
+
 int fasgd_push_sparse(fasgd_t* h, int32_t client, int64_t timestamp, const int32_t* idx,
                       const float* val, const int64_t* n_dev, int64_t n_max) {
     if (h == nullptr) return FASGD_EINVAL;
@@ -481,6 +664,7 @@ int fasgd_apply_pending(fasgd_t* h, int32_t K) {
     int k = 0;
     while (k < K) {
         const Push& first = h->fifo[(size_t)k];
+        if (first.kind != kBudget) h->t_sums_valid = false;   // this pass rewrites v
         if (first.kind == kDense) {
             // Fuse the run of consecutive dense pushes into one pass.
             fasgd::DenseArgs a;
@@ -537,6 +721,19 @@ int fasgd_apply_pending(fasgd_t* h, int32_t K) {
                 st = fasgd::launch_dense(a, rule, h->exact, h->num_sms, h->stream, &h->launches);
             }
             if (st != cudaSuccess) return h->cuda_fail(st, "fasgd_apply_pending: message push");
+            k += 1;
+        } else if (first.kind == kBudget) {
+            // Decide every tensor against the statistics now, then update the
+            // transmitted ones.
+            cudaError_t st = h->launch_budget(0, first.client, first.budget, first.sent_out,
+                                              first.c_out, first.count_out, h->push_count);
+            if (st == cudaSuccess) {
+                fasgd::RangeArgs r = h->range_args();
+                r.grad = first.grad;
+                r.coef = h->coef(h->T + k - first.j);
+                st = fasgd::launch_tensor_apply(r, rule, h->exact, h->stream, &h->launches);
+            }
+            if (st != cudaSuccess) return h->cuda_fail(st, "fasgd_apply_pending: budget push");
             k += 1;
         } else {
             fasgd::SparseArgs a;
@@ -779,6 +976,7 @@ int fasgd_set_state(fasgd_t* h, const float* theta, const float* n, const float*
         if (st != cudaSuccess) return h->cuda_fail(st, "fasgd_set_state");
     }
     h->T = T;
+    if (v != nullptr) h->t_sums_valid = false;
     return FASGD_OK;
 }
 

@@ -1,0 +1,417 @@
+// Per-tensor B-FASGD under a bandwidth budget (the paper's future-work
+// section: decide per tensor, and spread a fixed bandwidth budget over the
+// tensors according to their statistics).
+//
+// One decision takes one or two kernels:
+//   1. tensor_partial (only when the item sums are stale): one block per
+//      work item (a piece of one tensor of at most tensor_chunk(P)
+//      parameters) sums v over the item -- per thread an fp32 sum with its
+//      exact rounding errors (TwoSum), then a fixed float-float tree -- into
+//      one float-float pair per item;
+//   2. budget_resolve (one block of 1024 threads): vbar_t = fl32(sum of the
+//      item sums of tensor t / s_t), the budget threshold c, then the Philox
+//      draw and the exact Eq. 9 decision of every tensor and the number of
+//      parameters transmitted.
+// Then tensor_apply (a push: Eq. 4-8, or Eq. 1-2, on the transmitted
+// tensors) or tensor_copy (a fetch: theta into the client's copy) walks the
+// items of the transmitted tensors; the others cost one flag read.  The
+// apply re-forms the sums of the items it rewrote, in the partial kernel's
+// element order, so the item sums stay those of the current v and the next
+// decision skips the partial kernel (the host tracks when another pass has
+// changed v and the sums must be formed afresh).
+//
+// The threshold.  With a_t = fl(vbar_t + eps_b) and
+//   E(x) = sum_t floor(s_t * fl(a_t / fl(a_t + x)) * 2^32),
+// c is the smallest non-negative float x (or +inf) with E(x) <= limit.
+// Every term is an integer and non-increasing in x (IEEE rounding is
+// monotone), so E is exact in any summation order and the search has one
+// answer.  The block searches the bit patterns of the non-negative floats
+// (ordered as their values): each round evaluates E at 2^m - 1 points of
+// the current interval, one group of warps per point (lanes over tensors,
+// then an exact integer sum), and keeps the part between the last failing
+// and the first passing point.
+
+#include "eq9.cuh"
+#include "kernels.cuh"
+#include "tensors.cuh"
+#include "twosum.cuh"
+#include "update.cuh"
+
+namespace fasgd {
+namespace {
+
+constexpr int kItemThreads = 256;
+constexpr unsigned kFull = 0xffffffffu;
+
+// The sum of v over one item as a float-float pair, the same bits wherever
+// it is formed (the partial kernel, or the apply kernel after it rewrote the
+// item): thread tid adds, in this order and with TwoSum, the head element
+// s + tid (before the first whole 16-byte quad), the tail element 4 qe + tid
+// (after the last), then quads qs + tid, qs + tid + 256, ...; the threads'
+// pairs go through a fixed float-float tree.  Four quads are loaded before
+// they are added, so a thread keeps four loads in flight.  Called by every
+// thread of the block; the result is valid in thread 0.
+__device__ float2 item_v_sum(const TensorItem& it, const float* __restrict__ v, float2* smem) {
+    const int tid = threadIdx.x;
+    const int64_t s = it.start, e = s + it.len;
+    const int64_t qs = (s + 3) >> 2, qe = e >> 2;   // whole quads inside [s, e)
+    float hi = 0.f, lo = 0.f;
+    if (4 * qs >= e) {
+        for (int64_t p = s + tid; p < e; p += kItemThreads) two_sum_acc(hi, lo, v[p]);
+    } else {
+        if (tid < 4 * qs - s) two_sum_acc(hi, lo, v[s + tid]);
+        if (tid < e - 4 * qe) two_sum_acc(hi, lo, v[4 * qe + tid]);
+        const float4* v4 = reinterpret_cast<const float4*>(v);
+        for (int64_t q = qs + tid; q < qe; q += 4 * kItemThreads) {
+            float4 x[4];
+#pragma unroll
+            for (int k = 0; k < 4; ++k)
+                if (q + k * kItemThreads < qe) x[k] = v4[q + k * kItemThreads];
+#pragma unroll
+            for (int k = 0; k < 4; ++k)
+                if (q + k * kItemThreads < qe) {
+                    two_sum_acc(hi, lo, x[k].x);
+                    two_sum_acc(hi, lo, x[k].y);
+                    two_sum_acc(hi, lo, x[k].z);
+                    two_sum_acc(hi, lo, x[k].w);
+                }
+        }
+    }
+    float h, l;
+    two_sum(hi, lo, h, l);
+    ff_warp_sum(h, l);
+    if ((tid & 31) == 0) smem[tid >> 5] = make_float2(h, l);
+    __syncthreads();
+    float2 sum = make_float2(0.f, 0.f);
+    if (tid == 0)
+        for (int w = 0; w < kItemThreads / 32; ++w) ff_add(sum.x, sum.y, smem[w].x, smem[w].y);
+    __syncthreads();
+    return sum;
+}
+
+__global__ void __launch_bounds__(kItemThreads) tensor_partial_kernel(const __grid_constant__ TensorArgs a) {
+    __shared__ float2 smem[kItemThreads / 32];
+    for (int64_t i = blockIdx.x; i < a.n_items; i += gridDim.x) {
+        const float2 sum = item_v_sum(a.items[i], a.v, smem);
+        if (threadIdx.x == 0) a.partial[i] = sum;
+    }
+}
+
+// floor(size * q * 2^32) for q = fl(a / fl(a + x)), a = fl(vbar + eps_b),
+// exactly: q = M 2^e with M its 24-bit significand, so the term is
+// size * M shifted by e + 32 (q <= 1 keeps it at most size * 2^32).
+__device__ __forceinline__ uint64_t budget_term(int32_t size, float vbar, float eps_b, float x) {
+    const float a = __fadd_rn(vbar, eps_b);
+    if (!(a > 0.f) || a == __int_as_float(0x7f800000)) return 0;
+    const float q = __fdiv_rn(a, __fadd_rn(a, x));
+    const uint32_t bits = __float_as_uint(q);     // q in [0, 1]: sign bit clear
+    if (bits == 0) return 0;
+    const uint32_t ex = bits >> 23;
+    const uint64_t M = ex ? ((bits & 0x7fffffu) | 0x800000u) : (bits & 0x7fffffu);
+    const int shift = (ex ? (int)ex : 1) - 150 + 32;
+    const uint64_t prod = (uint64_t)(uint32_t)size * M;
+    if (shift >= 0) return prod << shift;
+    return shift > -64 ? prod >> (-shift) : 0;
+}
+
+// Candidate k (0 .. 2^m - 2) of a search round inside the open interval
+// (lo, hi) of bit patterns: 2^m - 1 points cutting it into 2^m near-equal
+// parts (consecutive patterns once the interval is short); values >= hi are
+// not evaluated.
+__device__ __forceinline__ long long candidate(long long lo, long long hi, int k, int m) {
+    const long long span = hi - lo;
+    return span <= (1ll << m) ? lo + 1 + k : lo + ((span * (k + 1)) >> m);
+}
+
+__global__ void __launch_bounds__(kTensorResolveThreads) budget_resolve_kernel(const __grid_constant__ TensorArgs a) {
+    // Dynamic shared memory (tensor_resolve_smem): the item sums, the
+    // per-tensor sums (whose high word then holds vbar_t), the item ranges
+    // and the sizes.  Everything the block reads more than once is loaded
+    // once, with all loads in flight together.
+    extern __shared__ __align__(16) unsigned char dsm[];
+    float2* s_part = reinterpret_cast<float2*>(dsm);
+    float2* s_tsum = s_part + a.n_items;
+    int32_t* s_begin = reinterpret_cast<int32_t*>(s_tsum + a.T);
+    int32_t* s_size = s_begin + a.T + 1;
+    __shared__ unsigned long long s_pw[2][32];
+    __shared__ unsigned long long s_count;
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    for (int i = tid; i < a.n_items; i += kTensorResolveThreads) s_part[i] = a.partial[i];
+    for (int t = tid; t <= a.T; t += kTensorResolveThreads) s_begin[t] = a.item_begin[t];
+    for (int t = tid; t < a.T; t += kTensorResolveThreads) s_size[t] = a.sizes[t];
+    if (tid == 0) s_count = 0;
+    __syncthreads();
+    // Sum of the item sums of tensor t: warp (t mod 32), lanes over the
+    // items, then a fixed shuffle tree, all in float-float.
+    for (int t = warp; t < a.T; t += 32) {
+        float h = 0.f, l = 0.f;
+        for (int i = s_begin[t] + lane; i < s_begin[t + 1]; i += 32)
+            ff_add(h, l, s_part[i].x, s_part[i].y);
+        ff_warp_sum(h, l);
+        if (lane == 0) s_tsum[t] = make_float2(h, l);
+    }
+    __syncthreads();
+    // vbar_t = fl32(sum / s_t): the pair widened to fp64 once, one fp64
+    // division per tensor, all tensors at once.
+    for (int t = tid; t < a.T; t += kTensorResolveThreads) {
+        const float2 p = s_tsum[t];
+        s_tsum[t].x = (float)(((double)p.x + (double)p.y) / (double)s_size[t]);
+    }
+    __syncthreads();
+    // Invariant: E(lo) > limit >= E(hi) (lo = -1 stands below 0, hi = +inf
+    // has E = 0); c = hi once they are adjacent.  2^m is chosen so that a
+    // thread takes about two tensors per candidate: the work of a round
+    // grows with the number of candidates times T, the number of rounds only
+    // with its log.  One barrier per round: every warp re-derives the new
+    // interval from the same partial sums (double-buffered).
+    int m = 5;
+    while (m > 1 && (a.T << m) > 2 * kTensorResolveThreads) --m;
+    const int gwarps = 32 >> m;                      // warps per group; the last group idles
+    const int group = warp / gwarps;
+    const int gthread = tid - group * gwarps * 32;
+    const int gsize = gwarps * 32;
+    const int ncand = (1 << m) - 1;
+    long long lo = -1, hi = 0x7f800000;
+    for (int round = 0; round < 64 && hi - lo > 1; ++round) {
+        const int buf = round & 1;
+        unsigned long long e = 0;
+        if (group < ncand) {
+            const long long cand = candidate(lo, hi, group, m);
+            if (cand < hi) {
+                const float x = __uint_as_float((uint32_t)cand);
+                for (int t = gthread; t < a.T; t += gsize)
+                    e += budget_term(s_size[t], s_tsum[t].x, a.eps_b, x);
+            }
+        }
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) e += __shfl_xor_sync(kFull, e, off);
+        if (lane == 0) s_pw[buf][warp] = e;
+        __syncthreads();
+        // Lane k adds the partials of group k and tests candidate k; E is
+        // non-increasing, so the passing candidates are a suffix.
+        int ok = 1;
+        long long cand = hi;
+        if (lane < ncand) {
+            cand = candidate(lo, hi, lane, m);
+            if (cand < hi) {
+                unsigned long long sum = 0;
+                for (int w = 0; w < gwarps; ++w) sum += s_pw[buf][lane * gwarps + w];
+                ok = (long long)sum <= a.limit;
+            } else {
+                cand = hi;
+            }
+        }
+        const unsigned pass = __ballot_sync(kFull, ok);   // lanes >= ncand pass
+        const int first = __ffs(pass) - 1;
+        const long long c_first = __shfl_sync(kFull, cand, first);
+        const long long c_prev = __shfl_sync(kFull, cand, first > 0 ? first - 1 : 0);
+        if (first > 0) lo = c_prev;
+        hi = c_first;
+    }
+    const float c = __uint_as_float((uint32_t)hi);
+    for (int t = tid; t < a.T; t += kTensorResolveThreads) {
+        const Philox4 r = philox4x32_10(0x80000000u + ((uint32_t)t >> 2), a.client_word, a.n_lo,
+                                        a.n_hi, a.round_key0, a.round_key1);
+        const uint32_t u = (t & 2) ? ((t & 1) ? r.x[3] : r.x[2]) : ((t & 1) ? r.x[1] : r.x[0]);
+        const uint32_t send = send_bit(u >> 8, s_tsum[t].x, c, a.eps_b);
+        a.sent[t] = (uint8_t)send;
+        if (a.user_sent != nullptr) a.user_sent[t] = (uint8_t)send;
+        if (send) atomicAdd(&s_count, (unsigned long long)s_size[t]);
+    }
+    __syncthreads();
+    if (tid == 0) {
+        *a.c_out = c;
+        *a.count_out = (int64_t)s_count;
+        if (a.user_c != nullptr) *a.user_c = c;
+        if (a.user_count != nullptr) *a.user_count = (int64_t)s_count;
+    }
+}
+
+template <int RULE, int ARITH>
+__device__ __forceinline__ void update4(float4& th, float4& n, float4& b, float4& v, const float4& g,
+                                        float coef, const StatParams& sp) {
+    if (RULE == kRuleSgd) {
+        sgd_update(th.x, g.x, coef);
+        sgd_update(th.y, g.y, coef);
+        sgd_update(th.z, g.z, coef);
+        sgd_update(th.w, g.w, coef);
+    } else {
+        constexpr bool STD = RULE == kRuleFasgdStd;
+        rule_update<ARITH, STD>(th.x, n.x, b.x, v.x, g.x, coef, sp);
+        rule_update<ARITH, STD>(th.y, n.y, b.y, v.y, g.y, coef, sp);
+        rule_update<ARITH, STD>(th.z, n.z, b.z, v.z, g.z, coef, sp);
+        rule_update<ARITH, STD>(th.w, n.w, b.w, v.w, g.w, coef, sp);
+    }
+}
+
+template <int RULE, int ARITH>
+__device__ __forceinline__ void update1(const RangeArgs& a, int64_t p) {
+    float th = a.theta[p];
+    if (RULE == kRuleSgd) {
+        sgd_update(th, a.grad[p], a.coef);
+    } else {
+        float n = a.n[p], b = a.b[p], v = a.v[p];
+        rule_update<ARITH, RULE == kRuleFasgdStd>(th, n, b, v, a.grad[p], a.coef, a.sp);
+        a.n[p] = n;
+        a.b[p] = b;
+        a.v[p] = v;
+    }
+    a.theta[p] = th;
+}
+
+__device__ __forceinline__ float4 ld4(const float* base, int64_t q) {
+    return reinterpret_cast<const float4*>(base)[q];
+}
+__device__ __forceinline__ void st4(float* base, int64_t q, const float4& x) {
+    reinterpret_cast<float4*>(base)[q] = x;
+}
+
+// Eq. 4-8 (or Eq. 1-2) on every parameter of the transmitted tensors.  The
+// head and tail of an item (outside whole 16-byte quads) go element by
+// element; the quads two per thread per step, loads before stores.  When
+// partial is set (rules that change v), the block then re-forms the item's
+// sum of v from the values it just wrote (from L2), with the same element
+// order as the partial kernel, so the next decision needs no pass over v.
+template <int RULE, int ARITH>
+__global__ void __launch_bounds__(kItemThreads) tensor_apply_kernel(const __grid_constant__ RangeArgs a) {
+    constexpr bool FAS = RULE != kRuleSgd;
+    __shared__ float2 smem[kItemThreads / 32];
+    const int tid = threadIdx.x;
+    for (int64_t i = blockIdx.x; i < a.n_items; i += gridDim.x) {
+        const TensorItem it = a.items[i];
+        if (!a.sent[it.tensor]) continue;
+        const int64_t s = it.start, e = s + it.len;
+        const int64_t qs = (s + 3) >> 2, qe = e >> 2;
+        if (4 * qs >= e) {
+            for (int64_t p = s + tid; p < e; p += kItemThreads) update1<RULE, ARITH>(a, p);
+        } else {
+            if (tid < 4 * qs - s) update1<RULE, ARITH>(a, s + tid);
+            if (tid < e - 4 * qe) update1<RULE, ARITH>(a, 4 * qe + tid);
+            for (int64_t q0 = qs + tid; q0 < qe; q0 += 2 * kItemThreads) {
+                const int64_t q1 = q0 + kItemThreads;
+                const bool two = q1 < qe;
+                float4 th0, n0, b0, v0, g0, th1, n1, b1, v1, g1;
+                g0 = __ldcs(reinterpret_cast<const float4*>(a.grad) + q0);
+                th0 = ld4(a.theta, q0);
+                if (FAS) {
+                    n0 = ld4(a.n, q0);
+                    b0 = ld4(a.b, q0);
+                    v0 = ld4(a.v, q0);
+                }
+                if (two) {
+                    g1 = __ldcs(reinterpret_cast<const float4*>(a.grad) + q1);
+                    th1 = ld4(a.theta, q1);
+                    if (FAS) {
+                        n1 = ld4(a.n, q1);
+                        b1 = ld4(a.b, q1);
+                        v1 = ld4(a.v, q1);
+                    }
+                }
+                update4<RULE, ARITH>(th0, n0, b0, v0, g0, a.coef, a.sp);
+                st4(a.theta, q0, th0);
+                if (FAS) {
+                    st4(a.n, q0, n0);
+                    st4(a.b, q0, b0);
+                    st4(a.v, q0, v0);
+                }
+                if (two) {
+                    update4<RULE, ARITH>(th1, n1, b1, v1, g1, a.coef, a.sp);
+                    st4(a.theta, q1, th1);
+                    if (FAS) {
+                        st4(a.n, q1, n1);
+                        st4(a.b, q1, b1);
+                        st4(a.v, q1, v1);
+                    }
+                }
+            }
+        }
+        if (FAS && a.partial != nullptr) {
+            __syncthreads();    // the block's writes of v are visible to the block
+            const float2 sum = item_v_sum(it, a.v, smem);
+            if (tid == 0) a.partial[i] = sum;
+        }
+    }
+}
+
+// dst <- src on every parameter of the transmitted tensors, four quads per
+// thread in flight.
+__global__ void __launch_bounds__(kItemThreads) tensor_copy_kernel(const __grid_constant__ RangeArgs a) {
+    const int tid = threadIdx.x;
+    for (int64_t i = blockIdx.x; i < a.n_items; i += gridDim.x) {
+        const TensorItem it = a.items[i];
+        if (!a.sent[it.tensor]) continue;
+        const int64_t s = it.start, e = s + it.len;
+        const int64_t qs = (s + 3) >> 2, qe = e >> 2;
+        if (4 * qs >= e) {
+            for (int64_t p = s + tid; p < e; p += kItemThreads) a.dst[p] = a.src[p];
+            continue;
+        }
+        if (tid < 4 * qs - s) a.dst[s + tid] = a.src[s + tid];
+        if (tid < e - 4 * qe) a.dst[4 * qe + tid] = a.src[4 * qe + tid];
+        for (int64_t q = qs + tid; q < qe; q += 4 * kItemThreads) {
+            float4 x[4];
+#pragma unroll
+            for (int k = 0; k < 4; ++k)
+                if (q + k * kItemThreads < qe) x[k] = ld4(a.src, q + k * kItemThreads);
+#pragma unroll
+            for (int k = 0; k < 4; ++k)
+                if (q + k * kItemThreads < qe) st4(a.dst, q + k * kItemThreads, x[k]);
+        }
+    }
+}
+
+unsigned item_grid(int32_t n_items) { return (unsigned)(n_items > 0 ? n_items : 1); }
+
+template <int RULE, int ARITH>
+cudaError_t launch_apply_rule(const RangeArgs& a, cudaStream_t stream) {
+    tensor_apply_kernel<RULE, ARITH><<<item_grid(a.n_items), kItemThreads, 0, stream>>>(a);
+    return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_tensor_decide(const TensorArgs& a, bool sums_valid, cudaStream_t stream,
+                                 int64_t* launches) {
+    cudaError_t st;
+    if (!sums_valid) {
+        tensor_partial_kernel<<<item_grid(a.n_items), kItemThreads, 0, stream>>>(a);
+        st = cudaGetLastError();
+        if (st != cudaSuccess) return st;
+        ++*launches;
+    }
+    const size_t smem = tensor_resolve_smem(a.n_items, a.T);
+    st = cudaFuncSetAttribute(budget_resolve_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              (int)smem);
+    if (st != cudaSuccess) return st;
+    budget_resolve_kernel<<<1, kTensorResolveThreads, smem, stream>>>(a);
+    st = cudaGetLastError();
+    if (st == cudaSuccess) ++*launches;
+    return st;
+}
+
+cudaError_t launch_tensor_apply(const RangeArgs& a, int rule, bool exact, cudaStream_t stream,
+                                int64_t* launches) {
+    const bool ftz = a.sp.eps >= kFtzSafeEps;
+    cudaError_t st;
+    if (rule == kRuleSgd)
+        st = launch_apply_rule<kRuleSgd, kArithApprox>(a, stream);
+    else if (rule == kRuleFasgd)
+        st = exact ? launch_apply_rule<kRuleFasgd, kArithExact>(a, stream)
+             : ftz ? launch_apply_rule<kRuleFasgd, kArithApproxFtz>(a, stream)
+                   : launch_apply_rule<kRuleFasgd, kArithApprox>(a, stream);
+    else
+        st = exact ? launch_apply_rule<kRuleFasgdStd, kArithExact>(a, stream)
+             : ftz ? launch_apply_rule<kRuleFasgdStd, kArithApproxFtz>(a, stream)
+                   : launch_apply_rule<kRuleFasgdStd, kArithApprox>(a, stream);
+    if (st == cudaSuccess) ++*launches;
+    return st;
+}
+
+cudaError_t launch_tensor_copy(const RangeArgs& a, cudaStream_t stream, int64_t* launches) {
+    tensor_copy_kernel<<<item_grid(a.n_items), kItemThreads, 0, stream>>>(a);
+    cudaError_t st = cudaGetLastError();
+    if (st == cudaSuccess) ++*launches;
+    return st;
+}
+
+}  // namespace fasgd

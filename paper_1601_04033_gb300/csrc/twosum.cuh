@@ -1,0 +1,50 @@
+// Compensated fp32 summation shared by the mean-of-v reductions.
+#pragma once
+
+namespace fasgd {
+
+// hi + lo += x, with the rounding error of the fp32 addition recovered
+// exactly (TwoSum: six operations, no branch, no contraction).  lo collects
+// the errors in fp32 and is itself rounded, which bounds the pair's error by
+// a few ulp of lo -- far below one ulp of the fp64 total.
+__device__ __forceinline__ void two_sum_acc(float& hi, float& lo, float x) {
+    const float t = __fadd_rn(hi, x);
+    const float xp = __fsub_rn(t, hi);
+    const float hp = __fsub_rn(t, xp);
+    const float err = __fadd_rn(__fsub_rn(hi, hp), __fsub_rn(x, xp));
+    lo = __fadd_rn(lo, err);
+    hi = t;
+}
+
+// s + e = a + b exactly (Knuth's TwoSum).
+__device__ __forceinline__ void two_sum(float a, float b, float& s, float& e) {
+    s = __fadd_rn(a, b);
+    const float bp = __fsub_rn(s, a);
+    const float ap = __fsub_rn(s, bp);
+    e = __fadd_rn(__fsub_rn(a, ap), __fsub_rn(b, bp));
+}
+
+// (h, l) += (h2, l2) for float-float pairs of non-negative sums: the sum of
+// the high parts exactly, the low parts and that error added in fp32, then
+// renormalised so that |l| <= ulp(h) / 2.  Relative error a few 2^-48 per
+// addition for non-negative terms (no cancellation); pure fp32, so it runs
+// on the full-width pipes (the fp64 pipe is narrow on this part).
+__device__ __forceinline__ void ff_add(float& h, float& l, float h2, float l2) {
+    float s, e;
+    two_sum(h, h2, s, e);
+    e = __fadd_rn(e, __fadd_rn(l, l2));
+    two_sum(s, e, h, l);
+}
+
+// Warp-wide float-float sum over a fixed xor tree: every lane ends with the
+// same pair.
+__device__ __forceinline__ void ff_warp_sum(float& h, float& l) {
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) {
+        const float h2 = __shfl_xor_sync(0xffffffffu, h, off);
+        const float l2 = __shfl_xor_sync(0xffffffffu, l, off);
+        ff_add(h, l, h2, l2);
+    }
+}
+
+}  // namespace fasgd

@@ -55,6 +55,9 @@ SIGNATURES = {
     "fasgd_set_fetch_counts": (_i32, [_p, _p]),
     "bfasgd_push_message": (_i32, [_p, _i32, _i64, _p, _p]),
     "bfasgd_fetch_message": (_i32, [_p, _i32, _p, _p]),
+    "bfasgd_set_tensors": (_i32, [_p, _i32, _p]),
+    "bfasgd_push_budget": (_i32, [_p, _i32, _i64, _p, _i64, _p, _p, _p]),
+    "bfasgd_fetch_budget": (_i32, [_p, _i32, _p, _i64, _p, _p, _p]),
     "fasgd_sim_quadratic_grad": (_i32, [_i64, _p, _p, _p, _p, _u64, _i32, _u64, _p, _p]),
     "fasgd_sim_quadratic_loss": (_i32, [_i64, _p, _p, _p, _p, _p, _p]),
     "bfasgd_select_compact_noalloc": (_i32, [_i64, _p, _p, _f32, _f32, _u64, _i32, _u64,
@@ -63,6 +66,7 @@ SIGNATURES = {
 }
 
 NOALLOC_PMAX = 1 << 24
+BFASGD_TMAX = 4096
 
 
 def _load() -> ctypes.CDLL:
@@ -163,6 +167,18 @@ def bfasgd_push_message(h, client, timestamp, grad, sent_dev):
 
 def bfasgd_fetch_message(h, client, theta_client, fetched_dev):
     return LIB.bfasgd_fetch_message(h, client, theta_client, fetched_dev)
+
+
+def bfasgd_set_tensors(h, T, sizes):
+    return LIB.bfasgd_set_tensors(h, T, sizes)
+
+
+def bfasgd_push_budget(h, client, timestamp, grad, budget, sent_dev, c_dev, count_dev):
+    return LIB.bfasgd_push_budget(h, client, timestamp, grad, budget, sent_dev, c_dev, count_dev)
+
+
+def bfasgd_fetch_budget(h, client, theta_client, budget, sent_dev, c_dev, count_dev):
+    return LIB.bfasgd_fetch_budget(h, client, theta_client, budget, sent_dev, c_dev, count_dev)
 
 
 def fasgd_sim_quadratic_grad(P, theta, h, star, sigma, seed, client, n, grad, stream):
@@ -340,6 +356,24 @@ class Server:
 
     def fetch_message(self, client: int, theta_client, fetched_dev=None):
         self._check(bfasgd_fetch_message(self.h, client, _ptr(theta_client), _ptr(fetched_dev)))
+
+    def set_tensors(self, sizes):
+        """Partition theta into contiguous tensors (sizes: ints summing to P)."""
+        import numpy as np
+        s = np.ascontiguousarray(sizes, dtype=np.int64)
+        self._check(bfasgd_set_tensors(self.h, int(s.size), s.ctypes.data))
+
+    def push_budget(self, client: int, timestamp: int, grad, budget: int, sent_dev=None,
+                    c_dev=None, count_dev=None):
+        """Per-tensor B-FASGD push under a budget of expected parameters."""
+        self._check(bfasgd_push_budget(self.h, client, timestamp, _ptr(grad), int(budget),
+                                       _ptr(sent_dev), _ptr(c_dev), _ptr(count_dev)))
+
+    def fetch_budget(self, client: int, theta_client, budget: int, sent_dev=None, c_dev=None,
+                     count_dev=None):
+        """Per-tensor B-FASGD fetch into theta_client under a budget."""
+        self._check(bfasgd_fetch_budget(self.h, client, _ptr(theta_client), int(budget),
+                                        _ptr(sent_dev), _ptr(c_dev), _ptr(count_dev)))
 
     def fetch_counts(self):
         import numpy as np

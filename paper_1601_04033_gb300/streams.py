@@ -59,6 +59,7 @@ class Workload:
     s_hi: float = 1e-1
     R: int = 16            # gradient pool slots (>= 2K)
     send_frac: float | None = None   # B-FASGD target send fraction, None = dense
+    tensors: int = 0       # per-tensor B-FASGD: tensors in the partition (0: not used)
 
     def replace(self, **kw) -> "Workload":
         return dataclasses.replace(self, **kw)
@@ -77,6 +78,9 @@ WORKLOADS = {
     # The paper's literal B-FASGD (one decision per message) on the 25M shape.
     "bfasgd-message-25m": Workload("bfasgd-message-25m", 25_000_000, 64, 10_000, 0.001, 1,
                                    (FASGD,), "poisson8", 3, send_frac=0.20),
+    # Per-tensor B-FASGD with a bandwidth budget on the 25M shape: 160 tensors.
+    "bfasgd-tensor-25m": Workload("bfasgd-tensor-25m", 25_000_000, 64, 10_000, 0.001, 1,
+                                  (FASGD,), "poisson8", 3, send_frac=0.20, tensors=160),
     "fasgd-268m-k16": Workload("fasgd-268m-k16", 268_435_456, 256, 2_000, 0.001, 16,
                                (FASGD,), "pareto1.5", 4, s_lo=1e-5, s_hi=1.0, R=32,
                                send_frac=0.20),
@@ -97,6 +101,13 @@ def grad_model(w: Workload, P: int | None = None):
          * np.float32(1e-3))
     lo, hi = math.log(w.s_lo), math.log(w.s_hi)
     s = np.exp(_rng(w.seed, _TAG_SPREAD).uniform(lo, hi, P)).astype(np.float32)
+    if w.tensors and P >= w.tensors:
+        # Layer structure: each tensor's spreads share a scale, log-uniform
+        # over two decades, so the per-tensor statistics differ.
+        sizes = tensor_sizes(w.seed, P, w.tensors)
+        scale = np.exp(_rng(w.seed, _TAG_TENSORS, 0).uniform(math.log(0.1), math.log(10.0),
+                                                               w.tensors))
+        s *= np.repeat(scale.astype(np.float32), sizes)
     return m, s
 
 
@@ -245,6 +256,38 @@ def quadratic_objective(seed: int, P: int, h_lo: float = 1e-2, h_hi: float = 10.
         sigma = np.exp(_rng(seed, _TAG_OBJ_SIGMA).uniform(math.log(sigma_lo), math.log(sigma_hi),
                                                           P)).astype(np.float32)
     return h, star, sigma
+
+
+_TAG_TENSORS = 11
+
+
+def tensor_sizes(seed: int, P: int, T: int) -> np.ndarray:
+    """A partition of P parameters into T contiguous tensors with the size mix
+    of a layered network: alternating weight tensors (relative sizes
+    log-uniform over three decades) and vector tensors (biases / scales,
+    log-uniform in [16, 4096] parameters, at most a quarter of P in all).
+    P = 7,850 with T = 2 is the paper's softmax-regression model on 28x28
+    inputs and 10 classes (784 x 10 weights, then 10 biases).  int64[T]."""
+    if T < 1 or P < T:
+        raise ValueError("need 1 <= T <= P")
+    if T == 1:
+        return np.array([P], np.int64)
+    if P == 7_850 and T == 2:
+        return np.array([7_840, 10], np.int64)
+    g = _rng(seed, _TAG_TENSORS, T)
+    n_vec = T // 2
+    n_mat = T - n_vec
+    vec = np.exp(g.uniform(math.log(16), math.log(4096), n_vec))
+    vec = np.maximum(1, np.floor(vec * min(1.0, (P / 4) / vec.sum()))).astype(np.int64)
+    rest = P - int(vec.sum())
+    w = np.exp(g.uniform(0.0, math.log(1000.0), n_mat))
+    mat = np.maximum(1, np.floor(w / w.sum() * (rest - n_mat))).astype(np.int64)
+    mat[int(np.argmax(mat))] += rest - int(mat.sum())
+    out = np.empty(T, np.int64)
+    out[0::2] = mat
+    out[1::2] = vec
+    assert out.min() >= 1 and int(out.sum()) == P
+    return out
 
 
 def dispatch_schedule(seed: int, lam: int, n_batches: int, K: int = 1, rho: float = 1.0):
