@@ -147,6 +147,9 @@ struct fasgd_s {
     uint8_t* t_sent = nullptr;
     float* t_c = nullptr;
     int64_t* t_count = nullptr;
+    float* t_vbar = nullptr;       // cached tensor means
+    uint8_t* t_dirty = nullptr;    // tensors whose v changed since their mean was formed
+    long long* t_cprev = nullptr;  // last threshold per stream (push, fetch)
     bool t_sums_valid = false;   // t_partial holds the item sums of the current v
 
     void free_tensors() {
@@ -157,6 +160,12 @@ struct fasgd_s {
         cudaFree(t_sent);
         cudaFree(t_c);
         cudaFree(t_count);
+        cudaFree(t_vbar);
+        cudaFree(t_dirty);
+        cudaFree(t_cprev);
+        t_vbar = nullptr;
+        t_dirty = nullptr;
+        t_cprev = nullptr;
         t_items = nullptr;
         t_item_begin = nullptr;
         t_sizes = nullptr;
@@ -197,6 +206,11 @@ struct fasgd_s {
         a.user_sent = sent_out;
         a.user_c = c_out;
         a.user_count = count_out;
+        a.vbar_cache = t_vbar;
+        a.dirty = t_dirty;
+        a.c_prev = t_cprev + stream_id;
+        a.all_dirty = t_sums_valid ? 0 : 1;
+        a.mark_dirty = (stream_id == 0 && variant != FASGD_ASGD && variant != FASGD_SASGD) ? 1 : 0;
         cudaError_t st = fasgd::launch_tensor_decide(a, t_sums_valid, stream, &launches);
         if (st == cudaSuccess) {
             t_sums_valid = true;
@@ -582,6 +596,11 @@ int bfasgd_set_tensors(fasgd_t* h, int32_t T, const int64_t* sizes) {
     if (st == cudaSuccess) st = cudaMalloc(reinterpret_cast<void**>(&h->t_sent), (size_t)T);
     if (st == cudaSuccess) st = cudaMalloc(reinterpret_cast<void**>(&h->t_c), sizeof(float));
     if (st == cudaSuccess) st = cudaMalloc(reinterpret_cast<void**>(&h->t_count), sizeof(int64_t));
+    if (st == cudaSuccess) st = cudaMalloc(reinterpret_cast<void**>(&h->t_vbar), (size_t)T * sizeof(float));
+    if (st == cudaSuccess) st = cudaMalloc(reinterpret_cast<void**>(&h->t_dirty), (size_t)T);
+    if (st == cudaSuccess) st = cudaMalloc(reinterpret_cast<void**>(&h->t_cprev), 2 * sizeof(long long));
+    if (st == cudaSuccess) st = cudaMemset(h->t_dirty, 1, (size_t)T);
+    if (st == cudaSuccess) st = cudaMemset(h->t_cprev, 0xff, 2 * sizeof(long long));   // none yet
     if (st == cudaSuccess)
         st = cudaMemcpy(h->t_items, items.data(), ni * sizeof(fasgd::TensorItem), cudaMemcpyHostToDevice);
     if (st == cudaSuccess)

@@ -9,9 +9,10 @@
 //      exact rounding errors (TwoSum), then a fixed float-float tree -- into
 //      one float-float pair per item;
 //   2. budget_resolve (one block of 1024 threads): vbar_t = fl32(sum of the
-//      item sums of tensor t / s_t), the budget threshold c, then the Philox
-//      draw and the exact Eq. 9 decision of every tensor and the number of
-//      parameters transmitted.
+//      item sums of tensor t / s_t) for the tensors whose v changed since the
+//      last decision (the others keep their cached vbar_t), the budget
+//      threshold c, then the Philox draw and the exact Eq. 9 decision of
+//      every tensor and the number of parameters transmitted.
 // Then tensor_apply (a push: Eq. 4-8, or Eq. 1-2, on the transmitted
 // tensors) or tensor_copy (a fetch: theta into the client's copy) walks the
 // items of the transmitted tensors; the others cost one flag read.  The
@@ -29,7 +30,8 @@
 // (ordered as their values): each round evaluates E at 2^m - 1 points of
 // the current interval, one group of warps per point (lanes over tensors,
 // then an exact integer sum), and keeps the part between the last failing
-// and the first passing point.
+// and the first passing point; the first round is centred on the previous
+// threshold of the same stream, since the statistics move little per call.
 
 #include "eq9.cuh"
 #include "kernels.cuh"
@@ -123,47 +125,69 @@ __device__ __forceinline__ long long candidate(long long lo, long long hi, int k
     return span <= (1ll << m) ? lo + 1 + k : lo + ((span * (k + 1)) >> m);
 }
 
+// Candidate k of a first round centred on the previous threshold's bit
+// pattern cp (the statistics move little between calls): cp itself and
+// cp -/+ 2^s for s growing to 18 (about 3 % of the value), non-decreasing in
+// k; if c has moved further, the round still leaves a valid, wider interval.
+__device__ __forceinline__ long long warm_candidate(long long cp, int k, int m) {
+    const int h = (1 << (m - 1)) - 1;
+    const int j = k - h;
+    if (j == 0) return cp;
+    const int aj = j < 0 ? -j : j;
+    const long long off = 1ll << ((18 * aj + h / 2) / h);
+    const long long c = j < 0 ? cp - off : cp + off;
+    return c < 0 ? 0 : (c > 0x7f800000 ? 0x7f800000 : c);
+}
+
 __global__ void __launch_bounds__(kTensorResolveThreads) budget_resolve_kernel(const __grid_constant__ TensorArgs a) {
-    // Dynamic shared memory (tensor_resolve_smem): the item sums, the
-    // per-tensor sums (whose high word then holds vbar_t), the item ranges
-    // and the sizes.  Everything the block reads more than once is loaded
-    // once, with all loads in flight together.
+    // Dynamic shared memory (tensor_resolve_smem): the item sums, vbar_t,
+    // the item ranges, the sizes and the stale flags, each loaded once with
+    // all loads in flight together.
     extern __shared__ __align__(16) unsigned char dsm[];
     float2* s_part = reinterpret_cast<float2*>(dsm);
-    float2* s_tsum = s_part + a.n_items;
-    int32_t* s_begin = reinterpret_cast<int32_t*>(s_tsum + a.T);
+    float* s_vbar = reinterpret_cast<float*>(s_part + a.n_items);
+    int32_t* s_begin = reinterpret_cast<int32_t*>(s_vbar + a.T);
     int32_t* s_size = s_begin + a.T + 1;
-    __shared__ unsigned long long s_pw[2][32];
+    uint8_t* s_dirty = reinterpret_cast<uint8_t*>(s_size + a.T);
+    __shared__ unsigned long long s_e[32];
+    __shared__ long long s_lo, s_hi, s_cp;
     __shared__ unsigned long long s_count;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     for (int i = tid; i < a.n_items; i += kTensorResolveThreads) s_part[i] = a.partial[i];
     for (int t = tid; t <= a.T; t += kTensorResolveThreads) s_begin[t] = a.item_begin[t];
-    for (int t = tid; t < a.T; t += kTensorResolveThreads) s_size[t] = a.sizes[t];
-    if (tid == 0) s_count = 0;
+    for (int t = tid; t < a.T; t += kTensorResolveThreads) {
+        s_size[t] = a.sizes[t];
+        s_dirty[t] = a.all_dirty ? 1 : a.dirty[t];
+        s_vbar[t] = a.vbar_cache[t];
+    }
+    if (tid == 0) {
+        s_count = 0;
+        s_cp = *a.c_prev;
+    }
     __syncthreads();
-    // Sum of the item sums of tensor t: warp (t mod 32), lanes over the
-    // items, then a fixed shuffle tree, all in float-float.
+    // vbar_t of every tensor whose v changed since it was last formed: warp
+    // (t mod 32) adds its item sums (lanes over the items, then a fixed
+    // shuffle tree, all in float-float), lane 0 divides in fp64.  The others
+    // keep the cached value -- the same bits, since the item sums are.
     for (int t = warp; t < a.T; t += 32) {
+        if (!s_dirty[t]) continue;
         float h = 0.f, l = 0.f;
         for (int i = s_begin[t] + lane; i < s_begin[t + 1]; i += 32)
             ff_add(h, l, s_part[i].x, s_part[i].y);
         ff_warp_sum(h, l);
-        if (lane == 0) s_tsum[t] = make_float2(h, l);
-    }
-    __syncthreads();
-    // vbar_t = fl32(sum / s_t): the pair widened to fp64 once, one fp64
-    // division per tensor, all tensors at once.
-    for (int t = tid; t < a.T; t += kTensorResolveThreads) {
-        const float2 p = s_tsum[t];
-        s_tsum[t].x = (float)(((double)p.x + (double)p.y) / (double)s_size[t]);
+        if (lane == 0) {
+            const float vb = (float)(((double)h + (double)l) / (double)s_size[t]);
+            s_vbar[t] = vb;
+            a.vbar_cache[t] = vb;
+            a.dirty[t] = 0;
+        }
     }
     __syncthreads();
     // Invariant: E(lo) > limit >= E(hi) (lo = -1 stands below 0, hi = +inf
     // has E = 0); c = hi once they are adjacent.  2^m is chosen so that a
     // thread takes about two tensors per candidate: the work of a round
     // grows with the number of candidates times T, the number of rounds only
-    // with its log.  One barrier per round: every warp re-derives the new
-    // interval from the same partial sums (double-buffered).
+    // with its log.
     int m = 5;
     while (m > 1 && (a.T << m) > 2 * kTensorResolveThreads) --m;
     const int gwarps = 32 >> m;                      // warps per group; the last group idles
@@ -171,57 +195,71 @@ __global__ void __launch_bounds__(kTensorResolveThreads) budget_resolve_kernel(c
     const int gthread = tid - group * gwarps * 32;
     const int gsize = gwarps * 32;
     const int ncand = (1 << m) - 1;
+    const long long cp = s_cp;
+    const bool warm = m >= 3 && cp >= 0 && cp <= 0x7f800000;
     long long lo = -1, hi = 0x7f800000;
     for (int round = 0; round < 64 && hi - lo > 1; ++round) {
-        const int buf = round & 1;
+        const bool w0 = warm && round == 0;
         unsigned long long e = 0;
         if (group < ncand) {
-            const long long cand = candidate(lo, hi, group, m);
+            const long long cand = w0 ? warm_candidate(cp, group, m) : candidate(lo, hi, group, m);
             if (cand < hi) {
                 const float x = __uint_as_float((uint32_t)cand);
                 for (int t = gthread; t < a.T; t += gsize)
-                    e += budget_term(s_size[t], s_tsum[t].x, a.eps_b, x);
+                    e += budget_term(s_size[t], s_vbar[t], a.eps_b, x);
             }
         }
 #pragma unroll
         for (int off = 16; off > 0; off >>= 1) e += __shfl_xor_sync(kFull, e, off);
-        if (lane == 0) s_pw[buf][warp] = e;
+        if (lane == 0) s_e[warp] = e;
         __syncthreads();
-        // Lane k adds the partials of group k and tests candidate k; E is
-        // non-increasing, so the passing candidates are a suffix.
-        int ok = 1;
-        long long cand = hi;
-        if (lane < ncand) {
-            cand = candidate(lo, hi, lane, m);
-            if (cand < hi) {
-                unsigned long long sum = 0;
-                for (int w = 0; w < gwarps; ++w) sum += s_pw[buf][lane * gwarps + w];
-                ok = (long long)sum <= a.limit;
-            } else {
-                cand = hi;
+        if (warp == 0) {
+            // Lane k adds the partials of group k and tests candidate k; E is
+            // non-increasing and the candidates non-decreasing, so the passing
+            // candidates are a suffix.
+            int ok = 1;
+            long long cand = hi;
+            if (lane < ncand) {
+                cand = w0 ? warm_candidate(cp, lane, m) : candidate(lo, hi, lane, m);
+                if (cand < hi) {
+                    unsigned long long sum = 0;
+                    for (int w = 0; w < gwarps; ++w) sum += s_e[lane * gwarps + w];
+                    ok = (long long)sum <= a.limit;
+                } else {
+                    cand = hi;
+                }
+            }
+            const unsigned pass = __ballot_sync(kFull, ok);   // lanes >= ncand pass
+            const int first = __ffs(pass) - 1;
+            const long long c_first = __shfl_sync(kFull, cand, first);
+            const long long c_prev = __shfl_sync(kFull, cand, first > 0 ? first - 1 : 0);
+            if (lane == 0) {
+                s_hi = c_first;
+                s_lo = first > 0 ? c_prev : lo;
             }
         }
-        const unsigned pass = __ballot_sync(kFull, ok);   // lanes >= ncand pass
-        const int first = __ffs(pass) - 1;
-        const long long c_first = __shfl_sync(kFull, cand, first);
-        const long long c_prev = __shfl_sync(kFull, cand, first > 0 ? first - 1 : 0);
-        if (first > 0) lo = c_prev;
-        hi = c_first;
+        __syncthreads();
+        lo = s_lo;
+        hi = s_hi;
     }
     const float c = __uint_as_float((uint32_t)hi);
     for (int t = tid; t < a.T; t += kTensorResolveThreads) {
         const Philox4 r = philox4x32_10(0x80000000u + ((uint32_t)t >> 2), a.client_word, a.n_lo,
                                         a.n_hi, a.round_key0, a.round_key1);
         const uint32_t u = (t & 2) ? ((t & 1) ? r.x[3] : r.x[2]) : ((t & 1) ? r.x[1] : r.x[0]);
-        const uint32_t send = send_bit(u >> 8, s_tsum[t].x, c, a.eps_b);
+        const uint32_t send = send_bit(u >> 8, s_vbar[t], c, a.eps_b);
         a.sent[t] = (uint8_t)send;
         if (a.user_sent != nullptr) a.user_sent[t] = (uint8_t)send;
-        if (send) atomicAdd(&s_count, (unsigned long long)s_size[t]);
+        if (send) {
+            atomicAdd(&s_count, (unsigned long long)s_size[t]);
+            if (a.mark_dirty) a.dirty[t] = 1;    // the apply that follows rewrites its v
+        }
     }
     __syncthreads();
     if (tid == 0) {
         *a.c_out = c;
         *a.count_out = (int64_t)s_count;
+        *a.c_prev = hi;
         if (a.user_c != nullptr) *a.user_c = c;
         if (a.user_count != nullptr) *a.user_count = (int64_t)s_count;
     }

@@ -20,7 +20,7 @@ inline int64_t tensor_chunk(int64_t P) {
 constexpr int kTensorResolveThreads = 1024;
 // Dynamic shared memory of the decision kernel for n_items items and T tensors.
 inline size_t tensor_resolve_smem(int32_t n_items, int32_t T) {
-    return (size_t)n_items * 8 + (size_t)T * 8 + ((size_t)T + 1) * 4 + (size_t)T * 4;
+    return (size_t)n_items * 8 + (size_t)T * 4 + ((size_t)T + 1) * 4 + (size_t)T * 4 + (size_t)T;
 }
 struct TensorArgs {
     const float* v;               // the server's statistic, fp32[P]
@@ -42,6 +42,11 @@ struct TensorArgs {
     uint8_t* user_sent;           // caller copies, each may be null
     float* user_c;
     int64_t* user_count;
+    float* vbar_cache;            // T: vbar_t as last formed
+    uint8_t* dirty;               // T: v of tensor t changed since vbar_t was formed
+    long long* c_prev;            // bit pattern of this stream's last threshold (< 0: none)
+    int32_t all_dirty;            // form every vbar_t afresh
+    int32_t mark_dirty;           // the transmitted tensors' v is about to change (a push)
 };
 // The transmitted tensors of one decision: Eq. 4-8 (or Eq. 1-2) with grad,
 // or (copy mode) dst <- src.
