@@ -116,6 +116,22 @@ __device__ __forceinline__ uint64_t budget_term(int32_t size, float vbar, float 
     return shift > -64 ? prod >> (-shift) : 0;
 }
 
+// fl32((h + l) / s) for a float-float pair (h >= 0, |l| <= ulp(h)) and an
+// integer 1 <= s < 2^31, in fp32 only (the fp64 pipe is narrow here): with
+// sh = fl(s) and sl = s - sh (exact, |sl| <= 64), q0 = fl(h / sh) leaves the
+// residual h - q0 sh exactly representable (one fused multiply-add forms
+// it); adding l and subtracting q0 sl rounds terms some 2^-20 of ulp(q0)
+// small, so fl(q0 + r / sh) is the correctly rounded quotient except within
+// about 2^-43 (relative) of a rounding boundary.
+__device__ __forceinline__ float ff_div_int(float h, float l, int32_t s) {
+    const float sh = __int2float_rn(s);
+    const float sl = __ll2float_rn((long long)s - __float2ll_rn(sh));
+    const float q0 = __fdiv_rn(h, sh);
+    const float e1 = __fmaf_rn(-q0, sh, h);
+    const float r = __fsub_rn(__fadd_rn(e1, l), __fmul_rn(q0, sl));
+    return __fadd_rn(q0, __fdiv_rn(r, sh));
+}
+
 // Candidate k (0 .. 2^m - 2) of a search round inside the open interval
 // (lo, hi) of bit patterns: 2^m - 1 points cutting it into 2^m near-equal
 // parts (consecutive patterns once the interval is short); values >= hi are
@@ -134,18 +150,19 @@ __device__ __forceinline__ long long warm_candidate(long long cp, int k, int m) 
     const int j = k - h;
     if (j == 0) return cp;
     const int aj = j < 0 ? -j : j;
-    const long long off = 1ll << ((18 * aj + h / 2) / h);
+    const long long off = 1ll << ((18 * aj + (h >> 1)) / h);
     const long long c = j < 0 ? cp - off : cp + off;
     return c < 0 ? 0 : (c > 0x7f800000 ? 0x7f800000 : c);
 }
 
 __global__ void __launch_bounds__(kTensorResolveThreads) budget_resolve_kernel(const __grid_constant__ TensorArgs a) {
-    // Dynamic shared memory (tensor_resolve_smem): the item sums, vbar_t,
-    // the item ranges, the sizes and the stale flags, each loaded once with
-    // all loads in flight together.
+    // Dynamic shared memory (tensor_resolve_smem): the item sums, the tensor
+    // sums, vbar_t, the item ranges, the sizes and the stale flags, each
+    // loaded once with all loads in flight together.
     extern __shared__ __align__(16) unsigned char dsm[];
     float2* s_part = reinterpret_cast<float2*>(dsm);
-    float* s_vbar = reinterpret_cast<float*>(s_part + a.n_items);
+    float2* s_sum = s_part + a.n_items;
+    float* s_vbar = reinterpret_cast<float*>(s_sum + a.T);
     int32_t* s_begin = reinterpret_cast<int32_t*>(s_vbar + a.T);
     int32_t* s_size = s_begin + a.T + 1;
     uint8_t* s_dirty = reinterpret_cast<uint8_t*>(s_size + a.T);
@@ -153,12 +170,27 @@ __global__ void __launch_bounds__(kTensorResolveThreads) budget_resolve_kernel(c
     __shared__ long long s_lo, s_hi, s_cp;
     __shared__ unsigned long long s_count;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    for (int i = tid; i < a.n_items; i += kTensorResolveThreads) s_part[i] = a.partial[i];
-    for (int t = tid; t <= a.T; t += kTensorResolveThreads) s_begin[t] = a.item_begin[t];
-    for (int t = tid; t < a.T; t += kTensorResolveThreads) {
-        s_size[t] = a.sizes[t];
-        s_dirty[t] = a.all_dirty ? 1 : a.dirty[t];
-        s_vbar[t] = a.vbar_cache[t];
+    // One pass of loads (every load of a thread issued before any store).
+    const int nload = a.n_items > a.T + 1 ? a.n_items : a.T + 1;
+    for (int i = tid; i < nload; i += kTensorResolveThreads) {
+        float2 pv = make_float2(0.f, 0.f);
+        int32_t bg = 0, sz = 0;
+        uint8_t dt = 1;
+        float vb = 0.f;
+        if (i < a.n_items) pv = a.partial[i];
+        if (i <= a.T) bg = a.item_begin[i];
+        if (i < a.T) {
+            sz = a.sizes[i];
+            vb = a.vbar_cache[i];
+            if (!a.all_dirty) dt = a.dirty[i];
+        }
+        if (i < a.n_items) s_part[i] = pv;
+        if (i <= a.T) s_begin[i] = bg;
+        if (i < a.T) {
+            s_size[i] = sz;
+            s_vbar[i] = vb;
+            s_dirty[i] = dt;
+        }
     }
     if (tid == 0) {
         s_count = 0;
@@ -167,20 +199,25 @@ __global__ void __launch_bounds__(kTensorResolveThreads) budget_resolve_kernel(c
     __syncthreads();
     // vbar_t of every tensor whose v changed since it was last formed: warp
     // (t mod 32) adds its item sums (lanes over the items, then a fixed
-    // shuffle tree, all in float-float), lane 0 divides in fp64.  The others
-    // keep the cached value -- the same bits, since the item sums are.
+    // shuffle tree, all in float-float); then thread t divides (ff_div_int).
+    // The other tensors keep the cached value -- the same bits, since the
+    // item sums are.
     for (int t = warp; t < a.T; t += 32) {
         if (!s_dirty[t]) continue;
         float h = 0.f, l = 0.f;
         for (int i = s_begin[t] + lane; i < s_begin[t + 1]; i += 32)
             ff_add(h, l, s_part[i].x, s_part[i].y);
         ff_warp_sum(h, l);
-        if (lane == 0) {
-            const float vb = (float)(((double)h + (double)l) / (double)s_size[t]);
-            s_vbar[t] = vb;
-            a.vbar_cache[t] = vb;
-            a.dirty[t] = 0;
-        }
+        if (lane == 0) s_sum[t] = make_float2(h, l);
+    }
+    __syncthreads();
+    for (int t = tid; t < a.T; t += kTensorResolveThreads) {
+        if (!s_dirty[t]) continue;
+        const float2 p = s_sum[t];
+        const float vb = ff_div_int(p.x, p.y, s_size[t]);
+        s_vbar[t] = vb;
+        a.vbar_cache[t] = vb;
+        a.dirty[t] = 0;
     }
     __syncthreads();
     // Invariant: E(lo) > limit >= E(hi) (lo = -1 stands below 0, hi = +inf
@@ -243,17 +280,23 @@ __global__ void __launch_bounds__(kTensorResolveThreads) budget_resolve_kernel(c
         hi = s_hi;
     }
     const float c = __uint_as_float((uint32_t)hi);
-    for (int t = tid; t < a.T; t += kTensorResolveThreads) {
-        const Philox4 r = philox4x32_10(0x80000000u + ((uint32_t)t >> 2), a.client_word, a.n_lo,
-                                        a.n_hi, a.round_key0, a.round_key1);
-        const uint32_t u = (t & 2) ? ((t & 1) ? r.x[3] : r.x[2]) : ((t & 1) ? r.x[1] : r.x[0]);
-        const uint32_t send = send_bit(u >> 8, s_vbar[t], c, a.eps_b);
-        a.sent[t] = (uint8_t)send;
-        if (a.user_sent != nullptr) a.user_sent[t] = (uint8_t)send;
-        if (send) {
-            atomicAdd(&s_count, (unsigned long long)s_size[t]);
-            if (a.mark_dirty) a.dirty[t] = 1;    // the apply that follows rewrites its v
+    // Whole warps walk the tensors (the count is summed with a shuffle).
+    for (int t0 = tid - lane; t0 < a.T; t0 += kTensorResolveThreads) {
+        const int t = t0 + lane;
+        unsigned long long n = 0;
+        if (t < a.T) {
+            const Philox4 r = philox4x32_10(0x80000000u + ((uint32_t)t >> 2), a.client_word, a.n_lo,
+                                            a.n_hi, a.round_key0, a.round_key1);
+            const uint32_t u = (t & 2) ? ((t & 1) ? r.x[3] : r.x[2]) : ((t & 1) ? r.x[1] : r.x[0]);
+            const uint32_t send = send_bit(u >> 8, s_vbar[t], c, a.eps_b);
+            a.sent[t] = (uint8_t)send;
+            if (a.user_sent != nullptr) a.user_sent[t] = (uint8_t)send;
+            if (send && a.mark_dirty) a.dirty[t] = 1;    // the apply that follows rewrites its v
+            n = send ? (unsigned long long)s_size[t] : 0ull;
         }
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) n += __shfl_xor_sync(kFull, n, off);
+        if (lane == 0 && n != 0) atomicAdd(&s_count, n);
     }
     __syncthreads();
     if (tid == 0) {
@@ -371,7 +414,7 @@ __global__ void __launch_bounds__(kItemThreads) tensor_apply_kernel(const __grid
     }
 }
 
-// dst <- src on every parameter of the transmitted tensors, four quads per
+// dst <- src on every parameter of the transmitted tensors, eight quads per
 // thread in flight.
 __global__ void __launch_bounds__(kItemThreads) tensor_copy_kernel(const __grid_constant__ RangeArgs a) {
     const int tid = threadIdx.x;
@@ -386,13 +429,13 @@ __global__ void __launch_bounds__(kItemThreads) tensor_copy_kernel(const __grid_
         }
         if (tid < 4 * qs - s) a.dst[s + tid] = a.src[s + tid];
         if (tid < e - 4 * qe) a.dst[4 * qe + tid] = a.src[4 * qe + tid];
-        for (int64_t q = qs + tid; q < qe; q += 4 * kItemThreads) {
-            float4 x[4];
+        for (int64_t q = qs + tid; q < qe; q += 8 * kItemThreads) {
+            float4 x[8];
 #pragma unroll
-            for (int k = 0; k < 4; ++k)
+            for (int k = 0; k < 8; ++k)
                 if (q + k * kItemThreads < qe) x[k] = ld4(a.src, q + k * kItemThreads);
 #pragma unroll
-            for (int k = 0; k < 4; ++k)
+            for (int k = 0; k < 8; ++k)
                 if (q + k * kItemThreads < qe) st4(a.dst, q + k * kItemThreads, x[k]);
         }
     }
