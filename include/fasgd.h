@@ -239,7 +239,7 @@ FASGD_API int bfasgd_fetch_apply(int64_t P, float* theta_client, const int32_t* 
  * bfasgd_push_message -- the paper's literal B-FASGD push (Sec. 2.3): one
  * decision for the whole message.  When the push is applied (in arrival
  * order, by fasgd_apply_pending), the server forms vbar = the mean of v over
- * all P parameters (fp64 sum in a fixed order, rounded once to fp32), draws u
+ * all P parameters (a compensated sum in a fixed order, rounded once to fp32), draws u
  * (Philox4x32-10 word 0 at counter (2^32-1, client, n, n >> 32), key = seed,
  * n = the client's push count, which then advances) and transmits iff Eq. 9
  * holds: u / 2^24 < 1 / (1 + c_push / (vbar + eps_b)), decided exactly in

@@ -88,28 +88,6 @@ struct ScatterArgs {
     int32_t* err;              // may be null; flags 1 (count) and 2 (index)
 };
 
-// One per-message B-FASGD decision (push or fetch) and, when the message is
-// transmitted, the copy src -> dst (P floats, both 16-byte aligned).
-constexpr int kMessageMaxBlocks = 1024;
-
-struct MessageArgs {
-    const float* v;            // the server's statistic, fp32[P]
-    int64_t P;
-    double* partial;           // scratch: nblocks partial sums
-    int32_t nblocks;           // message_partial_blocks(P)
-    float c;                   // c_push or c_fetch
-    float eps_b;
-    uint32_t round_key0[10];
-    uint32_t round_key1[10];
-    uint32_t client_word;      // client + 2^31 * stream (0: push, 1: fetch)
-    uint32_t n_lo, n_hi;       // the client's count of earlier messages of that stream
-    const float* src;          // may be null: decide only
-    float* dst;
-    int32_t* flag_out;         // may be null: 1 transmitted, 0 dropped
-};
-
-int32_t message_partial_blocks(int64_t P);
-
 // Closed-loop simulation: stochastic gradient and loss of the synthetic
 // quadratic objective (sim.cu).
 struct SimGradArgs {
@@ -143,8 +121,6 @@ cudaError_t launch_sparse(const SparseArgs& a, int rule, bool exact, int num_sms
                           int64_t* launches);
 cudaError_t launch_select(const SelectArgs& a, cudaStream_t stream, int64_t* launches);
 cudaError_t launch_scatter(const ScatterArgs& a, int num_sms, cudaStream_t stream);
-cudaError_t launch_message(const MessageArgs& a, int num_sms, cudaStream_t stream,
-                           int64_t* launches);
 cudaError_t launch_sim_grad(const SimGradArgs& a, int num_sms, cudaStream_t stream);
 cudaError_t launch_sim_loss(const SimLossArgs& a, cudaStream_t stream);
 

@@ -6,9 +6,10 @@
 //   1. vbar_partial: fixed partition of the parameters into contiguous
 //      chunks, one per block; each block sums its chunk of v (fixed order: per
 //      thread in index order as an fp32 sum plus its exact rounding errors,
-//      then a fixed fp64 shuffle tree) into one fp64 partial;
-//   2. message_resolve: every block adds the partials in the same fixed order,
-//      forms vbar = fl32(sum / P), draws u (Philox4x32-10, word 0 at counter
+//      then a fixed float-float tree) into one float-float partial;
+//   2. message_resolve: every block adds the partials in the same fixed order
+//      (float-float), forms vbar = fl32(sum / P) (ff_div_int), draws u
+//      (Philox4x32-10, word 0 at counter
 //      (2^32-1, client + 2^31 * stream, n)), takes the exact Eq. 9 decision,
 //      and, if the message is transmitted, copies src to dst (grid-stride,
 //      128-bit); block 0 reports the decision.
@@ -20,58 +21,71 @@
 
 #include "eq9.cuh"
 #include "kernels.cuh"
+#include "message.cuh"
 #include "twosum.cuh"
 
 namespace fasgd {
 namespace {
 
 constexpr int kMsgThreads = 256;
-constexpr unsigned kFull = 0xffffffffu;
-
-__device__ __forceinline__ double block_sum(double s, double* smem) {
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1) s += __shfl_xor_sync(kFull, s, off);
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    if (lane == 0) smem[warp] = s;
-    __syncthreads();
-    double t = 0.0;
-    if (threadIdx.x == 0)
-        for (int w = 0; w < kMsgThreads / 32; ++w) t += smem[w];
-    return t;  // valid in thread 0
-}
 
 __global__ void __launch_bounds__(kMsgThreads) vbar_partial_kernel(const __grid_constant__ MessageArgs a) {
-    __shared__ double smem[kMsgThreads / 32];
+    __shared__ float2 smem[kMsgThreads / 32];
     const int64_t nq = a.P >> 2;
     const int64_t chunk = (nq + a.nblocks - 1) / a.nblocks;
     const int64_t q0 = (int64_t)blockIdx.x * chunk;
     const int64_t q1 = q0 + chunk < nq ? q0 + chunk : nq;
     // Per thread: an fp32 sum with its exact rounding error carried alongside
-    // (Knuth's TwoSum), so the pair is the exact sum of the values added;
-    // only the per-thread and per-block combines use the (slow) fp64 pipe.
+    // (Knuth's TwoSum), four quads loaded before they are added.
     float hi = 0.f, lo = 0.f;
-    for (int64_t q = q0 + threadIdx.x; q < q1; q += kMsgThreads) {
-        const float4 x = __ldcs(reinterpret_cast<const float4*>(a.v + 4 * q));
-        two_sum_acc(hi, lo, x.x);
-        two_sum_acc(hi, lo, x.y);
-        two_sum_acc(hi, lo, x.z);
-        two_sum_acc(hi, lo, x.w);
+    const float4* v4 = reinterpret_cast<const float4*>(a.v);
+    for (int64_t q = q0 + threadIdx.x; q < q1; q += 4 * kMsgThreads) {
+        float4 x[4];
+#pragma unroll
+        for (int k = 0; k < 4; ++k)
+            if (q + k * kMsgThreads < q1) x[k] = __ldcs(v4 + q + k * kMsgThreads);
+#pragma unroll
+        for (int k = 0; k < 4; ++k)
+            if (q + k * kMsgThreads < q1) {
+                two_sum_acc(hi, lo, x[k].x);
+                two_sum_acc(hi, lo, x[k].y);
+                two_sum_acc(hi, lo, x[k].z);
+                two_sum_acc(hi, lo, x[k].w);
+            }
     }
     if (blockIdx.x == 0 && threadIdx.x < (int)(a.P & 3)) two_sum_acc(hi, lo, a.v[4 * nq + threadIdx.x]);
-    const double t = block_sum((double)hi + (double)lo, smem);
-    if (threadIdx.x == 0) a.partial[blockIdx.x] = t;
+    // Fixed float-float tree over the block (the fp64 pipe is narrow on this part).
+    float h, l;
+    two_sum(hi, lo, h, l);
+    ff_warp_sum(h, l);
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    if (lane == 0) smem[warp] = make_float2(h, l);
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        float2 t = make_float2(0.f, 0.f);
+        for (int w = 0; w < kMsgThreads / 32; ++w) ff_add(t.x, t.y, smem[w].x, smem[w].y);
+        a.partial[blockIdx.x] = t;
+    }
 }
 
 __global__ void __launch_bounds__(kMsgThreads) message_resolve_kernel(const __grid_constant__ MessageArgs a) {
     __shared__ uint32_t s_send;
     if (threadIdx.x < 32) {
         const int lane = threadIdx.x;
-        double s = 0.0;
-        for (int b = lane; b < a.nblocks; b += 32) s += a.partial[b];
+        float h = 0.f, l = 0.f;
+        // Lane l adds partials l, l + 32, ... in order, eight loads in flight.
+        for (int b = lane; b < a.nblocks; b += 8 * 32) {
+            float2 x[8];
 #pragma unroll
-        for (int off = 16; off > 0; off >>= 1) s += __shfl_xor_sync(kFull, s, off);
+            for (int k = 0; k < 8; ++k)
+                if (b + 32 * k < a.nblocks) x[k] = a.partial[b + 32 * k];
+#pragma unroll
+            for (int k = 0; k < 8; ++k)
+                if (b + 32 * k < a.nblocks) ff_add(h, l, x[k].x, x[k].y);
+        }
+        ff_warp_sum(h, l);
         if (lane == 0) {
-            const float vbar = (float)(s / (double)a.P);
+            const float vbar = ff_div_int(h, l, (int32_t)a.P);
             const Philox4 r = philox4x32_10(0xFFFFFFFFu, a.client_word, a.n_lo, a.n_hi,
                                             a.round_key0, a.round_key1);
             const uint32_t send = send_bit(r.x[0] >> 8, vbar, a.c, a.eps_b);

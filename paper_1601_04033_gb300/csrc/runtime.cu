@@ -24,6 +24,7 @@
 #include "eq9.cuh"
 #include "fasgd.h"
 #include "kernels.cuh"
+#include "message.cuh"
 #include "tensors.cuh"
 
 namespace {
@@ -134,7 +135,7 @@ struct fasgd_s {
     // floats, allocated by the first message push) and the partial sums.
     float* grad_cache = nullptr;
     int64_t cache_stride = 0;
-    double* msg_partial = nullptr;
+    float2* msg_partial = nullptr;
 
     // Per-tensor B-FASGD: the partition, its work items on the device, the
     // item sums of v and the decision of the latest call.
@@ -237,7 +238,7 @@ struct fasgd_s {
         cudaError_t st = cudaSuccess;
         if (msg_partial == nullptr)
             st = cudaMalloc(reinterpret_cast<void**>(&msg_partial),
-                            fasgd::kMessageMaxBlocks * sizeof(double));
+                            fasgd::kMessageMaxBlocks * sizeof(float2));
         if (st == cudaSuccess && cache && grad_cache == nullptr) {
             cache_stride = (P + 63) / 64 * 64;   // 256-byte aligned slots
             const size_t bytes = (size_t)lambda * (size_t)cache_stride * sizeof(float);

@@ -116,22 +116,6 @@ __device__ __forceinline__ uint64_t budget_term(int32_t size, float vbar, float 
     return shift > -64 ? prod >> (-shift) : 0;
 }
 
-// fl32((h + l) / s) for a float-float pair (h >= 0, |l| <= ulp(h)) and an
-// integer 1 <= s < 2^31, in fp32 only (the fp64 pipe is narrow here): with
-// sh = fl(s) and sl = s - sh (exact, |sl| <= 64), q0 = fl(h / sh) leaves the
-// residual h - q0 sh exactly representable (one fused multiply-add forms
-// it); adding l and subtracting q0 sl rounds terms some 2^-20 of ulp(q0)
-// small, so fl(q0 + r / sh) is the correctly rounded quotient except within
-// about 2^-43 (relative) of a rounding boundary.
-__device__ __forceinline__ float ff_div_int(float h, float l, int32_t s) {
-    const float sh = __int2float_rn(s);
-    const float sl = __ll2float_rn((long long)s - __float2ll_rn(sh));
-    const float q0 = __fdiv_rn(h, sh);
-    const float e1 = __fmaf_rn(-q0, sh, h);
-    const float r = __fsub_rn(__fadd_rn(e1, l), __fmul_rn(q0, sl));
-    return __fadd_rn(q0, __fdiv_rn(r, sh));
-}
-
 // Candidate k (0 .. 2^m - 2) of a search round inside the open interval
 // (lo, hi) of bit patterns: 2^m - 1 points cutting it into 2^m near-equal
 // parts (consecutive patterns once the interval is short); values >= hi are

@@ -1,6 +1,8 @@
 // Compensated fp32 summation shared by the mean-of-v reductions.
 #pragma once
 
+#include <stdint.h>
+
 namespace fasgd {
 
 // hi + lo += x, with the rounding error of the fp32 addition recovered
@@ -45,6 +47,22 @@ __device__ __forceinline__ void ff_warp_sum(float& h, float& l) {
         const float l2 = __shfl_xor_sync(0xffffffffu, l, off);
         ff_add(h, l, h2, l2);
     }
+}
+
+// fl32((h + l) / s) for a float-float pair (h >= 0, |l| <= ulp(h)) and an
+// integer 1 <= s < 2^31, in fp32 only (the fp64 pipe is narrow here): with
+// sh = fl(s) and sl = s - sh (exact, |sl| <= 64), q0 = fl(h / sh) leaves the
+// residual h - q0 sh exactly representable (one fused multiply-add forms
+// it); adding l and subtracting q0 sl rounds terms some 2^-20 of ulp(q0)
+// small, so fl(q0 + r / sh) is the correctly rounded quotient except within
+// about 2^-43 (relative) of a rounding boundary.
+__device__ __forceinline__ float ff_div_int(float h, float l, int32_t s) {
+    const float sh = __int2float_rn(s);
+    const float sl = __ll2float_rn((long long)s - __float2ll_rn(sh));
+    const float q0 = __fdiv_rn(h, sh);
+    const float e1 = __fmaf_rn(-q0, sh, h);
+    const float r = __fsub_rn(__fadd_rn(e1, l), __fmul_rn(q0, sl));
+    return __fadd_rn(q0, __fdiv_rn(r, sh));
 }
 
 }  // namespace fasgd
