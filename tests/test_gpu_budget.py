@@ -306,3 +306,35 @@ def test_full_size_25m_160_tensors():
     os_ = pair.o.state()
     compare_states([x[idx] for x in gs[:4]] + [gs[4]], [x[idx] for x in os_[:4]] + [os_[4]],
                    oracle.FASGD, "25M sampled")
+
+
+@pytest.mark.slow
+def test_size_2_28_64_tensors():
+    """P = 2^28 in 64 tensors (work items of 32,768 parameters, ~8,200 items):
+    three pushes at a 20 % budget and three fetches at 10 %, decisions and
+    counts exact, thresholds within 1e-5, the state on sampled parameters."""
+    torch = torch_cuda()
+    P = 1 << 28
+    sizes = streams.tensor_sizes(4, P, 64)
+    pair = Pair(P, sizes, pool_workload="fasgd-268m-k16", R=4)
+    ps = streams.push_stream(pair.w, 3, 1)
+    for t in range(3):
+        cl, js, sl = ps.batch(t)
+        got, want = pair.push(int(cl[0]), int(js[0]), int(sl[0]), int(0.2 * P))
+        pair.check_decision(got, want, f"2^28 push {t}", c_exact=False)
+        copy = torch.zeros(P, device="cuda")
+        pair.srv.fetch_budget(t % 4, copy, int(0.1 * P), pair.sent, pair.c, pair.count)
+        ocopy = np.zeros(P, np.float32)
+        fwant = pair.o.fetch_budget(t % 4, ocopy, int(0.1 * P))
+        pair.check_decision(pair.decision(), fwant, f"2^28 fetch {t}", c_exact=False)
+        idx = streams.sample_indices(P, 20_000, seed=t)
+        assert_close(copy.cpu().numpy()[idx], ocopy[idx], "2^28 fetched copy")
+        del copy
+    idx = torch.from_numpy(streams.sample_indices(P, 50_000)).cuda()
+    full = [torch.empty(P, device="cuda") for _ in range(4)]
+    T = pair.srv.get_state(*full)
+    gs = [x[idx].cpu().numpy() for x in full] + [T]
+    del full
+    ih = idx.cpu().numpy()
+    os_ = pair.o.state()
+    compare_states(gs, [x[ih] for x in os_[:4]] + [os_[4]], oracle.FASGD, "2^28 sampled")
