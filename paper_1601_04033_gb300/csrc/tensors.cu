@@ -19,7 +19,9 @@
 // apply re-forms the sums of the items it rewrote, in the partial kernel's
 // element order, so the item sums stay those of the current v and the next
 // decision skips the partial kernel (the host tracks when another pass has
-// changed v and the sums must be formed afresh).
+// changed v and the sums must be formed afresh).  All four are launched as
+// programmatic dependents (pdl.cuh), so each one's launch overlaps the tail
+// of the kernel before it.
 //
 // The threshold.  With a_t = fl(vbar_t + eps_b) and
 //   E(x) = sum_t floor(s_t * fl(a_t / fl(a_t + x)) * 2^32),
@@ -35,6 +37,7 @@
 
 #include "eq9.cuh"
 #include "kernels.cuh"
+#include "pdl.cuh"
 #include "tensors.cuh"
 #include "twosum.cuh"
 #include "update.cuh"
@@ -93,6 +96,8 @@ __device__ float2 item_v_sum(const TensorItem& it, const float* __restrict__ v, 
 
 __global__ void __launch_bounds__(kItemThreads) tensor_partial_kernel(const __grid_constant__ TensorArgs a) {
     __shared__ float2 smem[kItemThreads / 32];
+    pdl_wait();
+    pdl_trigger();
     for (int64_t i = blockIdx.x; i < a.n_items; i += gridDim.x) {
         const float2 sum = item_v_sum(a.items[i], a.v, smem);
         if (threadIdx.x == 0) a.partial[i] = sum;
@@ -154,6 +159,8 @@ __global__ void __launch_bounds__(kTensorResolveThreads) budget_resolve_kernel(c
     __shared__ long long s_lo, s_hi, s_cp;
     __shared__ unsigned long long s_count;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    pdl_wait();
+    pdl_trigger();
     // One pass of loads (every load of a thread issued before any store).
     const int nload = a.n_items > a.T + 1 ? a.n_items : a.T + 1;
     for (int i = tid; i < nload; i += kTensorResolveThreads) {
@@ -342,6 +349,8 @@ __global__ void __launch_bounds__(kItemThreads) tensor_apply_kernel(const __grid
     constexpr bool FAS = RULE != kRuleSgd;
     __shared__ float2 smem[kItemThreads / 32];
     const int tid = threadIdx.x;
+    pdl_wait();
+    pdl_trigger();
     for (int64_t i = blockIdx.x; i < a.n_items; i += gridDim.x) {
         const TensorItem it = a.items[i];
         if (!a.sent[it.tensor]) continue;
@@ -402,6 +411,8 @@ __global__ void __launch_bounds__(kItemThreads) tensor_apply_kernel(const __grid
 // thread in flight.
 __global__ void __launch_bounds__(kItemThreads) tensor_copy_kernel(const __grid_constant__ RangeArgs a) {
     const int tid = threadIdx.x;
+    pdl_wait();
+    pdl_trigger();
     for (int64_t i = blockIdx.x; i < a.n_items; i += gridDim.x) {
         const TensorItem it = a.items[i];
         if (!a.sent[it.tensor]) continue;
@@ -429,8 +440,8 @@ unsigned item_grid(int32_t n_items) { return (unsigned)(n_items > 0 ? n_items : 
 
 template <int RULE, int ARITH>
 cudaError_t launch_apply_rule(const RangeArgs& a, cudaStream_t stream) {
-    tensor_apply_kernel<RULE, ARITH><<<item_grid(a.n_items), kItemThreads, 0, stream>>>(a);
-    return cudaGetLastError();
+    return launch_pdl(tensor_apply_kernel<RULE, ARITH>, item_grid(a.n_items), kItemThreads, 0,
+                      stream, a);
 }
 
 }  // namespace
@@ -439,8 +450,7 @@ cudaError_t launch_tensor_decide(const TensorArgs& a, bool sums_valid, cudaStrea
                                  int64_t* launches) {
     cudaError_t st;
     if (!sums_valid) {
-        tensor_partial_kernel<<<item_grid(a.n_items), kItemThreads, 0, stream>>>(a);
-        st = cudaGetLastError();
+        st = launch_pdl(tensor_partial_kernel, item_grid(a.n_items), kItemThreads, 0, stream, a);
         if (st != cudaSuccess) return st;
         ++*launches;
     }
@@ -448,8 +458,7 @@ cudaError_t launch_tensor_decide(const TensorArgs& a, bool sums_valid, cudaStrea
     st = cudaFuncSetAttribute(budget_resolve_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                               (int)smem);
     if (st != cudaSuccess) return st;
-    budget_resolve_kernel<<<1, kTensorResolveThreads, smem, stream>>>(a);
-    st = cudaGetLastError();
+    st = launch_pdl(budget_resolve_kernel, 1, kTensorResolveThreads, smem, stream, a);
     if (st == cudaSuccess) ++*launches;
     return st;
 }
@@ -473,8 +482,7 @@ cudaError_t launch_tensor_apply(const RangeArgs& a, int rule, bool exact, cudaSt
 }
 
 cudaError_t launch_tensor_copy(const RangeArgs& a, cudaStream_t stream, int64_t* launches) {
-    tensor_copy_kernel<<<item_grid(a.n_items), kItemThreads, 0, stream>>>(a);
-    cudaError_t st = cudaGetLastError();
+    cudaError_t st = launch_pdl(tensor_copy_kernel, item_grid(a.n_items), kItemThreads, 0, stream, a);
     if (st == cudaSuccess) ++*launches;
     return st;
 }
