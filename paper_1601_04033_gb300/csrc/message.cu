@@ -22,6 +22,7 @@
 #include "eq9.cuh"
 #include "kernels.cuh"
 #include "message.cuh"
+#include "pdl.cuh"
 #include "twosum.cuh"
 
 namespace fasgd {
@@ -31,6 +32,8 @@ constexpr int kMsgThreads = 256;
 
 __global__ void __launch_bounds__(kMsgThreads) vbar_partial_kernel(const __grid_constant__ MessageArgs a) {
     __shared__ float2 smem[kMsgThreads / 32];
+    pdl_wait();
+    pdl_trigger();
     const int64_t nq = a.P >> 2;
     const int64_t chunk = (nq + a.nblocks - 1) / a.nblocks;
     const int64_t q0 = (int64_t)blockIdx.x * chunk;
@@ -70,6 +73,8 @@ __global__ void __launch_bounds__(kMsgThreads) vbar_partial_kernel(const __grid_
 
 __global__ void __launch_bounds__(kMsgThreads) message_resolve_kernel(const __grid_constant__ MessageArgs a) {
     __shared__ uint32_t s_send;
+    pdl_wait();
+    pdl_trigger();
     if (threadIdx.x < 32) {
         const int lane = threadIdx.x;
         float h = 0.f, l = 0.f;
@@ -115,16 +120,14 @@ int32_t message_partial_blocks(int64_t P) {
 
 cudaError_t launch_message(const MessageArgs& a, int num_sms, cudaStream_t stream,
                            int64_t* launches) {
-    vbar_partial_kernel<<<a.nblocks, kMsgThreads, 0, stream>>>(a);
-    cudaError_t st = cudaGetLastError();
+    cudaError_t st = launch_pdl(vbar_partial_kernel, a.nblocks, kMsgThreads, 0, stream, a);
     if (st != cudaSuccess) return st;
     ++*launches;
     int64_t grid = ((a.P >> 2) + kMsgThreads - 1) / kMsgThreads;
     const int64_t cap = (int64_t)(num_sms > 0 ? num_sms : 1) * 8;
     if (grid > cap) grid = cap;
     if (grid < 1) grid = 1;
-    message_resolve_kernel<<<(unsigned)grid, kMsgThreads, 0, stream>>>(a);
-    st = cudaGetLastError();
+    st = launch_pdl(message_resolve_kernel, (unsigned)grid, kMsgThreads, 0, stream, a);
     if (st != cudaSuccess) return st;
     ++*launches;
     return cudaSuccess;

@@ -20,6 +20,7 @@
 
 #include "eq9.cuh"
 #include "kernels.cuh"
+#include "pdl.cuh"
 
 namespace fasgd {
 namespace {
@@ -31,6 +32,8 @@ constexpr unsigned kFull = 0xffffffffu;
 
 __global__ void __launch_bounds__(kSelectThreads) bfasgd_mask_kernel(const __grid_constant__ SelectArgs a) {
     __shared__ int32_t warp_cnt[kWarps];
+    pdl_wait();
+    pdl_trigger();
     const int lane = threadIdx.x & 31;
     const int warp = threadIdx.x >> 5;
     const int64_t tile_start = (int64_t)blockIdx.x * kSelectTile;
@@ -88,6 +91,8 @@ constexpr int kScanThreads = 1024;
 
 __global__ void __launch_bounds__(kScanThreads) bfasgd_scan_kernel(const __grid_constant__ SelectArgs a) {
     __shared__ int64_t warp_sum[kScanThreads / 32];
+    pdl_wait();
+    pdl_trigger();
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int per = (a.ntiles + kScanThreads - 1) / kScanThreads;
     const int lo = tid * per;
@@ -123,6 +128,8 @@ __global__ void __launch_bounds__(kScanThreads) bfasgd_scan_kernel(const __grid_
 
 __global__ void __launch_bounds__(kSelectThreads) bfasgd_compact_kernel(const __grid_constant__ SelectArgs a) {
     __shared__ int32_t warp_cnt[kWarps];
+    pdl_wait();
+    pdl_trigger();
     const int lane = threadIdx.x & 31;
     const int warp = threadIdx.x >> 5;
     const int64_t tile_start = (int64_t)blockIdx.x * kSelectTile;
@@ -188,16 +195,13 @@ void select_key_schedule(SelectArgs& a, uint64_t seed) {
 }
 
 cudaError_t launch_select(const SelectArgs& a, cudaStream_t stream, int64_t* launches) {
-    bfasgd_mask_kernel<<<a.ntiles, kSelectThreads, 0, stream>>>(a);
-    cudaError_t st = cudaGetLastError();
+    cudaError_t st = launch_pdl(bfasgd_mask_kernel, a.ntiles, kSelectThreads, 0, stream, a);
     if (st != cudaSuccess) return st;
     ++*launches;
-    bfasgd_scan_kernel<<<1, kScanThreads, 0, stream>>>(a);
-    st = cudaGetLastError();
+    st = launch_pdl(bfasgd_scan_kernel, 1, kScanThreads, 0, stream, a);
     if (st != cudaSuccess) return st;
     ++*launches;
-    bfasgd_compact_kernel<<<a.ntiles, kSelectThreads, 0, stream>>>(a);
-    st = cudaGetLastError();
+    st = launch_pdl(bfasgd_compact_kernel, a.ntiles, kSelectThreads, 0, stream, a);
     if (st != cudaSuccess) return st;
     ++*launches;
     return cudaSuccess;

@@ -12,6 +12,7 @@
 // flight per thread.
 
 #include "kernels.cuh"
+#include "pdl.cuh"
 #include "update.cuh"
 
 namespace fasgd {
@@ -23,6 +24,8 @@ constexpr int kUnroll = 4;
 template <int RULE, bool EXACT>
 __global__ void __launch_bounds__(kSparseThreads) fasgd_sparse_kernel(const __grid_constant__ SparseArgs a) {
     constexpr bool FAS = RULE != kRuleSgd;
+    pdl_wait();
+    pdl_trigger();
     int64_t count = a.count_max;
     if (a.count_dev != nullptr) {
         const int64_t c = *a.count_dev;
@@ -103,14 +106,15 @@ cudaError_t launch_rule(const SparseArgs& a, int num_sms, cudaStream_t stream) {
     const int64_t cap = (int64_t)num_sms * blocks_per_sm;
     if (want > cap) want = cap;
     if (want < 1) want = 1;
-    fasgd_sparse_kernel<RULE, EXACT><<<(unsigned)want, kSparseThreads, 0, stream>>>(a);
-    return cudaGetLastError();
+    return launch_pdl(fasgd_sparse_kernel<RULE, EXACT>, (unsigned)want, kSparseThreads, 0, stream, a);
 }
 
 // Client side of a B-FASGD fetch: theta[idx[i]] = val[i] for i < count.
 // Indices come from one compaction, so they are distinct and no two threads
 // write the same parameter; an index outside [0, P) is skipped and flagged.
 __global__ void __launch_bounds__(kSparseThreads) fetch_scatter_kernel(const __grid_constant__ ScatterArgs a) {
+    pdl_wait();
+    pdl_trigger();
     int64_t count = a.count_max;
     if (a.count_dev != nullptr) {
         const int64_t c = *a.count_dev;
@@ -138,8 +142,7 @@ cudaError_t launch_scatter(const ScatterArgs& a, int num_sms, cudaStream_t strea
     const int64_t cap = (int64_t)(num_sms > 0 ? num_sms : 1) * 8;
     if (want > cap) want = cap;
     if (want < 1) want = 1;
-    fetch_scatter_kernel<<<(unsigned)want, kSparseThreads, 0, stream>>>(a);
-    return cudaGetLastError();
+    return launch_pdl(fetch_scatter_kernel, (unsigned)want, kSparseThreads, 0, stream, a);
 }
 
 cudaError_t launch_sparse(const SparseArgs& a, int rule, bool exact, int num_sms,
