@@ -568,15 +568,17 @@ def run_message(args, w, world, rank, local):
     srv.close()
     step_s = total_ms / 1e3 / args.steps
     peak, peak_kind = peaks()
-    # A push: vbar read (4 B), the cache refresh when sent (8 B), the dense
-    # K=1 pass over the cache slot (36 B); per parameter.
-    push_bytes = P * (4 + 8 * s_frac + 36)
+    # A push: the cache refresh when sent (8 B per parameter) and the dense
+    # K = 1 pass over the cache slot (36 B per parameter); the statistic
+    # comes from chunk sums the previous pass left (8 B read + 8 B written
+    # per 128 parameters), not from a pass over v.
+    push_bytes = P * (8 * s_frac + 36) + 16 * ((P + 127) // 128)
     achieved = push_bytes / (push_ms / 1e3) / 1e9
     return {
         "value": P * world / step_s, "ms_per_step": total_ms / args.steps,
         "roofline": {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
                      "frac": round(achieved / peak, 4), "peak_source": peak_kind,
-                     "kernel": "message push (vbar + cache refresh + dense pass)",
+                     "kernel": "message push (decision + cache refresh + dense pass)",
                      "bytes_per_launch": push_bytes, "launch_ms": round(push_ms, 5),
                      "traffic": None, "fetch_ms": round(fetch_ms, 5)},
         "clocks": clock_info, "e2e": None, "gpu_launches": launches,

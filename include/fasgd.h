@@ -269,6 +269,15 @@ FASGD_API int bfasgd_fetch_message(fasgd_t* h, int32_t client, float* theta_clie
                                    int32_t* fetched_dev);
 
 /*
+ * bfasgd_message_vbar -- the statistic the per-message decision would use
+ * now: vbar = the mean of the server's v over all P parameters (a
+ * compensated sum in a fixed order, rounded once to fp32), written to
+ * vbar_dev (device float) on the handle's stream.  No draw is consumed and
+ * no counter advances.  Errors: EINVAL, ENOMEM, ECUDA.
+ */
+FASGD_API int bfasgd_message_vbar(fasgd_t* h, float* vbar_dev);
+
+/*
  * Per-tensor B-FASGD under a bandwidth budget (Sec. 5, future work: decide
  * per tensor, and spread a fixed bandwidth budget over the tensors by their
  * statistics).  The paper gives no formula; the reading implemented:

@@ -19,12 +19,18 @@
 // several stages per tile (the state travels with the first one only).  The
 // last P mod 2048 parameters are handled by plain loads in the last block.
 //
+// With SUMS (one push, a.vsum set) the pass also leaves the float-float sum
+// of the new v over every 128-parameter chunk (one warp's share of a tile)
+// in a.vsum, formed in registers, so the next per-message decision needs no
+// pass over v (message.cu forms the same chunk sums from v, bit for bit).
+//
 // Every wait on an mbarrier is bounded (about one second of wall clock);
 // on expiry the block sets flag 8 of the error word, waits (bounded) for its
 // own copies in flight, and returns.  Elements are independent, so the
 // result does not depend on the grid or on which path handled an element.
 
 #include "kernels.cuh"
+#include "twosum.cuh"
 #include "update.cuh"
 
 namespace fasgd {
@@ -171,6 +177,46 @@ __device__ void apply_range_direct(const DenseArgs& a, int64_t begin, int tid) {
     }
 }
 
+// The SUMS form of the tail: parameters [begin, P) chunk by chunk, consumer
+// warp w taking chunks begin/128 + w, + 16, ...; lane l updates parameters
+// 4l .. 4l + 3 of the chunk (guarded at P) and the warp forms the chunk's sum
+// of the new v in registers.  begin is a multiple of 2048.
+template <int RULE, int ARITH>
+__device__ void apply_range_chunks(const DenseArgs& a, int64_t begin, int tid) {
+    const int warp = tid >> 5, lane = tid & 31;
+    const int64_t nch = (a.P + kVsumChunk - 1) / kVsumChunk;
+    for (int64_t c = begin / kVsumChunk + warp; c < nch; c += kConsumers / 32) {
+        const int64_t e = c * kVsumChunk + 4 * lane;
+        float th[4] = {0.f, 0.f, 0.f, 0.f}, n[4] = {0.f, 0.f, 0.f, 0.f};
+        float b[4] = {0.f, 0.f, 0.f, 0.f}, v[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+        for (int j = 0; j < 4; ++j)
+            if (e + j < a.P) {
+                th[j] = a.theta[e + j];
+                n[j] = a.n[e + j];
+                b[j] = a.b[e + j];
+                v[j] = a.v[e + j];
+            }
+        for (int k = 0; k < a.K; ++k)
+#pragma unroll
+            for (int j = 0; j < 4; ++j)
+                if (e + j < a.P)
+                    rule_update<ARITH, RULE == kRuleFasgdStd>(th[j], n[j], b[j], v[j],
+                                                              __ldcs(a.grad[k] + e + j),
+                                                              a.coef[k], a.sp);
+#pragma unroll
+        for (int j = 0; j < 4; ++j)
+            if (e + j < a.P) {
+                a.theta[e + j] = th[j];
+                a.n[e + j] = n[j];
+                a.b[e + j] = b[j];
+                a.v[e + j] = v[j];
+            }
+        const float2 cs = chunk_sum4(make_float4(v[0], v[1], v[2], v[3]));
+        if (lane == 0) a.vsum[c] = cs;
+    }
+}
+
 // Ring geometry, identical on host and device.
 struct Ring {
     int stages;     // stages in the ring
@@ -178,8 +224,9 @@ struct Ring {
 };
 
 // RULE: kRuleSgd / kRuleFasgd / kRuleFasgdStd; ARITH: kArithApprox /
-// kArithApproxFtz / kArithExact (see update.cuh); CH: gradient slices per stage.
-template <int RULE, int ARITH, int CH>
+// kArithApproxFtz / kArithExact (see update.cuh); CH: gradient slices per stage;
+// SUMS: also leave the chunk sums of the new v (FASGD rules, K = 1).
+template <int RULE, int ARITH, int CH, bool SUMS>
 __global__ void __launch_bounds__(kThreads, 1)
 fasgd_dense_kernel(const __grid_constant__ DenseArgs a, const Ring ring, const int64_t ntiles) {
     constexpr bool FAS = RULE != kRuleSgd;
@@ -298,12 +345,21 @@ fasgd_dense_kernel(const __grid_constant__ DenseArgs a, const Ring ring, const i
             *reinterpret_cast<float4*>(a.b + e) = b;
             *reinterpret_cast<float4*>(a.v + e) = v;
         }
+        if (SUMS) {
+            const float2 cs = chunk_sum4(v);
+            if (lane == 0) a.vsum[(t * kTile) / kVsumChunk + warp] = cs;
+        }
     }
     // Parameters after the last full tile.
-    if (ok && blockIdx.x == gridDim.x - 1) apply_range_direct<RULE, ARITH>(a, ntiles * kTile, tid);
+    if (ok && blockIdx.x == gridDim.x - 1) {
+        if (SUMS)
+            apply_range_chunks<RULE, ARITH>(a, ntiles * kTile, tid);
+        else
+            apply_range_direct<RULE, ARITH>(a, ntiles * kTile, tid);
+    }
 }
 
-template <int RULE, int ARITH, int CH>
+template <int RULE, int ARITH, int CH, bool SUMS = false>
 cudaError_t launch_ch(const DenseArgs& a, int num_sms, cudaStream_t stream) {
     constexpr int kState = RULE != kRuleSgd ? 4 : 1;
     constexpr int kStageBytes = (kState + CH) * kTile * 4;
@@ -314,7 +370,7 @@ cudaError_t launch_ch(const DenseArgs& a, int num_sms, cudaStream_t stream) {
     const size_t smem = (size_t)ring.stages * kStageBytes + 2 * ring.stages * sizeof(uint64_t);
     static bool configured = false;  // per instantiation
     if (!configured) {
-        cudaError_t st = cudaFuncSetAttribute(fasgd_dense_kernel<RULE, ARITH, CH>,
+        cudaError_t st = cudaFuncSetAttribute(fasgd_dense_kernel<RULE, ARITH, CH, SUMS>,
                                               cudaFuncAttributeMaxDynamicSharedMemorySize,
                                               kSmemBudget);
         if (st != cudaSuccess) return st;
@@ -323,12 +379,18 @@ cudaError_t launch_ch(const DenseArgs& a, int num_sms, cudaStream_t stream) {
     const int64_t ntiles = a.P / kTile;
     int64_t grid = ntiles < num_sms ? ntiles : num_sms;  // one block per SM (shared-memory bound)
     if (grid < 1) grid = 1;
-    fasgd_dense_kernel<RULE, ARITH, CH><<<(unsigned)grid, kThreads, smem, stream>>>(a, ring, ntiles);
+    fasgd_dense_kernel<RULE, ARITH, CH, SUMS><<<(unsigned)grid, kThreads, smem, stream>>>(a, ring, ntiles);
     return cudaGetLastError();
 }
 
 template <int RULE, int ARITH>
 cudaError_t launch_rule(const DenseArgs& a, int num_sms, cudaStream_t stream) {
+    if constexpr (RULE != kRuleSgd) {
+        if (a.vsum != nullptr) {
+            if (a.K != 1) return cudaErrorInvalidValue;
+            return launch_ch<RULE, ARITH, 1, true>(a, num_sms, stream);
+        }
+    }
     // Gradient slices per stage: K rounded up to a power of two, at most 8.
     if (a.K > 4) return launch_ch<RULE, ARITH, 8>(a, num_sms, stream);
     if (a.K > 2) return launch_ch<RULE, ARITH, 4>(a, num_sms, stream);

@@ -34,7 +34,11 @@ struct DenseArgs {
     int32_t K;
     StatParams sp;
     int32_t* err;                   // device error flags (bit 3: a pipeline wait expired)
+    float2* vsum;                   // if set (K = 1, FASGD rules): the float-float sum of
+                                    // the new v over every 128-parameter chunk
 };
+// Parameters per chunk of the per-message statistic's partial sums.
+constexpr int kVsumChunk = 128;
 
 // One sparse push: idx[i] receives val[i] for i < count.
 struct SparseArgs {

@@ -3,10 +3,12 @@
 // of the server's moving averages.
 //
 // Two kernels per decision:
-//   1. vbar_partial: fixed partition of the parameters into contiguous
-//      chunks, one per block; each block sums its chunk of v (fixed order: per
-//      thread in index order as an fp32 sum plus its exact rounding errors,
-//      then a fixed float-float tree) into one float-float partial;
+//   1. vbar_partial: the parameters are cut into 128-parameter chunks and
+//      the chunks into one contiguous range per block; each block combines
+//      its chunks' float-float sums in a fixed order into one partial.  The
+//      chunk sums are those the dense pass leaves after a message push (so
+//      v is not read again), or, when another pass has changed v since, the
+//      block forms them from v with the same arithmetic and stores them;
 //   2. message_resolve: every block adds the partials in the same fixed order
 //      (float-float), forms vbar = fl32(sum / P) (ff_div_int), draws u
 //      (Philox4x32-10, word 0 at counter
@@ -30,43 +32,71 @@ namespace {
 
 constexpr int kMsgThreads = 256;
 
+// This lane's four values of chunk c of v (parameters 4 lane .. 4 lane + 3
+// of the chunk), zeros past P.  chunk_sum4 over them gives the same bits the
+// dense pass leaves for the chunk.
+__device__ __forceinline__ float4 chunk_values(const float* v, int64_t P, int64_t c, int lane) {
+    const int64_t e = c * kVsumChunk + 4 * lane;
+    if (e + 3 < P) return __ldcs(reinterpret_cast<const float4*>(v + e));
+    float4 x;
+    x.x = e < P ? v[e] : 0.f;
+    x.y = e + 1 < P ? v[e + 1] : 0.f;
+    x.z = e + 2 < P ? v[e + 2] : 0.f;
+    x.w = e + 3 < P ? v[e + 3] : 0.f;
+    return x;
+}
+
+// Block b combines chunks [c0, c1) in a fixed order: chunk c0 + w + 8 i goes
+// to warp w, slot i, and lane (i mod 32) of that warp adds its slots in
+// increasing i; then each warp's tree, then the warps in order.  from_v: the
+// warp forms each chunk sum from v (four chunks' loads in flight) and stores
+// it; otherwise lane l loads its slots' stored sums.  Both give the same bits.
 __global__ void __launch_bounds__(kMsgThreads) vbar_partial_kernel(const __grid_constant__ MessageArgs a) {
     __shared__ float2 smem[kMsgThreads / 32];
     pdl_wait();
     pdl_trigger();
-    const int64_t nq = a.P >> 2;
-    const int64_t chunk = (nq + a.nblocks - 1) / a.nblocks;
-    const int64_t q0 = (int64_t)blockIdx.x * chunk;
-    const int64_t q1 = q0 + chunk < nq ? q0 + chunk : nq;
-    // Per thread: an fp32 sum with its exact rounding error carried alongside
-    // (Knuth's TwoSum), four quads loaded before they are added.
-    float hi = 0.f, lo = 0.f;
-    const float4* v4 = reinterpret_cast<const float4*>(a.v);
-    for (int64_t q = q0 + threadIdx.x; q < q1; q += 4 * kMsgThreads) {
-        float4 x[4];
-#pragma unroll
-        for (int k = 0; k < 4; ++k)
-            if (q + k * kMsgThreads < q1) x[k] = __ldcs(v4 + q + k * kMsgThreads);
-#pragma unroll
-        for (int k = 0; k < 4; ++k)
-            if (q + k * kMsgThreads < q1) {
-                two_sum_acc(hi, lo, x[k].x);
-                two_sum_acc(hi, lo, x[k].y);
-                two_sum_acc(hi, lo, x[k].z);
-                two_sum_acc(hi, lo, x[k].w);
-            }
-    }
-    if (blockIdx.x == 0 && threadIdx.x < (int)(a.P & 3)) two_sum_acc(hi, lo, a.v[4 * nq + threadIdx.x]);
-    // Fixed float-float tree over the block (the fp64 pipe is narrow on this part).
-    float h, l;
-    two_sum(hi, lo, h, l);
-    ff_warp_sum(h, l);
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    constexpr int kWarps = kMsgThreads / 32;
+    const int64_t nch = (a.P + kVsumChunk - 1) / kVsumChunk;
+    const int64_t per = (nch + a.nblocks - 1) / a.nblocks;
+    const int64_t c0 = (int64_t)blockIdx.x * per;
+    const int64_t c1 = c0 + per < nch ? c0 + per : nch;
+    const int64_t nslots = c1 > c0 + warp ? (c1 - c0 - warp + kWarps - 1) / kWarps : 0;
+    float h = 0.f, l = 0.f;
+    if (a.from_v) {
+        for (int64_t i0 = 0; i0 < nslots; i0 += 4) {
+            float4 x[4];
+#pragma unroll
+            for (int k = 0; k < 4; ++k)
+                if (i0 + k < nslots) x[k] = chunk_values(a.v, a.P, c0 + warp + kWarps * (i0 + k), lane);
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+                const int64_t i = i0 + k;
+                if (i < nslots) {   // warp-uniform: the tree below uses every lane
+                    const int64_t c = c0 + warp + kWarps * i;
+                    const float2 cs = chunk_sum4(x[k]);
+                    if (lane == 0) a.chunks[c] = cs;
+                    if (lane == (int)(i & 31)) ff_add(h, l, cs.x, cs.y);
+                }
+            }
+        }
+    } else {
+        for (int64_t i0 = lane; i0 < nslots; i0 += 4 * 32) {
+            float2 x[4];
+#pragma unroll
+            for (int k = 0; k < 4; ++k)
+                if (i0 + 32 * k < nslots) x[k] = a.chunks[c0 + warp + kWarps * (i0 + 32 * k)];
+#pragma unroll
+            for (int k = 0; k < 4; ++k)
+                if (i0 + 32 * k < nslots) ff_add(h, l, x[k].x, x[k].y);
+        }
+    }
+    ff_warp_sum(h, l);
     if (lane == 0) smem[warp] = make_float2(h, l);
     __syncthreads();
     if (threadIdx.x == 0) {
         float2 t = make_float2(0.f, 0.f);
-        for (int w = 0; w < kMsgThreads / 32; ++w) ff_add(t.x, t.y, smem[w].x, smem[w].y);
+        for (int w = 0; w < kWarps; ++w) ff_add(t.x, t.y, smem[w].x, smem[w].y);
         a.partial[blockIdx.x] = t;
     }
 }
@@ -96,6 +126,7 @@ __global__ void __launch_bounds__(kMsgThreads) message_resolve_kernel(const __gr
             const uint32_t send = send_bit(r.x[0] >> 8, vbar, a.c, a.eps_b);
             s_send = send;
             if (blockIdx.x == 0 && a.flag_out != nullptr) *a.flag_out = (int32_t)send;
+            if (blockIdx.x == 0 && a.vbar_out != nullptr) *a.vbar_out = vbar;
         }
     }
     __syncthreads();
@@ -111,8 +142,8 @@ __global__ void __launch_bounds__(kMsgThreads) message_resolve_kernel(const __gr
 }  // namespace
 
 int32_t message_partial_blocks(int64_t P) {
-    const int64_t nq = P >> 2;
-    int64_t b = (nq + 8191) / 8192;  // ~8192 quads per block
+    const int64_t nch = (P + kVsumChunk - 1) / kVsumChunk;
+    int64_t b = (nch + 255) / 256;   // ~256 chunks (32,768 parameters) per block
     if (b < 1) b = 1;
     if (b > kMessageMaxBlocks) b = kMessageMaxBlocks;
     return (int32_t)b;

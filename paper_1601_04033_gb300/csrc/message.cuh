@@ -14,6 +14,9 @@ struct MessageArgs {
     int64_t P;
     float2* partial;           // scratch: nblocks float-float partial sums
     int32_t nblocks;           // message_partial_blocks(P)
+    float2* chunks;            // ceil(P / 128) chunk sums of v
+    int32_t from_v;            // 1: form the chunk sums from v (and store them);
+                               // 0: they are current (left by the dense pass)
     float c;                   // c_push or c_fetch
     float eps_b;
     uint32_t round_key0[10];
@@ -23,6 +26,7 @@ struct MessageArgs {
     const float* src;          // may be null: decide only
     float* dst;
     int32_t* flag_out;         // may be null: 1 transmitted, 0 dropped
+    float* vbar_out;           // may be null: the statistic vbar the decision used
 };
 
 int32_t message_partial_blocks(int64_t P);

@@ -136,6 +136,8 @@ struct fasgd_s {
     float* grad_cache = nullptr;
     int64_t cache_stride = 0;
     float2* msg_partial = nullptr;
+    float2* msg_chunks = nullptr;   // chunk sums of v (128 parameters each)
+    bool msg_sums_valid = false;    // msg_chunks holds those of the current v
 
     // Per-tensor B-FASGD: the partition, its work items on the device, the
     // item sums of v and the decision of the latest call.
@@ -239,6 +241,11 @@ struct fasgd_s {
         if (msg_partial == nullptr)
             st = cudaMalloc(reinterpret_cast<void**>(&msg_partial),
                             fasgd::kMessageMaxBlocks * sizeof(float2));
+        if (st == cudaSuccess && msg_chunks == nullptr) {
+            st = cudaMalloc(reinterpret_cast<void**>(&msg_chunks),
+                            (size_t)((P + fasgd::kVsumChunk - 1) / fasgd::kVsumChunk) * sizeof(float2));
+            msg_sums_valid = false;
+        }
         if (st == cudaSuccess && cache && grad_cache == nullptr) {
             cache_stride = (P + 63) / 64 * 64;   // 256-byte aligned slots
             const size_t bytes = (size_t)lambda * (size_t)cache_stride * sizeof(float);
@@ -255,25 +262,32 @@ struct fasgd_s {
     // One per-message decision of `stream_id` for `client` (advancing its
     // counter), copying src -> dst if transmitted.
     cudaError_t launch_message(uint32_t stream_id, int32_t client, const float* src, float* dst,
-                               int32_t* flag, float c, std::vector<uint64_t>& counter) {
+                               int32_t* flag, float c, std::vector<uint64_t>* counter,
+                               float* vbar_out = nullptr) {
         fasgd::MessageArgs a;
         std::memset(&a, 0, sizeof a);
         a.v = v;
         a.P = P;
         a.partial = msg_partial;
         a.nblocks = fasgd::message_partial_blocks(P);
+        a.chunks = msg_chunks;
+        a.from_v = msg_sums_valid ? 0 : 1;
         a.c = c;
         a.eps_b = eps_b;
         fasgd::philox_key_schedule(seed, a.round_key0, a.round_key1);
-        const uint64_t n = counter[(size_t)client];
+        const uint64_t n = counter != nullptr ? (*counter)[(size_t)client] : 0;
         a.client_word = (uint32_t)client | (stream_id << 31);
         a.n_lo = (uint32_t)n;
         a.n_hi = (uint32_t)(n >> 32);
         a.src = src;
         a.dst = dst;
         a.flag_out = flag;
+        a.vbar_out = vbar_out;
         cudaError_t st = fasgd::launch_message(a, num_sms, stream, &launches);
-        if (st == cudaSuccess) counter[(size_t)client] = n + 1;
+        if (st == cudaSuccess) {
+            msg_sums_valid = true;
+            if (counter != nullptr) (*counter)[(size_t)client] = n + 1;
+        }
         return st;
     }
 
@@ -314,6 +328,9 @@ struct fasgd_s {
         cudaFree(dev_err);
         cudaFree(grad_cache);
         cudaFree(msg_partial);
+        cudaFree(msg_chunks);
+        msg_chunks = nullptr;
+        msg_sums_valid = false;
         grad_cache = nullptr;
         msg_partial = nullptr;
         free_tensors();
@@ -553,7 +570,7 @@ int bfasgd_fetch_message(fasgd_t* h, int32_t client, float* theta_client, int32_
     cudaError_t st = h->ensure_message_scratch(false);
     if (st == cudaSuccess)
         st = h->launch_message(1, client, h->theta, theta_client, fetched_dev, h->c_fetch,
-                               h->fetch_count);
+                               &h->fetch_count);
     if (st != cudaSuccess) return h->cuda_fail(st, "bfasgd_fetch_message");
     return FASGD_OK;
 }
@@ -657,6 +674,18 @@ int bfasgd_fetch_budget(fasgd_t* h, int32_t client, float* theta_client, int64_t
     return FASGD_OK;
 }
 
+int bfasgd_message_vbar(fasgd_t* h, float* vbar_dev) {
+    if (h == nullptr) return FASGD_EINVAL;
+    if (vbar_dev == nullptr || !aligned(vbar_dev, 4))
+        return h->fail(FASGD_EINVAL, "vbar_dev must be a non-NULL 4-byte aligned device pointer");
+    DeviceGuard g(h->device);
+    cudaError_t st = h->ensure_message_scratch(false);
+    if (st == cudaSuccess)
+        st = h->launch_message(0, 0, nullptr, nullptr, nullptr, h->c_push, nullptr, vbar_dev);
+    if (st != cudaSuccess) return h->cuda_fail(st, "bfasgd_message_vbar");
+    return FASGD_OK;
+}
+
 int fasgd_push_sparse(fasgd_t* h, int32_t client, int64_t timestamp, const int32_t* idx,
                       const float* val, const int64_t* n_dev, int64_t n_max) {
     if (h == nullptr) return FASGD_EINVAL;
@@ -685,6 +714,7 @@ int fasgd_apply_pending(fasgd_t* h, int32_t K) {
     while (k < K) {
         const Push& first = h->fifo[(size_t)k];
         if (first.kind != kBudget) h->t_sums_valid = false;   // this pass rewrites v
+        if (first.kind != kMessage) h->msg_sums_valid = false;
         if (first.kind == kDense) {
             // Fuse the run of consecutive dense pushes into one pass.
             fasgd::DenseArgs a;
@@ -724,7 +754,7 @@ int fasgd_apply_pending(fasgd_t* h, int32_t K) {
             // slot if the push is transmitted, then apply the slot.
             float* slot = h->grad_cache + (size_t)first.client * (size_t)h->cache_stride;
             cudaError_t st = h->launch_message(0, first.client, first.grad, slot, first.flag,
-                                               h->c_push, h->push_count);
+                                               h->c_push, &h->push_count);
             if (st == cudaSuccess) {
                 fasgd::DenseArgs a;
                 std::memset(&a, 0, sizeof a);
@@ -738,7 +768,9 @@ int fasgd_apply_pending(fasgd_t* h, int32_t K) {
                 a.grad[0] = slot;
                 a.coef[0] = h->coef(h->T + k - first.j);
                 a.K = 1;
+                if (rule != fasgd::kRuleSgd) a.vsum = h->msg_chunks;   // keep the chunk sums current
                 st = fasgd::launch_dense(a, rule, h->exact, h->num_sms, h->stream, &h->launches);
+                h->msg_sums_valid = st == cudaSuccess;
             }
             if (st != cudaSuccess) return h->cuda_fail(st, "fasgd_apply_pending: message push");
             k += 1;
@@ -996,7 +1028,10 @@ int fasgd_set_state(fasgd_t* h, const float* theta, const float* n, const float*
         if (st != cudaSuccess) return h->cuda_fail(st, "fasgd_set_state");
     }
     h->T = T;
-    if (v != nullptr) h->t_sums_valid = false;
+    if (v != nullptr) {
+        h->t_sums_valid = false;
+        h->msg_sums_valid = false;
+    }
     return FASGD_OK;
 }
 

@@ -49,6 +49,23 @@ __device__ __forceinline__ void ff_warp_sum(float& h, float& l) {
     }
 }
 
+// The sum of one 128-parameter chunk of v, as a float-float pair, from this
+// lane's four consecutive values (lane l holds parameters 4l .. 4l + 3 of the
+// chunk; values past the end are passed as 0, which adds nothing): TwoSum in
+// the order x, y, z, w, renormalised, then the fixed warp tree.  Every lane
+// ends with the same pair; the bits depend only on the values.
+__device__ __forceinline__ float2 chunk_sum4(float4 v) {
+    float hi = 0.f, lo = 0.f;
+    two_sum_acc(hi, lo, v.x);
+    two_sum_acc(hi, lo, v.y);
+    two_sum_acc(hi, lo, v.z);
+    two_sum_acc(hi, lo, v.w);
+    float h, l;
+    two_sum(hi, lo, h, l);
+    ff_warp_sum(h, l);
+    return make_float2(h, l);
+}
+
 // fl32((h + l) / s) for a float-float pair (h >= 0, |l| <= ulp(h)) and an
 // integer 1 <= s < 2^31, in fp32 only (the fp64 pipe is narrow here): with
 // sh = fl(s) and sl = s - sh (exact, |sl| <= 64), q0 = fl(h / sh) leaves the

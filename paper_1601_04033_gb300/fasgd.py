@@ -55,6 +55,7 @@ SIGNATURES = {
     "fasgd_set_fetch_counts": (_i32, [_p, _p]),
     "bfasgd_push_message": (_i32, [_p, _i32, _i64, _p, _p]),
     "bfasgd_fetch_message": (_i32, [_p, _i32, _p, _p]),
+    "bfasgd_message_vbar": (_i32, [_p, _p]),
     "bfasgd_set_tensors": (_i32, [_p, _i32, _p]),
     "bfasgd_push_budget": (_i32, [_p, _i32, _i64, _p, _i64, _p, _p, _p]),
     "bfasgd_fetch_budget": (_i32, [_p, _i32, _p, _i64, _p, _p, _p]),
@@ -167,6 +168,10 @@ def bfasgd_push_message(h, client, timestamp, grad, sent_dev):
 
 def bfasgd_fetch_message(h, client, theta_client, fetched_dev):
     return LIB.bfasgd_fetch_message(h, client, theta_client, fetched_dev)
+
+
+def bfasgd_message_vbar(h, vbar_dev):
+    return LIB.bfasgd_message_vbar(h, vbar_dev)
 
 
 def bfasgd_set_tensors(h, T, sizes):
@@ -356,6 +361,14 @@ class Server:
 
     def fetch_message(self, client: int, theta_client, fetched_dev=None):
         self._check(bfasgd_fetch_message(self.h, client, _ptr(theta_client), _ptr(fetched_dev)))
+
+    def message_vbar(self, vbar_dev=None):
+        """The per-message statistic (mean of v) now: written to vbar_dev if
+        given (returns None), else returned as a float (synchronises)."""
+        import torch
+        out = vbar_dev if vbar_dev is not None else torch.empty(1, device="cuda")
+        self._check(bfasgd_message_vbar(self.h, _ptr(out)))
+        return None if vbar_dev is not None else float(out.item())
 
     def set_tensors(self, sizes):
         """Partition theta into contiguous tensors (sizes: ints summing to P)."""

@@ -97,3 +97,32 @@ def test_fetch_messages_against_oracle():
             assert int(flag.item()) == int(ok), (c, k)
             assert_bitwise(gcopy.cpu().numpy(), ocopy, f"fetched copy c={c} k={k}")
     assert list(srv.fetch_counts()) == o.fetch_count
+
+
+@pytest.mark.parametrize("P", [5, 2048 * 3 + 129, 100_003, 300_000])
+def test_statistic_kept_by_the_dense_pass_equals_a_fresh_sum(P):
+    """After a message push the dense pass leaves the chunk sums of the new v;
+    the statistic formed from them equals, bit for bit, the one formed afresh
+    from v (after set_state, which discards the kept sums), and equals the
+    oracle's mean of v.  Sizes cover the dense pass's tail (P mod 2048, 128, 4)."""
+    import torch
+    from paper_1601_04033_gb300 import fasgd
+    w = streams.WORKLOADS["fasgd-1.29m"].replace(lam=3, R=4)
+    pool = streams.gradient_pool(w, P)
+    srv = fasgd.Server(P, 3, w.alpha, fasgd.FASGD, c_push=1.0, seed=SEED)
+    srv.set_params(torch.from_numpy(streams.theta0(w, P)).cuda())
+    _, dpool = fasgd.aligned_vectors(pool)
+    state = [torch.empty(P, device="cuda") for _ in range(4)]
+    for t in range(6):
+        if t == 3:                      # a fused dense pass in between (it discards the sums)
+            srv.push(0, srv.T, dpool[1])
+            srv.push(1, srv.T, dpool[2])
+            srv.apply_pending(2)
+        srv.push_message(t % 3, srv.T, dpool[t % 4])
+        srv.apply_pending(1)
+        kept = srv.message_vbar()
+        T = srv.get_state(*state)
+        srv.set_state(*state, T)
+        fresh = srv.message_vbar()
+        assert np.float32(kept).view(np.uint32) == np.float32(fresh).view(np.uint32), (t, kept, fresh)
+        assert fresh == oracle.mean_v(state[3].cpu().numpy()), (t, fresh)
