@@ -15,11 +15,15 @@ from . import OracleServer, fetch_apply, sim_grad, sim_loss
 
 class OracleSimulation:
     def __init__(self, P, lam, alpha, variant, *, gamma=0.95, beta=0.95, eps=1e-4, seed=0,
-                 fetch="full", c_fetch=0.0, objective, theta0, lib=None):
+                 fetch="full", c_fetch=0.0, objective, theta0, lib=None, eps_b=1e-8,
+                 tensor_sizes=None, fetch_budget=None, push_budget=None):
         self.P, self.lam, self.seed, self.fetch = P, lam, seed, fetch
         self.lib = lib
         self.srv = OracleServer(P, lam, alpha, variant, gamma=gamma, beta=beta, eps=eps, seed=seed,
-                                lib=lib)
+                                eps_b=eps_b, lib=lib)
+        if tensor_sizes is not None:
+            self.srv.set_tensors(tensor_sizes)
+        self.fetch_budget, self.push_budget = fetch_budget, push_budget
         self.srv.set_fetch_threshold(c_fetch)
         self.srv.set_params(theta0)
         self.h, self.star, self.sigma = [np.ascontiguousarray(x, np.float32) for x in objective]
@@ -36,8 +40,13 @@ class OracleSimulation:
             g = sim_grad(self.clients[c], self.h, self.star, self.sigma, self.seed, c,
                          self.grad_count[c], lib=self.lib)
             self.grad_count[c] += 1
-            self.srv.push(c, self.client_T[c], g)
-        self.srv.apply_pending(len(batch))
+            if self.push_budget is None:
+                self.srv.push(c, self.client_T[c], g)
+            else:
+                self.srv.push_budget(c, self.client_T[c], g, self.push_budget)
+                self.srv.apply_pending(1)
+        if self.push_budget is None:
+            self.srv.apply_pending(len(batch))
         T = self.srv.T
         for c in batch:
             c = int(c)
@@ -47,6 +56,9 @@ class OracleSimulation:
             elif self.fetch == "param":
                 idx, val = self.srv.fetch_compact(c)
                 fetch_apply(self.clients[c], idx, val, lib=self.lib)
+                self.client_T[c] = T
+            elif self.fetch == "budget":
+                self.srv.fetch_budget(c, self.clients[c], self.fetch_budget)
                 self.client_T[c] = T
             else:
                 if self.srv.fetch_message(c, self.clients[c]):

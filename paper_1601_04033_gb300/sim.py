@@ -6,9 +6,12 @@ own copies of the parameters, a dispatcher decides which clients push next
 gradient of a synthetic quadratic at its (stale) copy, the server applies the
 pushes in arrival order (ASGD / SASGD / FASGD / divide-by-std), and each
 pushing client then refreshes its copy -- fully (``fetch="full"``), per
-parameter through B-FASGD's fetch compaction (``"param"``), or through one
-per-message B-FASGD decision (``"message"``).  Everything on the device runs
-in the library's kernels, through the C ABI.
+parameter through B-FASGD's fetch compaction (``"param"``), through one
+per-message B-FASGD decision (``"message"``), or per tensor under a bandwidth
+budget (``"budget"``: ``fetch_budget`` expected parameters per fetch over the
+partition ``tensor_sizes``).  With ``push_budget`` the pushes, too, go per
+tensor under that budget.  Everything on the device runs in the library's
+kernels, through the C ABI.
 
 Run as a script to compare the update rules over a learning-rate sweep:
 ``python -m paper_1601_04033_gb300.sim --compare``.
@@ -29,15 +32,23 @@ class Simulation:
     def __init__(self, P: int, lam: int, alpha: float, variant: int, *, K: int = 1,
                  gamma: float = 0.95, beta: float = 0.95, eps: float = 1e-4, seed: int = 0,
                  fetch: str = "full", c_fetch: float = 0.0, objective=None, theta0=None,
-                 exact: bool = False, device: str = "cuda"):
+                 exact: bool = False, device: str = "cuda", eps_b: float = 1e-8,
+                 tensor_sizes=None, fetch_budget: int | None = None,
+                 push_budget: int | None = None):
         import torch
-        if fetch not in ("full", "param", "message"):
-            raise ValueError("fetch must be full, param or message")
+        if fetch not in ("full", "param", "message", "budget"):
+            raise ValueError("fetch must be full, param, message or budget")
+        if (fetch == "budget" and fetch_budget is None) or \
+                ((fetch == "budget" or push_budget is not None) and tensor_sizes is None):
+            raise ValueError("per-tensor budgets need tensor_sizes (and fetch_budget)")
+        self.fetch_budget, self.push_budget = fetch_budget, push_budget
         self.torch = torch
         self.P, self.lam, self.K, self.seed, self.fetch = P, lam, K, seed, fetch
         self.stream = torch.cuda.current_stream()
         self.srv = fasgd.Server(P, lam, alpha, variant, gamma=gamma, beta=beta, eps=eps,
-                                seed=seed, stream=self.stream)
+                                eps_b=eps_b, seed=seed, stream=self.stream)
+        if tensor_sizes is not None:
+            self.srv.set_tensors(tensor_sizes)
         self.srv.set_fetch_threshold(c_fetch)
         self.srv.set_exact(exact)
         h, star, sigma = objective if objective is not None else streams.quadratic_objective(seed, P)
@@ -56,6 +67,9 @@ class Simulation:
         self.flag = torch.empty(1, dtype=torch.int32, device=device)
         self.fetched = 0
         self.fetch_opportunities = 0
+        # Parameters moved by per-tensor pushes and fetches (device counters).
+        self.pushed_params = torch.zeros(1, dtype=torch.int64, device=device)
+        self.fetched_params = torch.zeros(1, dtype=torch.int64, device=device)
 
     def _check(self, rc):
         if rc != fasgd.OK:
@@ -83,8 +97,15 @@ class Simulation:
                 self.sigma.data_ptr(), self.seed, c, self.grad_count[c], self.grads[k].data_ptr(),
                 self.stream.cuda_stream))
             self.grad_count[c] += 1
-            self.srv.push(c, self.client_T[c], self.grads[k])
-        self.srv.apply_pending(len(batch))
+            if self.push_budget is None:
+                self.srv.push(c, self.client_T[c], self.grads[k])
+            else:
+                self.srv.push_budget(c, self.client_T[c], self.grads[k], self.push_budget,
+                                     count_dev=self.cnt)
+                self.srv.apply_pending(1)
+                self.pushed_params += self.cnt
+        if self.push_budget is None:
+            self.srv.apply_pending(len(batch))
         T = self.srv.T
         for c in batch:
             c = int(c)
@@ -100,6 +121,12 @@ class Simulation:
                 self.srv.fetch_compact(c, self.idx, self.val, self.cnt)
                 fasgd.fetch_apply(self.clients[c], self.idx, self.val, n_dev=self.cnt,
                                   n_max=self.P, stream=self.stream)
+                self.client_T[c] = T
+            elif self.fetch == "budget":
+                # As for per-parameter fetches, the client reports this fetch's
+                # timestamp.
+                self.srv.fetch_budget(c, self.clients[c], self.fetch_budget, count_dev=self.cnt)
+                self.fetched_params += self.cnt
                 self.client_T[c] = T
             else:
                 self.srv.fetch_message(c, self.clients[c], fetched_dev=self.flag)
@@ -150,6 +177,44 @@ def compare(P: int, lam: int, n_batches: int, K: int, alphas, seed: int = 0, log
     return out
 
 
+def bandwidth_compare(P: int, lam: int, n_batches: int, T: int, fractions, seed: int = 0,
+                      noise: str = "independent"):
+    """Per-tensor fetch budgets (the future-work section's allocation by
+    statistics) against the same budgets spread uniformly over the tensors
+    (eps_b so large that every tensor's Eq. 9 probability is the same) and
+    against full fetches: for each rule and each fetch mode, the best final
+    loss over a learning-rate sweep, on one schedule, objective and start."""
+    sizes = streams.tensor_sizes(seed, P, T)
+    sched = streams.dispatch_schedule(seed, lam, n_batches, 1)
+    obj = streams.quadratic_objective(seed, P, noise=noise, tensors=sizes)
+    th0 = np.zeros(P, np.float32)
+    grid = [10.0 ** e for e in np.arange(-5.0, 0.01, 0.5)]
+    rules = (("sasgd", fasgd.SASGD, grid), ("fasgd", fasgd.FASGD, grid),
+             ("fasgd-std", fasgd.FASGD_STD, [g * 1e-3 for g in grid]))
+    modes = [("full", {})]
+    for f in fractions:
+        modes.append((f"stats_{f}", {"fetch": "budget", "fetch_budget": int(f * P)}))
+        modes.append((f"uniform_{f}", {"fetch": "budget", "fetch_budget": int(f * P), "eps_b": 1e6}))
+    out = {"P": P, "lambda": lam, "tensors": T, "batches": n_batches, "noise": noise,
+           "initial_loss": float(0.5 * np.sum(obj[0].astype(np.float64) * obj[1].astype(np.float64) ** 2)),
+           "rows": []}
+    for name, var, alphas in rules:
+        row = {"rule": name}
+        for mode, kw in modes:
+            best = (np.inf, None, 0.0)
+            for a in alphas:
+                sim = Simulation(P, lam, a, var, seed=seed, objective=obj, theta0=th0,
+                                 tensor_sizes=sizes, **kw)
+                loss = float(sim.run(sched)[-1])
+                moved = int(sim.fetched_params.item()) / (n_batches * P)
+                sim.close()
+                if np.isfinite(loss) and loss < best[0]:
+                    best = (loss, a, moved)
+            row[mode] = {"loss": best[0], "alpha": best[1], "fetched_fraction": best[2]}
+        out["rows"].append(row)
+    return out
+
+
 def main():
     ap = argparse.ArgumentParser(description=__doc__,
                                  formatter_class=argparse.RawDescriptionHelpFormatter)
@@ -160,7 +225,14 @@ def main():
     ap.add_argument("--K", type=int, default=1)
     ap.add_argument("--seed", type=int, default=0)
     ap.add_argument("--noise", choices=["independent", "fisher"], default="independent")
+    ap.add_argument("--bandwidth", action="store_true",
+                    help="compare per-tensor fetch budgets (by statistics vs uniform)")
+    ap.add_argument("--tensors", type=int, default=16)
     args = ap.parse_args()
+    if args.bandwidth:
+        print(json.dumps(bandwidth_compare(args.P, args.lam, args.batches, args.tensors,
+                                           (0.1, 0.3), args.seed, args.noise)))
+        return
     grid = [10.0 ** e for e in np.arange(-5.0, 1.01, 0.5)]
     alphas = {"asgd": grid, "sasgd": grid, "fasgd": grid, "fasgd-std": [g * 1e-3 for g in grid]}
     res = compare(args.P, args.lam, args.batches, args.K, alphas, args.seed,

@@ -240,15 +240,23 @@ _TAG_OBJ_H, _TAG_OBJ_STAR, _TAG_OBJ_SIGMA, _TAG_DISPATCH = 7, 8, 9, 10
 
 
 def quadratic_objective(seed: int, P: int, h_lo: float = 1e-2, h_hi: float = 10.0,
-                        sigma_lo: float = 1e-3, sigma_hi: float = 1e-1, noise: str = "independent"):
+                        sigma_lo: float = 1e-3, sigma_hi: float = 1e-1, noise: str = "independent",
+                        tensors=None):
     """A synthetic separable quadratic for the closed-loop simulation:
     curvatures h_p log-uniform[h_lo, h_hi], minimiser star_p ~ N(0, 0.1^2),
     gradient-noise scales sigma_p log-uniform[sigma_lo, sigma_hi] (fp32[P] each;
     noise="fisher" instead ties the noise to the curvature, sigma_p =
     0.03 sqrt(h_p), as when the gradient covariance tracks the Hessian).
     The spread of h makes a single learning rate a compromise across
-    parameters, as in a real network."""
+    parameters, as in a real network.  tensors (sizes of a partition of P):
+    each tensor's curvatures are also scaled by a common factor, log-uniform
+    over [0.1, 10], so that the tensors' statistics differ as layers do."""
     h = np.exp(_rng(seed, _TAG_OBJ_H).uniform(math.log(h_lo), math.log(h_hi), P)).astype(np.float32)
+    if tensors is not None:
+        sizes = np.asarray(tensors, dtype=np.int64)
+        assert int(sizes.sum()) == P
+        f = np.exp(_rng(seed, _TAG_OBJ_H, 1).uniform(math.log(0.1), math.log(10.0), sizes.size))
+        h = (h * np.repeat(f.astype(np.float32), sizes)).astype(np.float32)
     star = (_rng(seed, _TAG_OBJ_STAR).standard_normal(P, dtype=np.float32) * np.float32(0.1))
     if noise == "fisher":
         sigma = (np.float32(0.03) * np.sqrt(h)).astype(np.float32)

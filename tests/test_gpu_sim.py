@@ -76,3 +76,37 @@ def test_simulation_against_oracle(variant, K, fetch, exact):
     if fetch == "full":
         assert gl[-1] < gl[0]
     g.close()
+
+
+@pytest.mark.parametrize("exact", [False, True])
+@pytest.mark.parametrize("variant", [oracle.FASGD, oracle.SASGD])
+@pytest.mark.parametrize("mode", ["fetch", "push", "both"])
+def test_simulation_with_per_tensor_budgets(variant, mode, exact):
+    """Closed loop with per-tensor budgets: fetches of 10 % of P, pushes of
+    30 % of P, or both, over 12 tensors whose curvature scales differ.  Exact
+    mode reproduces the oracle bit for bit; the fast forms agree in loss."""
+    from paper_1601_04033_gb300.sim import Simulation
+    P, lam, n_batches = 20_011, 8, 120
+    alpha = {oracle.SASGD: 0.005, oracle.FASGD: 0.0005}[variant]   # curvatures up to ~100
+    sizes = streams.tensor_sizes(7, P, 12)
+    obj = streams.quadratic_objective(3, P, tensors=sizes)
+    th0 = np.zeros(P, np.float32)
+    sched = streams.dispatch_schedule(3, lam, n_batches, 1, rho=0.5)
+    kw = dict(seed=9, objective=obj, theta0=th0, eps_b=1e-3, tensor_sizes=sizes,
+              fetch="budget" if mode in ("fetch", "both") else "full",
+              fetch_budget=P // 10, push_budget=(3 * P // 10) if mode in ("push", "both") else None)
+    g = Simulation(P, lam, alpha, variant, exact=exact, **kw)
+    o = osim.OracleSimulation(P, lam, alpha, variant, **kw)
+    gl = g.run(sched, log_every=40)
+    ol = o.run(sched, log_every=40)
+    np.testing.assert_allclose(gl, ol, rtol=1e-10 if exact else 1e-5)
+    if exact or variant == oracle.SASGD:
+        th = g.torch.empty(P, device="cuda")
+        g.srv.pull(th)
+        assert_bitwise(th.cpu().numpy(), o.srv.theta.astype(np.float32), "budget sim theta")
+    if variant == oracle.SASGD:
+        assert gl[-1] < gl[0]
+    moved = int(g.fetched_params.item()) + int(g.pushed_params.item())
+    assert 0 < moved < n_batches * P * (2 if mode == "both" else 1)
+    g.close()
+
