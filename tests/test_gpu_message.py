@@ -126,3 +126,51 @@ def test_statistic_kept_by_the_dense_pass_equals_a_fresh_sum(P):
         fresh = srv.message_vbar()
         assert np.float32(kept).view(np.uint32) == np.float32(fresh).view(np.uint32), (t, kept, fresh)
         assert fresh == oracle.mean_v(state[3].cpu().numpy()), (t, fresh)
+
+
+@pytest.mark.slow
+def test_full_size_25m_messages():
+    """P = 25,000,000 (the benchmark's message workload, 4 clients): 10 message
+    pushes and 10 message fetches, every decision equal to the oracle's, the
+    statistic kept by the dense pass equal to a fresh sum at the end, and the
+    state on sampled parameters."""
+    import torch
+    from paper_1601_04033_gb300 import fasgd
+    w = streams.WORKLOADS["bfasgd-message-25m"].replace(lam=4, R=4)
+    P = w.P
+    pool = streams.gradient_pool(w, P)
+    th0 = streams.theta0(w, P)
+    g = GpuRun(w, oracle.FASGD, P, pool, th0, c_push=2.0, seed=SEED)
+    o = OracleRun(w, oracle.FASGD, P, pool, th0, c_push=2.0, seed=SEED)
+    g.srv.set_fetch_threshold(4.0)
+    o.srv.set_fetch_threshold(4.0)
+    flag = torch.full((1,), -1, dtype=torch.int32, device="cuda")
+    sent = torch.full((10,), -1, dtype=torch.int32, device="cuda")
+    ps = streams.push_stream(w, 10, 1)
+    fetched = []
+    for t in range(10):
+        cl, js, sl = ps.batch(t)
+        c, j, s = int(cl[0]), int(js[0]), int(sl[0])
+        g.srv.push_message(c, j, g.pool[s], sent_dev=sent[t:t + 1])
+        g.srv.apply_pending(1)
+        o.srv.push_message(c, j, pool[s])
+        o.srv.apply_pending(1)
+        copy = torch.zeros(P, device="cuda")
+        g.srv.fetch_message(c, copy, fetched_dev=flag)
+        ok = o.srv.fetch_message(c, np.zeros(P, np.float32))
+        assert int(flag.item()) == int(ok), f"fetch {t}"
+        fetched.append(ok)
+    assert g.srv.fetch_counts().tolist() == o.srv.fetch_count
+    kept = g.srv.message_vbar()
+    gs = g.state()
+    assert np.array_equal(sent.cpu().numpy(), np.array(o.srv.message_log, dtype=np.int32))
+    assert 0 < sum(o.srv.message_log) < 10 or 0 < sum(fetched) < 10
+    state = [torch.from_numpy(x).cuda() for x in gs[:4]]
+    g.srv.set_state(*state, gs[4])
+    fresh = g.srv.message_vbar()
+    assert np.float32(kept).view(np.uint32) == np.float32(fresh).view(np.uint32)
+    assert fresh == oracle.mean_v(gs[3])
+    idx = streams.sample_indices(P, 50_000)
+    os_ = o.state()
+    compare_states([x[idx] for x in gs[:4]] + [gs[4]], [x[idx] for x in os_[:4]] + [os_[4]],
+                   oracle.FASGD, "25M messages")
