@@ -243,6 +243,14 @@ def test_ragged_partitions(sizes):
     _stream(pair, 40, 0.4, 10)
 
 
+@pytest.mark.parametrize("sizes", [[1], [1, 1, 1], [2, 3], [5], [1, 1, 1, 1, 1]])
+def test_tiny_partitions(sizes):
+    """A handful of parameters, one-parameter tensors, no whole 16-byte quad."""
+    P = int(sum(sizes))
+    pair = Pair(P, np.array(sizes), exact=True)
+    _stream(pair, 30, 0.5, 10)
+
+
 def test_maximum_tensor_count():
     f = binding()
     P = 50_000
