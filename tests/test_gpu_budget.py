@@ -346,3 +346,45 @@ def test_size_2_28_64_tensors():
     ih = idx.cpu().numpy()
     os_ = pair.o.state()
     compare_states(gs, [x[ih] for x in os_[:4]] + [os_[4]], oracle.FASGD, "2^28 sampled")
+
+
+@pytest.mark.slow
+def test_largest_size_and_tensor_count():
+    """P = 2^31 - 1 in BFASGD_TMAX tensors (work items of 262,144 parameters,
+    the largest decision block): with v constant on each tensor the tensor
+    means are exact, so the oracle's threshold, decisions and counts are
+    computed from the partition alone and must match the GPU's bit for bit;
+    the fetched copy holds theta exactly on the transmitted tensors."""
+    torch = torch_cuda()
+    f = binding()
+    P = (1 << 31) - 1
+    T = f.BFASGD_TMAX
+    sizes = streams.tensor_sizes(13, P, T)
+    rng = np.random.default_rng(13)
+    vt = np.float32(2.0) ** rng.integers(-6, 7, T).astype(np.float32)   # exact means
+    srv = f.Server(P, 2, 0.001, f.FASGD, eps_b=1e-8, seed=SEED)
+    srv.set_tensors(sizes)
+    size_t = torch.from_numpy(sizes).cuda()
+    v = torch.repeat_interleave(torch.from_numpy(vt).cuda(), size_t, output_size=P)
+    theta = torch.arange(P, device="cuda", dtype=torch.float32)
+    z = torch.zeros(P, device="cuda")
+    srv.set_state(theta, z, z, v, 0)
+    del v, z
+    sent = torch.zeros(T, dtype=torch.uint8, device="cuda")
+    c = torch.zeros(1, device="cuda")
+    cnt = torch.zeros(1, dtype=torch.int64, device="cuda")
+    copy = torch.full((P,), -1.0, device="cuda")
+    off = np.concatenate([[0], np.cumsum(sizes)])
+    for k, budget in enumerate([P, P // 5, 0]):
+        srv.fetch_budget(1, copy, budget, sent, c, cnt)
+        want_c = oracle.budget_c(sizes, vt, 1e-8, budget)
+        want_sent, want_m = oracle.tensor_select(sizes, vt, want_c, 1e-8, SEED, 1, 1, k)
+        assert np.float32(c.item()).view(np.uint32) == np.float32(want_c).view(np.uint32), (budget, c.item(), want_c)
+        assert np.array_equal(sent.cpu().numpy(), want_sent), budget
+        assert int(cnt.item()) == want_m
+        if budget == P:
+            assert want_m == P
+        # The copy equals theta on a sample of parameters of every transmitted tensor.
+        for t in np.flatnonzero(want_sent)[:64]:
+            for p in (int(off[t]), int(off[t + 1]) - 1, int((off[t] + off[t + 1]) // 2)):
+                assert copy[p].item() == theta[p].item(), (budget, t, p)
