@@ -55,8 +55,9 @@ constexpr unsigned kFull = 0xffffffffu;
 // (after the last), then quads qs + tid, qs + tid + 256, ...; the threads'
 // pairs go through a fixed float-float tree.  Four quads are loaded before
 // they are added, so a thread keeps four loads in flight.  Called by every
-// thread of the block; the result is valid in thread 0.
-__device__ float2 item_v_sum(const TensorItem& it, const float* __restrict__ v, float2* smem) {
+// thread of the block; the result is valid in thread 0.  Plain loads (no
+// read-only path): the apply kernel reads values it has just written.
+__device__ float2 item_v_sum(const TensorItem& it, const float* v, float2* smem) {
     const int tid = threadIdx.x;
     const int64_t s = it.start, e = s + it.len;
     const int64_t qs = (s + 3) >> 2, qe = e >> 2;   // whole quads inside [s, e)
