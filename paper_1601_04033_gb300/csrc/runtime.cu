@@ -107,6 +107,8 @@ struct fasgd_s {
     std::vector<float*> stage;
     std::vector<char> stage_busy;       // held by a queued push
     std::vector<char> stage_used;       // slot_free has been recorded
+    std::vector<uint64_t> stage_seq;    // pass that last read the slot (larger = later)
+    uint64_t pass_seq = 0;
     std::vector<cudaEvent_t> slot_ready;  // the copy into the slot is done
     std::vector<cudaEvent_t> slot_free;   // the last pass reading the slot is done
     cudaStream_t copy_stream = nullptr;
@@ -504,14 +506,17 @@ int fasgd_push_host(fasgd_t* h, int32_t client, int64_t timestamp, const float* 
     if (st != cudaSuccess) return h->cuda_fail(st, "fasgd_push_host: streams");
     // Prefer a free slot no pass is still reading; else grow the pool; else
     // take any free slot (its copy then waits for the pass that read it).
+    // If no slot is free, the one read longest ago is taken: its reader is the
+    // likeliest to have finished, so the copy engine rarely waits on a pass.
     int slot = -1, waiting = -1;
+    bool must_wait = false;   // the slot's last reader may still be running
     for (size_t s = 0; s < h->stage.size(); ++s) {
         if (h->stage_busy[s]) continue;
         if (!h->stage_used[s] || cudaEventQuery(h->slot_free[s]) == cudaSuccess) {
             slot = (int)s;
             break;
         }
-        if (waiting < 0) waiting = (int)s;
+        if (waiting < 0 || h->stage_seq[s] < h->stage_seq[(size_t)waiting]) waiting = (int)s;
     }
     if (slot < 0 && (int)h->stage.size() < FASGD_KMAX) {
         float* p = nullptr;
@@ -527,13 +532,19 @@ int fasgd_push_host(fasgd_t* h, int32_t client, int64_t timestamp, const float* 
         h->stage.push_back(p);
         h->stage_busy.push_back(0);
         h->stage_used.push_back(0);
+        h->stage_seq.push_back(0);
         h->slot_ready.push_back(ready);
         h->slot_free.push_back(freed);
         slot = (int)h->stage.size() - 1;
     }
-    if (slot < 0) slot = waiting;
+    if (slot < 0 && waiting >= 0) {
+        slot = waiting;
+        must_wait = true;
+    }
     if (slot < 0) return h->fail(FASGD_EAGAIN, "%d host pushes already pending", FASGD_KMAX);
-    if (h->stage_used[(size_t)slot]) st = cudaStreamWaitEvent(h->copy_stream, h->slot_free[(size_t)slot], 0);
+    // A slot whose last reader has finished needs no dependency: skipping the
+    // wait keeps the copy engine streaming from one copy into the next.
+    if (must_wait) st = cudaStreamWaitEvent(h->copy_stream, h->slot_free[(size_t)slot], 0);
     if (st == cudaSuccess)
         st = cudaMemcpyAsync(h->stage[(size_t)slot], grad_host, (size_t)h->P * sizeof(float),
                              cudaMemcpyDefault, h->copy_stream);
@@ -740,11 +751,13 @@ int fasgd_apply_pending(fasgd_t* h, int32_t K) {
                 if (slot >= 0) st = cudaStreamWaitEvent(h->stream, h->slot_ready[(size_t)slot], 0);
             }
             if (st == cudaSuccess) st = fasgd::launch_dense(a, rule, h->exact, h->num_sms, h->stream, &h->launches);
+            ++h->pass_seq;
             for (int i = 0; i < r && st == cudaSuccess; ++i) {  // the slots may be refilled after this
                 const int slot = h->fifo[(size_t)(k + i)].stage;
                 if (slot >= 0) {
                     st = cudaEventRecord(h->slot_free[(size_t)slot], h->stream);
                     h->stage_used[(size_t)slot] = 1;
+                    h->stage_seq[(size_t)slot] = h->pass_seq;
                 }
             }
             if (st != cudaSuccess) return h->cuda_fail(st, "fasgd_apply_pending: dense pass");
