@@ -97,8 +97,18 @@ __global__ void __launch_bounds__(kScanThreads) bfasgd_scan_kernel(const __grid_
     const int per = (a.ntiles + kScanThreads - 1) / kScanThreads;
     const int lo = tid * per;
     const int hi = min(lo + per, a.ntiles);
+    // Up to four counts per thread (P up to 32M) are loaded at once and kept.
+    constexpr int kKeep = 4;
+    int32_t kept[kKeep];
     int64_t local = 0;
-    for (int t = lo; t < hi; ++t) local += a.tile_count[t];
+    if (per <= kKeep) {
+#pragma unroll
+        for (int k = 0; k < kKeep; ++k) kept[k] = lo + k < hi ? a.tile_count[lo + k] : 0;
+#pragma unroll
+        for (int k = 0; k < kKeep; ++k) local += kept[k];
+    } else {
+        for (int t = lo; t < hi; ++t) local += a.tile_count[t];
+    }
     // Inclusive scan of the per-thread sums across the block.
     int64_t incl = local;
 #pragma unroll
@@ -119,9 +129,18 @@ __global__ void __launch_bounds__(kScanThreads) bfasgd_scan_kernel(const __grid_
     }
     __syncthreads();
     int64_t run = incl - local + (warp > 0 ? warp_sum[warp - 1] : 0);  // exclusive prefix
-    for (int t = lo; t < hi; ++t) {
-        a.tile_base[t] = run;
-        run += a.tile_count[t];
+    if (per <= kKeep) {
+#pragma unroll
+        for (int k = 0; k < kKeep; ++k)
+            if (lo + k < hi) {
+                a.tile_base[lo + k] = run;
+                run += kept[k];
+            }
+    } else {
+        for (int t = lo; t < hi; ++t) {
+            a.tile_base[t] = run;
+            run += a.tile_count[t];
+        }
     }
     if (tid == kScanThreads - 1) *a.count = warp_sum[kScanThreads / 32 - 1];
 }
