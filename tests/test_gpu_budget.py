@@ -388,3 +388,38 @@ def test_largest_size_and_tensor_count():
         for t in np.flatnonzero(want_sent)[:64]:
             for p in (int(off[t]), int(off[t + 1]) - 1, int((off[t] + off[t + 1]) // 2)):
                 assert copy[p].item() == theta[p].item(), (budget, t, p)
+
+
+def test_mixed_kinds_in_one_apply():
+    """Dense, per-tensor, sparse and per-message pushes queued together and
+    applied by single fasgd_apply_pending calls: each in arrival order at its
+    own timestamp, bit for bit with the oracle (exact mode)."""
+    torch = torch_cuda()
+    P = 40_009
+    sizes = streams.tensor_sizes(6, P, 11)
+    pair = Pair(P, sizes, exact=True)
+    pair.srv.set_hparams(HP["gamma"], HP["beta"], HP["eps"], 2.0, 1e-8, SEED)
+    pair.o.set_hparams(HP["gamma"], HP["beta"], HP["eps"], 2.0, 1e-8, SEED)
+    idx = torch.empty(P, dtype=torch.int32, device="cuda")
+    val = torch.empty(P, dtype=torch.float32, device="cuda")
+    cnt = torch.empty(1, dtype=torch.int64, device="cuda")
+    for rnd in range(6):
+        T = pair.srv.T
+        assert T == pair.o.T
+        s0, s1, s2, s3, s4 = [(rnd * 5 + k) % 8 for k in range(5)]
+        pair.srv.push(0, T, pair.dpool[s0])
+        pair.o.push(0, T, pair.pool[s0])
+        pair.srv.push_budget(1, max(T - 1, 0), pair.dpool[s1], P // 3, pair.sent, pair.c, pair.count)
+        pair.o.push_budget(1, max(T - 1, 0), pair.pool[s1], P // 3)
+        pair.srv.select_compact(2, pair.dpool[s2], idx, val, cnt)
+        pair.srv.push_sparse(2, T, idx, val, n_dev=cnt, n_max=P)
+        oi, ov = pair.o.select_compact(2, pair.pool[s2])
+        pair.o.push_sparse(2, T, oi, ov)
+        pair.srv.push_message(3, T, pair.dpool[s3])
+        pair.o.push_message(3, T, pair.pool[s3])
+        pair.srv.push(0, T, pair.dpool[s4])
+        pair.o.push(0, T, pair.pool[s4])
+        pair.srv.apply_pending(5)
+        pair.o.apply_pending(5)
+        pair.check_decision(pair.decision(), pair.o.budget_log[-1], f"mixed round {rnd}")
+    compare_states(pair.gpu_state(), list(pair.o.state()), oracle.FASGD, "mixed", exact=True)
