@@ -203,3 +203,37 @@ def test_exact_mode_is_bitwise(variant, K, eps):
         w = w.replace(alpha=w.alpha * 1e-3)
     n = 100 * K // np.gcd(100, K)
     run_parity(w, variant, 30_011, n, K, eps=eps, exact=True)
+
+
+@pytest.mark.slow
+def test_largest_size_sampled():
+    """P = 2^31 - 1 (the largest the ABI accepts; 2047 parameters after the last
+    full tile go through the tail path), K = 2, three passes, on gradients and
+    start values drawn on the device; every sampled parameter, and the last
+    4096, against the oracle run on those parameters alone."""
+    import torch
+    from paper_1601_04033_gb300 import fasgd
+    P = (1 << 31) - 1
+    gen = torch.Generator(device="cuda").manual_seed(31)
+    grads = [torch.randn(P, device="cuda", generator=gen) * 0.05 for _ in range(2)]
+    theta0 = torch.randn(P, device="cuda", generator=gen) * 0.01
+    srv = fasgd.Server(P, 4, 0.001, fasgd.FASGD)
+    srv.set_params(theta0)
+    idx = np.unique(np.concatenate([streams.sample_indices(P, 20_000),
+                                    np.arange(P - 4096, P)])).astype(np.int64)
+    idx_t = torch.from_numpy(idx).cuda()
+    g_s = [g[idx_t].cpu().numpy() for g in grads]
+    o = oracle.OracleServer(idx.size, 4, 0.001, oracle.FASGD)
+    o.set_params(theta0[idx_t].cpu().numpy())
+    for b in range(3):
+        for k in range(2):
+            srv.push(k, max(srv.T - 1, 0), grads[k])
+            o.push(k, max(o.T - 1, 0), g_s[k])
+        srv.apply_pending(2)
+        o.apply_pending(2)
+    del grads, theta0
+    torch.cuda.empty_cache()
+    full = [torch.empty(P, device="cuda") for _ in range(4)]
+    T = srv.get_state(*full)
+    gs = [x[idx_t].cpu().numpy() for x in full] + [T]
+    compare_states(gs, list(o.state()), oracle.FASGD, "2^31-1 sampled")
