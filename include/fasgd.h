@@ -203,9 +203,9 @@ FASGD_API int bfasgd_select_compact(fasgd_t* h, int32_t client, const float* gra
 
 /*
  * bfasgd_fetch_compact -- B-FASGD fetch decision and compaction, per
- * parameter (Sec. 2.3: a client "given an opportunity to ... receive a
- * parameter update" takes it iff Eq. 9 holds, here with each parameter's own
- * v_p as the future-work section proposes).  Exactly as
+ * parameter (Sec. 2.3: at each chance to receive fresh parameters a client
+ * takes them iff Eq. 9 holds; here with each parameter's own v_p, as the
+ * future-work section proposes).  Exactly as
  * bfasgd_select_compact, with the fetch threshold c_fetch
  * (fasgd_set_fetch_threshold), draws from the fetch stream (counter word
  * client + 2^31, push# replaced by the client's count of earlier fetches),

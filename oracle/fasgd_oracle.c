@@ -246,9 +246,9 @@ int64_t ora_select(int64_t P, const float *g, const float *v, float c, float eps
 }
 
 /*
- * B-FASGD fetch, per parameter (Sec. 2.3: "given an opportunity to ...
- * receive a parameter update", with the per-parameter extension of the
- * future-work section): the server keeps p iff Eq. 9 holds for v[p] with the
+ * B-FASGD fetch, per parameter (Sec. 2.3 applies Eq. 9 to each chance a
+ * client has to receive fresh parameters; here per parameter, the extension
+ * of the future-work section): the server keeps p iff Eq. 9 holds for v[p] with the
  * fetch threshold c (stream 1 draws) and sends (p, theta[p]); the client
  * overwrites its copy at the kept indices and keeps computing with its own
  * stale values everywhere else.
