@@ -237,3 +237,22 @@ def test_largest_size_sampled():
     T = srv.get_state(*full)
     gs = [x[idx_t].cpu().numpy() for x in full] + [T]
     compare_states(gs, list(o.state()), oracle.FASGD, "2^31-1 sampled")
+
+
+@pytest.mark.parametrize("exact", [False, True])
+@pytest.mark.parametrize("gamma,beta,eps", [(0.0, 0.95, 1e-4), (1.0, 0.95, 1e-4),
+                                            (0.95, 0.0, 1e-4), (0.5, 0.5, 0.0),
+                                            (0.999, 0.999, 1.0)])
+def test_hyperparameter_extremes(gamma, beta, eps, exact):
+    """Degenerate and extreme settings of Eq. 4-6: gamma = 0 (n, b follow the last
+    gradient, the variance is 0), gamma = 1 (n, b stay 0), beta = 0 (v is the last
+    r), eps = 0 and a large eps; fused K = 3 passes.  With beta = 0.999 the first
+    v is 1e-3 r, so the first steps are of order 1 and theta swings through values
+    near 1 before it settles near 1e-3: the rounding of those swings alone is
+    above the relative bound, so the fast arithmetic runs that case at alpha / 1000
+    (the exact mode runs it as it is, bit for bit)."""
+    w = W["fasgd-7850"].replace(R=8)
+    if beta > 0.99 and not exact:
+        w = w.replace(alpha=w.alpha * 1e-3)
+    run_parity(w, oracle.FASGD, 20_011, 60, 3, check_every=30, gamma=gamma, beta=beta, eps=eps,
+               exact=exact)
