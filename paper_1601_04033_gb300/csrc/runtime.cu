@@ -11,6 +11,7 @@
 // rounded once to fp32.
 
 #include <cuda_runtime.h>
+#include <nvtx3/nvToolsExt.h>
 
 #include <cmath>
 #include <cstdarg>
@@ -51,6 +52,15 @@ struct Push {
     uint8_t* sent_out;     // budget push: caller copies of the decisions (each may be null)
     float* c_out;
     int64_t* count_out;
+};
+
+// An NVTX range around a call that launches work or copies (visible to
+// Nsight tools and to ncu --nvtx; free when no tool is attached).
+struct TraceRange {
+    explicit TraceRange(const char* name) { nvtxRangePushA(name); }
+    ~TraceRange() { nvtxRangePop(); }
+    TraceRange(const TraceRange&) = delete;
+    TraceRange& operator=(const TraceRange&) = delete;
 };
 
 bool aligned(const void* p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) & (a - 1)) == 0; }
@@ -497,6 +507,7 @@ int fasgd_push(fasgd_t* h, int32_t client, int64_t timestamp, const float* grad)
 }
 
 int fasgd_push_host(fasgd_t* h, int32_t client, int64_t timestamp, const float* grad_host) {
+    TraceRange trace("fasgd_push_host");
     if (h == nullptr) return FASGD_EINVAL;
     if (grad_host == nullptr) return h->fail(FASGD_EINVAL, "grad_host is NULL");
     int rc = check_push(h, client, timestamp);
@@ -571,6 +582,7 @@ int bfasgd_push_message(fasgd_t* h, int32_t client, int64_t timestamp, const flo
 }
 
 int bfasgd_fetch_message(fasgd_t* h, int32_t client, float* theta_client, int32_t* fetched_dev) {
+    TraceRange trace("bfasgd_fetch_message");
     if (h == nullptr) return FASGD_EINVAL;
     if (client < 0 || client >= h->lambda)
         return h->fail(FASGD_ERANGE, "client %d outside [0, %d)", client, h->lambda);
@@ -587,6 +599,7 @@ int bfasgd_fetch_message(fasgd_t* h, int32_t client, float* theta_client, int32_
 }
 
 int bfasgd_set_tensors(fasgd_t* h, int32_t T, const int64_t* sizes) {
+    TraceRange trace("bfasgd_set_tensors");
     if (h == nullptr) return FASGD_EINVAL;
     if (T < 1 || T > BFASGD_TMAX || sizes == nullptr)
         return h->fail(FASGD_EINVAL, "T must be in [1, %d] and sizes non-NULL", BFASGD_TMAX);
@@ -664,6 +677,7 @@ int bfasgd_push_budget(fasgd_t* h, int32_t client, int64_t timestamp, const floa
 
 int bfasgd_fetch_budget(fasgd_t* h, int32_t client, float* theta_client, int64_t budget,
                         uint8_t* sent_dev, float* c_dev, int64_t* count_dev) {
+    TraceRange trace("bfasgd_fetch_budget");
     if (h == nullptr) return FASGD_EINVAL;
     if (h->tensor_sizes.empty()) return h->fail(FASGD_EINVAL, "no tensor partition (bfasgd_set_tensors)");
     if (client < 0 || client >= h->lambda)
@@ -686,6 +700,7 @@ int bfasgd_fetch_budget(fasgd_t* h, int32_t client, float* theta_client, int64_t
 }
 
 int bfasgd_message_vbar(fasgd_t* h, float* vbar_dev) {
+    TraceRange trace("bfasgd_message_vbar");
     if (h == nullptr) return FASGD_EINVAL;
     if (vbar_dev == nullptr || !aligned(vbar_dev, 4))
         return h->fail(FASGD_EINVAL, "vbar_dev must be a non-NULL 4-byte aligned device pointer");
@@ -712,6 +727,7 @@ int fasgd_push_sparse(fasgd_t* h, int32_t client, int64_t timestamp, const int32
 }
 
 int fasgd_apply_pending(fasgd_t* h, int32_t K) {
+    TraceRange trace("fasgd_apply_pending");
     if (h == nullptr) return FASGD_EINVAL;
     if (K < 1 || K > FASGD_KMAX) return h->fail(FASGD_EINVAL, "K must be in [1, %d]", FASGD_KMAX);
     if ((int64_t)h->fifo.size() < K)
@@ -838,6 +854,7 @@ int fasgd_apply_pending(fasgd_t* h, int32_t K) {
 static int run_select(fasgd_t* h, const char* what, uint32_t stream, int32_t client,
                       const float* values, const float* v, int32_t* idx, float* val,
                       int64_t* n_dev, float c, std::vector<uint64_t>& counter) {
+    TraceRange trace(what);
     if (client < 0 || client >= h->lambda)
         return h->fail(FASGD_ERANGE, "%s: client %d outside [0, %d)", what, client, h->lambda);
     if (values == nullptr || !aligned(values, 16))
@@ -900,6 +917,7 @@ int fasgd_set_fetch_threshold(fasgd_t* h, float c_fetch) {
 
 int bfasgd_fetch_apply(int64_t P, float* theta_client, const int32_t* idx, const float* val,
                        const int64_t* n_dev, int64_t n_max, void* stream, int32_t* err_dev) {
+    TraceRange trace("bfasgd_fetch_apply");
     if (P < 1 || P > FASGD_PMAX) {
         g_create_error = "bfasgd_fetch_apply: P must be in [1, 2^31)";
         return FASGD_EINVAL;
@@ -988,6 +1006,7 @@ int fasgd_sim_quadratic_loss(int64_t P, const float* theta, const float* hcurv, 
 }
 
 int fasgd_pull(fasgd_t* h, float* params, int64_t* T) {
+    TraceRange trace("fasgd_pull");
     if (h == nullptr) return FASGD_EINVAL;
     if (params != nullptr) {
         // The copy runs on its own stream (so it overlaps host-push copies of
@@ -1009,6 +1028,7 @@ int fasgd_pull(fasgd_t* h, float* params, int64_t* T) {
 }
 
 int fasgd_get_state(fasgd_t* h, float* theta, float* n, float* b, float* v, int64_t* T) {
+    TraceRange trace("fasgd_get_state");
     if (h == nullptr) return FASGD_EINVAL;
     if (!h->fifo.empty()) return h->fail(FASGD_EAGAIN, "pushes are pending");
     DeviceGuard g(h->device);
@@ -1028,6 +1048,7 @@ int fasgd_get_state(fasgd_t* h, float* theta, float* n, float* b, float* v, int6
 
 int fasgd_set_state(fasgd_t* h, const float* theta, const float* n, const float* b,
                     const float* v, int64_t T) {
+    TraceRange trace("fasgd_set_state");
     if (h == nullptr) return FASGD_EINVAL;
     if (T < 0) return h->fail(FASGD_EINVAL, "T must be >= 0");
     if (!h->fifo.empty()) return h->fail(FASGD_EAGAIN, "pushes are pending");
