@@ -371,7 +371,7 @@ def run_bfasgd(args, w, world, rank, local):
     R = min(w.R, 8)
     pool = streams.gradient_pool(wr, P, R)
     th0 = streams.theta0(wr, P)
-    n_steps = args.warmup + args.steps + w.lam
+    n_steps = args.warmup + args.steps + w.lam + 100   # + the instrumented stage run
     ps = streams.push_stream(w.replace(R=R), n_steps, 1)
     pool_t, slots = fasgd.aligned_vectors(pool, device)
     stream = torch.cuda.current_stream()
@@ -408,31 +408,29 @@ def run_bfasgd(args, w, world, rank, local):
         of theta, client scatter)."""
         cl, js, sl = ps.batch(t)
         c = int(cl[0])
+        n_push = cnt if i is None else counts[i:i + 1]       # the kernels write the counts
+        n_fetch = fcnt if i is None else fcounts[i:i + 1]
         if ev is not None:
             ev[0].record(stream)
-        srv.select_compact(c, slots[int(sl[0])], idx, val, cnt)      # live server v
+        srv.select_compact(c, slots[int(sl[0])], idx, val, n_push)      # live server v
         if ev is not None:
             ev[1].record(stream)
-        srv.push_sparse(c, int(js[0]), idx, val, n_dev=cnt, n_max=P)
+        srv.push_sparse(c, int(js[0]), idx, val, n_dev=n_push, n_max=P)
         srv.apply_pending(1)
         if ev is not None:
             ev[2].record(stream)
-        srv.fetch_compact(c, fidx, fval, fcnt)
+        srv.fetch_compact(c, fidx, fval, n_fetch)
         if ev is not None:
             ev[3].record(stream)
-        fasgd.fetch_apply(client_theta[c], fidx, fval, n_dev=fcnt, n_max=P, stream=stream)
+        fasgd.fetch_apply(client_theta[c], fidx, fval, n_dev=n_fetch, n_max=P, stream=stream)
         if ev is not None:
             ev[4].record(stream)
-        if i is not None:
-            counts[i:i + 1].copy_(cnt, non_blocking=True)
-            fcounts[i:i + 1].copy_(fcnt, non_blocking=True)
 
     for _ in range(args.warmup):
         step(t)
         t += 1
     torch.cuda.synchronize()
     clocks = ClockSampler(gpu_identifier(torch))
-    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(args.steps)]
     start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     launches0 = srv.launches
     barrier(world)
@@ -440,8 +438,8 @@ def run_bfasgd(args, w, world, rank, local):
     clocks.start()
     time.sleep(0.3)
     start.record(stream)
-    for i in range(args.steps):
-        step(t, ev[i], i)
+    for i in range(args.steps):     # no events inside: they would split the launch chains
+        step(t, None, i)
         t += 1
     end.record(stream)
     torch.cuda.synchronize()
@@ -449,7 +447,14 @@ def run_bfasgd(args, w, world, rank, local):
     barrier(world)
     launches = srv.launches - launches0 + args.steps      # + one fetch scatter per step
     total_ms = max_over_ranks(start.elapsed_time(end), world, device)
-    stage = [sum(e[k].elapsed_time(e[k + 1]) for e in ev) / args.steps for k in range(4)]
+    # Stage times from a second, instrumented run of the same exchange.
+    n_diag = min(args.steps, 100)
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(n_diag)]
+    for i in range(n_diag):
+        step(t, ev[i])
+        t += 1
+    torch.cuda.synchronize()
+    stage = [sum(e[k].elapsed_time(e[k + 1]) for e in ev) / n_diag for k in range(4)]
     sel_ms, app_ms, fsel_ms, fapp_ms = stage
     sent = counts.cpu().numpy().astype(np.float64)
     fetched = fcounts.cpu().numpy().astype(np.float64)
@@ -500,7 +505,7 @@ def run_message(args, w, world, rank, local):
     R = min(w.R, 8)
     pool = streams.gradient_pool(wr, P, R)
     th0 = streams.theta0(wr, P)
-    n_steps = args.warmup + args.steps + w.lam
+    n_steps = args.warmup + args.steps + w.lam + 100   # + the instrumented stage run
     ps = streams.push_stream(w.replace(R=R), n_steps, 1)
     pool_t, slots = fasgd.aligned_vectors(pool, device)
     stream = torch.cuda.current_stream()
@@ -543,7 +548,6 @@ def run_message(args, w, world, rank, local):
         t += 1
     torch.cuda.synchronize()
     clocks = ClockSampler(gpu_identifier(torch))
-    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
     start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     launches0 = srv.launches
     barrier(world)
@@ -551,8 +555,8 @@ def run_message(args, w, world, rank, local):
     clocks.start()
     time.sleep(0.3)
     start.record(stream)
-    for i in range(args.steps):
-        step(t, ev[i], i)
+    for i in range(args.steps):     # no events inside: they would split the launch chains
+        step(t, None, i)
         t += 1
     end.record(stream)
     torch.cuda.synchronize()
@@ -560,8 +564,15 @@ def run_message(args, w, world, rank, local):
     barrier(world)
     launches = srv.launches - launches0
     total_ms = max_over_ranks(start.elapsed_time(end), world, device)
-    push_ms = sum(e[0].elapsed_time(e[1]) for e in ev) / args.steps
-    fetch_ms = sum(e[1].elapsed_time(e[2]) for e in ev) / args.steps
+    # Push / fetch times from a second, instrumented run of the same exchange.
+    n_diag = min(args.steps, 100)
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(n_diag)]
+    for i in range(n_diag):
+        step(t, ev[i])
+        t += 1
+    torch.cuda.synchronize()
+    push_ms = sum(e[0].elapsed_time(e[1]) for e in ev) / n_diag
+    fetch_ms = sum(e[1].elapsed_time(e[2]) for e in ev) / n_diag
     s_frac = float(sent.float().mean().item())
     f_frac = float(fetched.float().mean().item())
     srv.sync()
@@ -610,7 +621,7 @@ def run_tensor(args, w, world, rank, local):
     pool = streams.gradient_pool(wr, P, R)
     th0 = streams.theta0(wr, P)
     sizes = streams.tensor_sizes(w.seed, P, w.tensors)
-    n_steps = args.warmup + args.steps + w.lam
+    n_steps = args.warmup + args.steps + w.lam + 100   # + the instrumented stage run
     ps = streams.push_stream(w.replace(R=R), n_steps, 1)
     pool_t, slots = fasgd.aligned_vectors(pool, device)
     stream = torch.cuda.current_stream()
@@ -652,7 +663,6 @@ def run_tensor(args, w, world, rank, local):
         t += 1
     torch.cuda.synchronize()
     clocks = ClockSampler(gpu_identifier(torch))
-    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
     start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     launches0 = srv.launches
     barrier(world)
@@ -660,8 +670,8 @@ def run_tensor(args, w, world, rank, local):
     clocks.start()
     time.sleep(0.3)
     start.record(stream)
-    for i in range(args.steps):
-        step(t, ev[i], i)
+    for i in range(args.steps):     # no events inside: they would split the launch chains
+        step(t, None, i)
         t += 1
     end.record(stream)
     torch.cuda.synchronize()
@@ -669,8 +679,15 @@ def run_tensor(args, w, world, rank, local):
     barrier(world)
     launches = srv.launches - launches0
     total_ms = max_over_ranks(start.elapsed_time(end), world, device)
-    push_ms = sum(e[0].elapsed_time(e[1]) for e in ev) / args.steps
-    fetch_ms = sum(e[1].elapsed_time(e[2]) for e in ev) / args.steps
+    # Push / fetch times from a second, instrumented run of the same exchange.
+    n_diag = min(args.steps, 100)
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(n_diag)]
+    for i in range(n_diag):
+        step(t, ev[i])
+        t += 1
+    torch.cuda.synchronize()
+    push_ms = sum(e[0].elapsed_time(e[1]) for e in ev) / n_diag
+    fetch_ms = sum(e[1].elapsed_time(e[2]) for e in ev) / n_diag
     s_mean = float(sent.double().mean().item())
     f_mean = float(fetched.double().mean().item())
     c_med = float(cvals.median().item())
