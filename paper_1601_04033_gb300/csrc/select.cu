@@ -12,7 +12,8 @@
 //               total m;
 //   3. compact: per tile, rebuild each parameter's rank among the sent ones
 //               from the bit mask (warp popc + shuffles, block scan over
-//               warps) and write idx[rank] = p, val[rank] = grad[p].
+//               warps) and write idx[rank] = p, val[rank] = grad[p], staged
+//               per warp in shared memory so that the stores are coalesced.
 // The order of the output is the order of p, so the result is unique and
 // does not depend on the launch; no atomics are used.  Traffic per
 // parameter: v (4 B) + grad (4 B) + 2 x 1/8 B of mask, plus 8 B per sent
@@ -30,10 +31,19 @@ constexpr int kWarpSpan = kSelectTile / kWarps;  // 1024 parameters per warp
 constexpr int kIters = kWarpSpan / 128;          // 8 passes of 32 lanes x 4
 constexpr unsigned kFull = 0xffffffffu;
 
-__global__ void __launch_bounds__(kSelectThreads) bfasgd_mask_kernel(const __grid_constant__ SelectArgs a) {
+// The four values e .. e+3 of x (zero past P; FULL: the tile lies inside P).
+template <bool FULL>
+__device__ __forceinline__ float4 load_quad(const float* x, int64_t e, int64_t P) {
+    if (FULL || e + 3 < P) return __ldcs(reinterpret_cast<const float4*>(x + e));
+    float t[4] = {0.f, 0.f, 0.f, 0.f};
+    for (int j = 0; j < 4; ++j)
+        if (e + j < P) t[j] = x[e + j];
+    return make_float4(t[0], t[1], t[2], t[3]);
+}
+
+template <bool FULL>
+__device__ __forceinline__ void mask_tile(const SelectArgs& a) {
     __shared__ int32_t warp_cnt[kWarps];
-    pdl_wait();
-    pdl_trigger();
     const int lane = threadIdx.x & 31;
     const int warp = threadIdx.x >> 5;
     const int64_t tile_start = (int64_t)blockIdx.x * kSelectTile;
@@ -41,30 +51,23 @@ __global__ void __launch_bounds__(kSelectThreads) bfasgd_mask_kernel(const __gri
     // All of this lane's v loads first (eight quads), then the draws.
     float4 v4[kIters];
 #pragma unroll
-    for (int it = 0; it < kIters; ++it) {
-        const int64_t e = warp_start + it * 128 + 4 * lane;  // first parameter of this quad
-        if (e + 3 < a.P) {
-            v4[it] = __ldcs(reinterpret_cast<const float4*>(a.v + e));
-        } else {
-            float t[4] = {0.f, 0.f, 0.f, 0.f};
-            for (int j = 0; j < 4; ++j)
-                if (e + j < a.P) t[j] = a.v[e + j];
-            v4[it] = make_float4(t[0], t[1], t[2], t[3]);
-        }
-    }
+    for (int it = 0; it < kIters; ++it) v4[it] = load_quad<FULL>(a.v, warp_start + it * 128 + 4 * lane, a.P);
+    const uint32_t e_lane = (uint32_t)(warp_start + 4 * lane);  // P < 2^31
     int cnt = 0;
 #pragma unroll
     for (int it = 0; it < kIters; ++it) {
-        const int64_t e = warp_start + it * 128 + 4 * lane;
+        const uint32_t e = e_lane + it * 128;
         uint32_t nib = 0;
-        if (e < a.P) {
-            const Philox4 r = philox4x32_10((uint32_t)(e >> 2), a.client_word, a.push_lo, a.push_hi, a.round_key0, a.round_key1);
+        if (FULL || e < a.P) {
+            const Philox4 r = philox4x32_10(e >> 2, a.client_word, a.push_lo, a.push_hi, a.round_key0, a.round_key1);
             nib = send_bit(r.x[0] >> 8, v4[it].x, a.c, a.eps_b) |
                   (send_bit(r.x[1] >> 8, v4[it].y, a.c, a.eps_b) << 1) |
                   (send_bit(r.x[2] >> 8, v4[it].z, a.c, a.eps_b) << 2) |
                   (send_bit(r.x[3] >> 8, v4[it].w, a.c, a.eps_b) << 3);
-            const int64_t valid = a.P - e;  // parameters past P are never sent
-            if (valid < 4) nib &= (1u << valid) - 1u;
+            if (!FULL) {
+                const int64_t valid = a.P - e;  // parameters past P are never sent
+                if (valid < 4) nib &= (1u << valid) - 1u;
+            }
         }
         cnt += __popc(nib);
         // Eight lanes' nibbles form one 32-bit mask word (32 consecutive parameters).
@@ -85,6 +88,16 @@ __global__ void __launch_bounds__(kSelectThreads) bfasgd_mask_kernel(const __gri
         for (int w = 0; w < kWarps; ++w) t += warp_cnt[w];
         a.tile_count[blockIdx.x] = t;
     }
+}
+
+// Full tiles (all but perhaps the last) skip the per-quad bounds checks.
+__global__ void __launch_bounds__(kSelectThreads) bfasgd_mask_kernel(const __grid_constant__ SelectArgs a) {
+    pdl_wait();
+    pdl_trigger();
+    if ((int64_t)(blockIdx.x + 1) * kSelectTile <= a.P)
+        mask_tile<true>(a);
+    else
+        mask_tile<false>(a);
 }
 
 constexpr int kScanThreads = 1024;
@@ -145,32 +158,27 @@ __global__ void __launch_bounds__(kScanThreads) bfasgd_scan_kernel(const __grid_
     if (tid == kScanThreads - 1) *a.count = warp_sum[kScanThreads / 32 - 1];
 }
 
-__global__ void __launch_bounds__(kSelectThreads) bfasgd_compact_kernel(const __grid_constant__ SelectArgs a) {
+// Per warp and pass, the kept (index, value) pairs are first put in rank
+// order in shared memory, then written to idx and val by consecutive lanes
+// (coalesced), instead of each lane storing its own pairs at scattered ranks.
+constexpr int kPassParams = 128;
+
+template <bool FULL>
+__device__ __forceinline__ void compact_tile(const SelectArgs& a, uint2* stage) {
     __shared__ int32_t warp_cnt[kWarps];
-    pdl_wait();
-    pdl_trigger();
     const int lane = threadIdx.x & 31;
     const int warp = threadIdx.x >> 5;
     const int64_t tile_start = (int64_t)blockIdx.x * kSelectTile;
     const int64_t warp_start = tile_start + (int64_t)warp * kWarpSpan;
     // Lane l holds the mask word of parameters warp_start + 32 l .. + 31.  The
-    // word, the tile's output base and the gradient quads are all loaded
-    // before anything waits on them.
+    // word, the tile's output base and the value quads are all loaded before
+    // anything waits on them.
     const uint32_t word = a.mask[(warp_start >> 5) + lane];
     const int64_t tile_out = a.tile_base[blockIdx.x];
     float4 g4[kIters];
 #pragma unroll
-    for (int it = 0; it < kIters; ++it) {
-        const int64_t e = warp_start + it * 128 + 4 * lane;
-        if (e + 3 < a.P) {
-            g4[it] = __ldcs(reinterpret_cast<const float4*>(a.values + e));
-        } else {
-            float t[4] = {0.f, 0.f, 0.f, 0.f};
-            for (int j = 0; j < 4; ++j)
-                if (e + j < a.P) t[j] = a.values[e + j];
-            g4[it] = make_float4(t[0], t[1], t[2], t[3]);
-        }
-    }
+    for (int it = 0; it < kIters; ++it)
+        g4[it] = load_quad<FULL>(a.values, warp_start + it * kPassParams + 4 * lane, a.P);
     const int c = __popc(word);
     int incl = c;
 #pragma unroll
@@ -178,33 +186,49 @@ __global__ void __launch_bounds__(kSelectThreads) bfasgd_compact_kernel(const __
         const int y = __shfl_up_sync(kFull, incl, off);
         if (lane >= off) incl += y;
     }
-    const int excl = incl - c;
+    const int excl = incl - c;  // rank of this word's first kept entry in the warp's span
     if (lane == 31) warp_cnt[warp] = incl;
     __syncthreads();
     int64_t out = tile_out;
     for (int w = 0; w < warp; ++w) out += warp_cnt[w];
+    int32_t* idx_w = a.idx + out;
+    float* val_w = a.val + out;
+    const int32_t e_lane = (int32_t)(warp_start + 4 * lane);  // P < 2^31
+    const int sh = 4 * (lane & 7);
 #pragma unroll
     for (int it = 0; it < kIters; ++it) {
-        // This lane's quad lies in word (4 it + lane / 8), bits 4 (lane mod 8) .. +3.
+        // This lane's quad lies in word (4 it + lane / 8), bits sh .. sh + 3.
         const int owner = it * 4 + (lane >> 3);
         const uint32_t w = __shfl_sync(kFull, word, owner);
         const int wbase = __shfl_sync(kFull, excl, owner);
-        const int sh = 4 * (lane & 7);
+        const int pass_base = __shfl_sync(kFull, excl, it * 4);
+        const int pass_end = __shfl_sync(kFull, incl, it * 4 + 3);
         const uint32_t nib = (w >> sh) & 0xFu;
-        if (nib != 0) {
-            const int64_t e = warp_start + it * 128 + 4 * lane;
-            const float g[4] = {g4[it].x, g4[it].y, g4[it].z, g4[it].w};
-            int64_t pos = out + wbase + __popc(w & ((1u << sh) - 1u));
+        int r = wbase - pass_base + __popc(w & ((1u << sh) - 1u));
+        const int32_t e = e_lane + it * kPassParams;
+        const uint32_t g[4] = {__float_as_uint(g4[it].x), __float_as_uint(g4[it].y),
+                               __float_as_uint(g4[it].z), __float_as_uint(g4[it].w)};
 #pragma unroll
-            for (int j = 0; j < 4; ++j) {
-                if ((nib >> j) & 1u) {
-                    a.idx[pos] = (int32_t)(e + j);
-                    a.val[pos] = g[j];
-                    ++pos;
-                }
-            }
+        for (int j = 0; j < 4; ++j)
+            if ((nib >> j) & 1u) stage[r++] = make_uint2((uint32_t)(e + j), g[j]);
+        __syncwarp();
+        for (int k = lane; k < pass_end - pass_base; k += 32) {
+            const uint2 pr = stage[k];
+            idx_w[pass_base + k] = (int32_t)pr.x;
+            val_w[pass_base + k] = __uint_as_float(pr.y);
         }
+        __syncwarp();
     }
+}
+
+__global__ void __launch_bounds__(kSelectThreads) bfasgd_compact_kernel(const __grid_constant__ SelectArgs a) {
+    __shared__ uint2 stage[kWarps][kPassParams];
+    pdl_wait();
+    pdl_trigger();
+    if ((int64_t)(blockIdx.x + 1) * kSelectTile <= a.P)
+        compact_tile<true>(a, stage[threadIdx.x >> 5]);
+    else
+        compact_tile<false>(a, stage[threadIdx.x >> 5]);
 }
 
 }  // namespace

@@ -75,3 +75,68 @@ def test_noalloc_allocates_nothing_and_rejects_oversize():
     assert f.bfasgd_select_compact_noalloc(big, *args) == f.EINVAL
     assert "static scratch" in f.fasgd_last_error(None)
     assert f.bfasgd_select_compact_noalloc(0, *args) == f.EINVAL
+
+
+def test_noalloc_sizes_in_turn_match_oracle():
+    """Calls of different sizes share the one scratch array: every call must
+    see only its own tile status words, whatever an earlier, larger or
+    smaller call left there."""
+    import torch
+    import oracle
+    f = _f()
+    stream = torch.cuda.current_stream().cuda_stream
+    for k, P in enumerate([1 << 24, 5, 8193, (1 << 24) - 3, 100_000, 8192]):
+        rng = np.random.default_rng(1000 + k)
+        g = (rng.standard_normal(P) * 0.1).astype(np.float32)
+        v = (10 ** rng.uniform(-1, 2, P)).astype(np.float32)
+        c = np.float32(30.0)
+        g_t, v_t = torch.from_numpy(g).cuda(), torch.from_numpy(v).cuda()
+        idx, val, n = _outputs(P, "cuda")
+        rc = f.bfasgd_select_compact_noalloc(P, g_t.data_ptr(), v_t.data_ptr(), float(c), EPS_B,
+                                             SEED, 3, k, idx.data_ptr(), val.data_ptr(),
+                                             n.data_ptr(), stream)
+        assert rc == f.OK, f.fasgd_last_error(None)
+        torch.cuda.synchronize()
+        oi, ov = oracle.select(g, v, c, EPS_B, SEED, 3, k)
+        m = int(n.item())
+        assert m == oi.size, (P, m, oi.size)
+        assert np.array_equal(idx[:m].cpu().numpy(), oi)
+        assert np.array_equal(val[:m].cpu().numpy().view(np.int32), ov.view(np.int32))
+
+
+def test_noalloc_graph_replays_match_eager():
+    """A captured call replayed on new inputs gives what an eager call with the
+    same counter gives: nothing a call depends on is left behind in the
+    scratch array or fixed in the captured launches beyond their arguments."""
+    import torch
+    f = _f()
+    P = 200_003
+    g = torch.zeros(P, device="cuda")
+    v = torch.ones(P, device="cuda")
+    gi, gv, gn = _outputs(P, "cuda")
+    ei, ev, en = _outputs(P, "cuda")
+    c, client, push_no = 12.0, 4, 9
+
+    def call(i, vv, nn, stream):
+        return f.bfasgd_select_compact_noalloc(P, g.data_ptr(), v.data_ptr(), c, EPS_B, SEED,
+                                               client, push_no, i.data_ptr(), vv.data_ptr(),
+                                               nn.data_ptr(), stream)
+
+    assert call(ei, ev, en, torch.cuda.current_stream().cuda_stream) == f.OK  # address look-up
+    torch.cuda.synchronize()
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph):
+        assert call(gi, gv, gn, torch.cuda.current_stream().cuda_stream) == f.OK
+    torch.cuda.synchronize()
+    for r in range(4):
+        gen = torch.Generator(device="cuda").manual_seed(r)
+        g.copy_(torch.randn(P, device="cuda", generator=gen) * 0.1)
+        v.copy_(torch.rand(P, device="cuda", generator=gen) * 100 + 0.1)
+        graph.replay()
+        torch.cuda.synchronize()
+        assert call(ei, ev, en, torch.cuda.current_stream().cuda_stream) == f.OK
+        torch.cuda.synchronize()
+        m = int(en.item())
+        assert int(gn.item()) == m and 0 < m < P, (r, int(gn.item()), m)
+        assert torch.equal(gi[:m], ei[:m])
+        assert torch.equal(gv[:m].view(torch.int32), ev[:m].view(torch.int32))
