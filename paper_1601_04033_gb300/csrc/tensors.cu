@@ -47,6 +47,17 @@ namespace {
 
 constexpr int kItemThreads = 256;
 constexpr unsigned kFull = 0xffffffffu;
+constexpr int kTermsPerThread = 2;  // budget terms per thread and search round
+
+// Exact sum over the warp of one 64-bit value per lane, from three 32-bit
+// hardware reductions of 21-, 21- and 22-bit pieces (a sum of 32 pieces
+// stays below 2^27, so none of them wraps).  The total must fit in 64 bits.
+__device__ __forceinline__ unsigned long long warp_sum_u64(unsigned long long x) {
+    const unsigned p0 = __reduce_add_sync(kFull, (unsigned)(x & 0x1fffffu));
+    const unsigned p1 = __reduce_add_sync(kFull, (unsigned)((x >> 21) & 0x1fffffu));
+    const unsigned p2 = __reduce_add_sync(kFull, (unsigned)(x >> 42));
+    return (unsigned long long)p0 + ((unsigned long long)p1 << 21) + ((unsigned long long)p2 << 42);
+}
 
 // The sum of v over one item as a float-float pair, the same bits wherever
 // it is formed (the partial kernel, or the apply kernel after it rewrote the
@@ -107,10 +118,11 @@ __global__ void __launch_bounds__(kItemThreads) tensor_partial_kernel(const __gr
 
 // floor(size * q * 2^32) for q = fl(a / fl(a + x)), a = fl(vbar + eps_b),
 // exactly: q = M 2^e with M its 24-bit significand, so the term is
-// size * M shifted by e + 32 (q <= 1 keeps it at most size * 2^32).
-__device__ __forceinline__ uint64_t budget_term(int32_t size, float vbar, float eps_b, float x) {
-    const float a = __fadd_rn(vbar, eps_b);
-    if (!(a > 0.f) || a == __int_as_float(0x7f800000)) return 0;
+// size * M shifted by e + 32 (q <= 1 keeps it at most size * 2^32).  The
+// caller passes a = 0 where fl(vbar + eps_b) is not a positive finite
+// number: such a tensor's term is 0.
+__device__ __forceinline__ uint64_t budget_term(int32_t size, float a, float x) {
+    if (!(a > 0.f)) return 0;
     const float q = __fdiv_rn(a, __fadd_rn(a, x));
     const uint32_t bits = __float_as_uint(q);     // q in [0, 1]: sign bit clear
     if (bits == 0) return 0;
@@ -147,46 +159,64 @@ __device__ __forceinline__ long long warm_candidate(long long cp, int k, int m) 
 
 __global__ void __launch_bounds__(kTensorResolveThreads) budget_resolve_kernel(const __grid_constant__ TensorArgs a) {
     // Dynamic shared memory (tensor_resolve_smem): the item sums, the tensor
-    // sums, vbar_t, the item ranges, the sizes and the stale flags, each
-    // loaded once with all loads in flight together.
+    // sums, vbar_t, a_t, the item ranges, the sizes and the stale flags; the
+    // inputs are loaded once, four per thread in flight together.
     extern __shared__ __align__(16) unsigned char dsm[];
     float2* s_part = reinterpret_cast<float2*>(dsm);
     float2* s_sum = s_part + a.n_items;
     float* s_vbar = reinterpret_cast<float*>(s_sum + a.T);
-    int32_t* s_begin = reinterpret_cast<int32_t*>(s_vbar + a.T);
+    float* s_a = s_vbar + a.T;    // fl(vbar_t + eps_b), 0 where not positive and finite
+    int32_t* s_begin = reinterpret_cast<int32_t*>(s_a + a.T);
     int32_t* s_size = s_begin + a.T + 1;
     uint8_t* s_dirty = reinterpret_cast<uint8_t*>(s_size + a.T);
     __shared__ unsigned long long s_e[32];
+    __shared__ long long s_cand[32];   // this round's candidates (lanes >= ncand: hi)
     __shared__ long long s_lo, s_hi, s_cp;
     __shared__ unsigned long long s_count;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     pdl_wait();
     pdl_trigger();
-    // One pass of loads (every load of a thread issued before any store).
+    // Loads in passes of four per thread, every load of a pass issued before
+    // any of its stores to shared memory.
+    const long long cp_in = tid == 0 ? *a.c_prev : 0;
     const int nload = a.n_items > a.T + 1 ? a.n_items : a.T + 1;
-    for (int i = tid; i < nload; i += kTensorResolveThreads) {
-        float2 pv = make_float2(0.f, 0.f);
-        int32_t bg = 0, sz = 0;
-        uint8_t dt = 1;
-        float vb = 0.f;
-        if (i < a.n_items) pv = a.partial[i];
-        if (i <= a.T) bg = a.item_begin[i];
-        if (i < a.T) {
-            sz = a.sizes[i];
-            vb = a.vbar_cache[i];
-            if (!a.all_dirty) dt = a.dirty[i];
+    constexpr int kPass = 4;
+    for (int i0 = 0; i0 < nload; i0 += kPass * kTensorResolveThreads) {
+        float2 pv[kPass];
+        int32_t bg[kPass], sz[kPass];
+        uint8_t dt[kPass];
+        float vb[kPass];
+#pragma unroll
+        for (int u = 0; u < kPass; ++u) {
+            const int i = i0 + u * kTensorResolveThreads + tid;
+            pv[u] = make_float2(0.f, 0.f);
+            bg[u] = 0;
+            sz[u] = 0;
+            dt[u] = 1;
+            vb[u] = 0.f;
+            if (i < a.n_items) pv[u] = a.partial[i];
+            if (i <= a.T) bg[u] = a.item_begin[i];
+            if (i < a.T) {
+                sz[u] = a.sizes[i];
+                vb[u] = a.vbar_cache[i];
+                if (!a.all_dirty) dt[u] = a.dirty[i];
+            }
         }
-        if (i < a.n_items) s_part[i] = pv;
-        if (i <= a.T) s_begin[i] = bg;
-        if (i < a.T) {
-            s_size[i] = sz;
-            s_vbar[i] = vb;
-            s_dirty[i] = dt;
+#pragma unroll
+        for (int u = 0; u < kPass; ++u) {
+            const int i = i0 + u * kTensorResolveThreads + tid;
+            if (i < a.n_items) s_part[i] = pv[u];
+            if (i <= a.T) s_begin[i] = bg[u];
+            if (i < a.T) {
+                s_size[i] = sz[u];
+                s_vbar[i] = vb[u];
+                s_dirty[i] = dt[u];
+            }
         }
     }
     if (tid == 0) {
         s_count = 0;
-        s_cp = *a.c_prev;
+        s_cp = cp_in;
     }
     __syncthreads();
     // vbar_t of every tensor whose v changed since it was last formed: warp
@@ -204,67 +234,120 @@ __global__ void __launch_bounds__(kTensorResolveThreads) budget_resolve_kernel(c
     }
     __syncthreads();
     for (int t = tid; t < a.T; t += kTensorResolveThreads) {
-        if (!s_dirty[t]) continue;
-        const float2 p = s_sum[t];
-        const float vb = ff_div_int(p.x, p.y, s_size[t]);
-        s_vbar[t] = vb;
-        a.vbar_cache[t] = vb;
-        a.dirty[t] = 0;
+        float vb = s_vbar[t];
+        if (s_dirty[t]) {
+            const float2 p = s_sum[t];
+            vb = ff_div_int(p.x, p.y, s_size[t]);
+            s_vbar[t] = vb;
+            a.vbar_cache[t] = vb;
+            a.dirty[t] = 0;
+        }
+        const float at = __fadd_rn(vb, a.eps_b);
+        s_a[t] = at > 0.f && at != __int_as_float(0x7f800000) ? at : 0.f;
     }
     __syncthreads();
     // Invariant: E(lo) > limit >= E(hi) (lo = -1 stands below 0, hi = +inf
     // has E = 0); c = hi once they are adjacent.  2^m is chosen so that a
-    // thread takes about two tensors per candidate: the work of a round
-    // grows with the number of candidates times T, the number of rounds only
-    // with its log.
+    // thread takes at most kTermsPerThread tensors per round: more candidates
+    // per round mean fewer rounds, but every round's terms are issued by the
+    // one SM.  Warp 0 places the candidates and takes each round's decision;
+    // the other warps only evaluate terms.
     int m = 5;
-    while (m > 1 && (a.T << m) > 2 * kTensorResolveThreads) --m;
+    while (m > 1 && (a.T << m) > kTermsPerThread * kTensorResolveThreads) --m;
     const int gwarps = 32 >> m;                      // warps per group; the last group idles
     const int group = warp / gwarps;
     const int gthread = tid - group * gwarps * 32;
     const int gsize = gwarps * 32;
     const int ncand = (1 << m) - 1;
-    const long long cp = s_cp;
-    const bool warm = m >= 3 && cp >= 0 && cp <= 0x7f800000;
+    // Warp 0 also keeps E at both ends of the interval (E(+inf) = 0; E at
+    // lo = -1 unknown).  Once both are known, the next round's candidates
+    // sit on a ladder (0, +-1, +-4, +-16, ...) around the point where the
+    // straight line between them crosses the limit: E is smooth and the
+    // interval short, so the crossing is usually within an ulp or two.  A
+    // round placed that way that shrinks the interval less than an even
+    // split would is followed by an even split, so the search always ends.
+    long long w_elo = -1, w_ehi = 0, w_prev_span = 0;   // E(lo) (-1: unknown), E(hi)
+    bool w_interp = false;
+    if (warp == 0) {
+        const long long cp = s_cp;
+        const bool warm = m >= 3 && cp >= 0 && cp <= 0x7f800000;
+        long long cand = 0x7f800000;
+        if (lane < ncand) cand = warm ? warm_candidate(cp, lane, m) : candidate(-1, 0x7f800000, lane, m);
+        s_cand[lane] = cand < 0x7f800000 ? cand : 0x7f800000;
+        if (lane == 0) {
+            s_lo = -1;
+            s_hi = 0x7f800000;
+        }
+    }
+    __syncthreads();
     long long lo = -1, hi = 0x7f800000;
     for (int round = 0; round < 64 && hi - lo > 1; ++round) {
-        const bool w0 = warm && round == 0;
         unsigned long long e = 0;
-        if (group < ncand) {
-            const long long cand = w0 ? warm_candidate(cp, group, m) : candidate(lo, hi, group, m);
-            if (cand < hi) {
-                const float x = __uint_as_float((uint32_t)cand);
-                for (int t = gthread; t < a.T; t += gsize)
-                    e += budget_term(s_size[t], s_vbar[t], a.eps_b, x);
+        const long long cand = s_cand[group < 32 ? group : 31];
+        if (group < ncand && cand < hi) {
+            // Two tensors at a time with separate sums, so that the two
+            // divisions overlap.
+            const float x = __uint_as_float((uint32_t)cand);
+            unsigned long long e1 = 0;
+            int t = gthread;
+            for (; t + gsize < a.T; t += 2 * gsize) {
+                e += budget_term(s_size[t], s_a[t], x);
+                e1 += budget_term(s_size[t + gsize], s_a[t + gsize], x);
             }
+            if (t < a.T) e += budget_term(s_size[t], s_a[t], x);
+            e += e1;
         }
-#pragma unroll
-        for (int off = 16; off > 0; off >>= 1) e += __shfl_xor_sync(kFull, e, off);
+        e = warp_sum_u64(e);
         if (lane == 0) s_e[warp] = e;
         __syncthreads();
         if (warp == 0) {
             // Lane k adds the partials of group k and tests candidate k; E is
             // non-increasing and the candidates non-decreasing, so the passing
-            // candidates are a suffix.
-            int ok = 1;
-            long long cand = hi;
-            if (lane < ncand) {
-                cand = w0 ? warm_candidate(cp, lane, m) : candidate(lo, hi, lane, m);
-                if (cand < hi) {
-                    unsigned long long sum = 0;
-                    for (int w = 0; w < gwarps; ++w) sum += s_e[lane * gwarps + w];
-                    ok = (long long)sum <= a.limit;
-                } else {
-                    cand = hi;
-                }
+            // candidates are a suffix.  Then the next round's candidates.
+            const long long ck = s_cand[lane];
+            const bool evaluated = lane < ncand && ck < hi;
+            long long ek = 0;
+            if (evaluated) {
+                unsigned long long sum = 0;
+                for (int w = 0; w < gwarps; ++w) sum += s_e[lane * gwarps + w];
+                ek = (long long)sum;
             }
+            const int ok = !evaluated || ek <= a.limit;
+            const long long cv = evaluated ? ck : hi;
             const unsigned pass = __ballot_sync(kFull, ok);   // lanes >= ncand pass
             const int first = __ffs(pass) - 1;
-            const long long c_first = __shfl_sync(kFull, cand, first);
-            const long long c_prev = __shfl_sync(kFull, cand, first > 0 ? first - 1 : 0);
+            const long long c_first = __shfl_sync(kFull, cv, first);
+            const long long e_first = __shfl_sync(kFull, ek, first);
+            const bool first_eval = __shfl_sync(kFull, evaluated, first);
+            const long long c_prev = __shfl_sync(kFull, cv, first > 0 ? first - 1 : 0);
+            const long long e_prev = __shfl_sync(kFull, ek, first > 0 ? first - 1 : 0);
+            const long long nlo = first > 0 ? c_prev : lo;
+            const long long nhi = c_first;
+            w_elo = first > 0 ? e_prev : w_elo;
+            w_ehi = first_eval ? e_first : w_ehi;
+            const long long span = nhi - nlo;
+            const bool interp = w_elo >= 0 && span > (1ll << m) &&
+                                (!w_interp || (span << m) <= w_prev_span);
+            long long nc;
+            if (interp) {
+                const double f = (double)(w_elo - a.limit) / (double)(w_elo - w_ehi);  // in (0, 1]
+                long long xs = nlo + (long long)(f * (double)span);
+                xs = xs <= nlo ? nlo + 1 : (xs >= nhi ? nhi - 1 : xs);
+                const int h = (1 << (m - 1)) - 1;
+                const int j = lane - h;
+                const int aj = j < 0 ? -j : j;
+                const long long off = aj == 0 ? 0 : 1ll << (2 * (aj - 1) < 40 ? 2 * (aj - 1) : 40);
+                nc = j < 0 ? xs - off : xs + off;
+                nc = nc <= nlo ? nlo + 1 : nc;
+            } else {
+                nc = candidate(nlo, nhi, lane, m);
+            }
+            s_cand[lane] = lane < ncand && nc < nhi ? nc : nhi;
+            w_interp = interp;
+            w_prev_span = span;
             if (lane == 0) {
-                s_hi = c_first;
-                s_lo = first > 0 ? c_prev : lo;
+                s_lo = nlo;
+                s_hi = nhi;
             }
         }
         __syncthreads();

@@ -20,8 +20,8 @@ inline int64_t tensor_chunk(int64_t P) {
 constexpr int kTensorResolveThreads = 1024;
 // Dynamic shared memory of the decision kernel for n_items items and T tensors.
 inline size_t tensor_resolve_smem(int32_t n_items, int32_t T) {
-    return (size_t)n_items * 8 + (size_t)T * 8 + (size_t)T * 4 + ((size_t)T + 1) * 4 +
-           (size_t)T * 4 + (size_t)T;
+    return (size_t)n_items * 8 + (size_t)T * 8 + (size_t)T * 4 + (size_t)T * 4 +
+           ((size_t)T + 1) * 4 + (size_t)T * 4 + (size_t)T;
 }
 struct TensorArgs {
     const float* v;               // the server's statistic, fp32[P]
