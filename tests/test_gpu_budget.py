@@ -133,6 +133,31 @@ def test_decisions_at_a_fixed_state_many_budgets():
     assert list(pair.srv.fetch_counts()) == pair.o.fetch_count
 
 
+@pytest.mark.parametrize("T", [2, 33, 600, 3000])
+def test_thresholds_jumping_between_calls(T):
+    """Budgets in shuffled order on one stream, tensor means spread over twelve
+    decades: the threshold jumps far between calls and E is far from linear
+    over the first brackets, so the search leans on its even-split fallback.
+    Every threshold and decision equals the oracle's (2, 33, 600 and 3000
+    tensors give 31, 7, 3 and 1 candidates per round)."""
+    torch = torch_cuda()
+    P = 200_003
+    sizes = streams.tensor_sizes(11, P, T)
+    pair = Pair(P, sizes)
+    rng = np.random.default_rng(T)
+    scale = np.repeat(10 ** rng.uniform(-6, 6, T), sizes).astype(np.float32)
+    v = (scale * rng.uniform(0.9, 1.1, P)).astype(np.float32)
+    z = np.zeros(P, np.float32)
+    pair.srv.set_state(*[torch.from_numpy(x).cuda() for x in (z, z, z, v)], 5)
+    pair.o.theta[:], pair.o.v[:], pair.o.T = z, v, 5
+    budgets = [P // 2, 3, P - 7, P // 50, 0, P // 5, 1, P // 3, 2 * P, P // 7, 100, P // 2]
+    for k, budget in enumerate(budgets):
+        copy = torch.zeros(P, device="cuda")
+        pair.srv.fetch_budget(1, copy, budget, pair.sent, pair.c, pair.count)
+        want = pair.o.fetch_budget(1, np.zeros(P, np.float32), budget)
+        pair.check_decision(pair.decision(), want, f"T={T} call {k} budget {budget}")
+
+
 def test_full_budget_is_the_dense_pass_bitwise():
     """budget >= P transmits every tensor (c = 0): the same bits as fasgd_push."""
     torch = torch_cuda()
