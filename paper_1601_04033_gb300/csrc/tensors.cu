@@ -281,7 +281,9 @@ __global__ void __launch_bounds__(kTensorResolveThreads) budget_resolve_kernel(c
     }
     __syncthreads();
     long long lo = -1, hi = 0x7f800000;
-    for (int round = 0; round < 64 && hi - lo > 1; ++round) {
+    // At most 31 even splits with one candidate each (2^31 patterns), each
+    // possibly preceded by one placed round: the cap is never reached.
+    for (int round = 0; round < 128 && hi - lo > 1; ++round) {
         unsigned long long e = 0;
         const long long cand = s_cand[group < 32 ? group : 31];
         if (group < ncand && cand < hi) {
