@@ -306,7 +306,7 @@ FASGD_API int bfasgd_message_vbar(fasgd_t* h, float* vbar_dev);
  * tensor t covers [o_t, o_t + sizes[t]), o_0 = 0, o_{t+1} = o_t + sizes[t].
  * sizes: host int64[T], each >= 1, summing to P; 1 <= T <= BFASGD_TMAX.
  * Requires an empty queue; waits for the handle's stream; allocates small
- * device tables (a few bytes per tensor and per 16,384 parameters).
+ * device tables (a few bytes per tensor and per 8,192 parameters).
  * Errors: EINVAL, EAGAIN, ENOMEM, ECUDA.
  */
 FASGD_API int bfasgd_set_tensors(fasgd_t* h, int32_t T, const int64_t* sizes);

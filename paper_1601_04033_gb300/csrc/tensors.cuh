@@ -15,7 +15,7 @@ struct TensorItem {
 };
 inline int64_t tensor_chunk(int64_t P) {
     const int64_t c = (P + 8191) / 8192;   // at most ~8192 items besides one per tensor
-    return c > 16384 ? c : 16384;
+    return c > 8192 ? c : 8192;
 }
 constexpr int kTensorResolveThreads = 1024;
 // Dynamic shared memory of the decision kernel for n_items items and T tensors.
