@@ -393,8 +393,11 @@ def run_bfasgd(args, w, world, rank, local):
     v_now = torch.empty(P, device=device)
     srv.get_state(None, None, None, v_now)
     v_host = v_now.cpu().numpy()
-    c_push = calibrate_c(v_host, w.send_frac)
-    c_fetch = calibrate_c(v_host, FETCH_FRACTION)
+    # Large P: calibrate on a strided sample of about 4M parameters (the measured
+    # send and fetch fractions are reported either way).
+    v_cal = v_host if P <= (1 << 25) else v_host[:: P // (1 << 22)]
+    c_push = calibrate_c(v_cal, w.send_frac)
+    c_fetch = calibrate_c(v_cal, FETCH_FRACTION)
     srv.set_hparams(0.95, 0.95, 1e-4, c_push, 1e-8, w.seed)
     srv.set_fetch_threshold(c_fetch)
     idx = torch.empty(P, dtype=torch.int32, device=device)
@@ -405,8 +408,11 @@ def run_bfasgd(args, w, world, rank, local):
     fcnt = torch.empty(1, dtype=torch.int64, device=device)
     counts = torch.zeros(args.steps, dtype=torch.int64, device=device)
     fcounts = torch.zeros(args.steps, dtype=torch.int64, device=device)
-    # Every client keeps its own (stale) copy of the parameters.
-    client_theta = torch.from_numpy(th0).to(device).repeat(w.lam, 1)
+    # Every client keeps its own (stale) copy of the parameters; at large P the
+    # clients share at most 32 GB of copies (client c uses copy c mod n_copies),
+    # which changes whose copy a scatter writes, not what it costs.
+    n_copies = int(min(w.lam, max(1, (32 << 30) // (4 * P))))
+    client_theta = torch.from_numpy(th0).to(device).repeat(n_copies, 1)
 
     def step(t, ev=None, i=None):
         """One B-FASGD exchange: client c pushes (decision + compaction, sparse
@@ -428,7 +434,8 @@ def run_bfasgd(args, w, world, rank, local):
         srv.fetch_compact(c, fidx, fval, n_fetch)
         if ev is not None:
             ev[3].record(stream)
-        fasgd.fetch_apply(client_theta[c], fidx, fval, n_dev=n_fetch, n_max=P, stream=stream)
+        fasgd.fetch_apply(client_theta[c % n_copies], fidx, fval, n_dev=n_fetch, n_max=P,
+                          stream=stream)
         if ev is not None:
             ev[4].record(stream)
 
@@ -492,6 +499,7 @@ def run_bfasgd(args, w, world, rank, local):
                    "K": 1, "variant": "b-fasgd", "c_push": c_push, "target_send_fraction": w.send_frac,
                    "c_fetch": c_fetch, "target_fetch_fraction": FETCH_FRACTION,
                    "step": "push select/compact + sparse apply + fetch select/compact + client scatter",
+                   "client_copies": n_copies,
                    "staleness": w.delay, "parallelism": f"param-shard{world}",
                    "l2": "inputs larger than L2, no flush"},
     }
@@ -753,7 +761,7 @@ def main():
         mode = "message"
     elif w.tensors:
         mode = "tensor"
-    elif w.send_frac is not None and args.workload == "bfasgd-25m":
+    elif w.send_frac is not None and w.K == 1:
         mode = "bfasgd"
     else:
         mode = "dense"

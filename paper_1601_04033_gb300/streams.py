@@ -84,6 +84,10 @@ WORKLOADS = {
     "fasgd-268m-k16": Workload("fasgd-268m-k16", 268_435_456, 256, 2_000, 0.001, 16,
                                (FASGD,), "pareto1.5", 4, s_lo=1e-5, s_hi=1.0, R=32,
                                send_frac=0.20),
+    # Per-parameter B-FASGD exchanges on the 2^28 shape.
+    "bfasgd-268m": Workload("bfasgd-268m", 268_435_456, 256, 2_000, 0.001, 1,
+                            (FASGD,), "pareto1.5", 4, s_lo=1e-5, s_hi=1.0, R=32,
+                            send_frac=0.20),
 }
 
 
