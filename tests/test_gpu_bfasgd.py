@@ -227,6 +227,43 @@ def test_bfasgd_full_size_25m_sampled():
 
 
 @pytest.mark.slow
+def test_bfasgd_full_size_2_28_sampled():
+    """The bench's 2^28 exchange shape (bfasgd-268m): select with a client's v
+    snapshot, then the sparse apply, for 4 pushes of 2 clients; every list
+    bit-exact, the state compared on 20,000 sampled parameters."""
+    import torch
+    w = W["bfasgd-268m"].replace(R=2)
+    P = w.P
+    pool = streams.gradient_pool(w, P)
+    th0 = streams.theta0(w, P)
+    vsnap = [streams.client_v_snapshot(w, c, P) for c in range(2)]
+    c_push = calibrate_c(vsnap[0][:: P // (1 << 22)], 0.2)
+    idx_s = streams.sample_indices(P, 20_000)
+    g = GpuRun(w, oracle.FASGD, P, pool, th0, c_push=c_push, seed=SEED)
+    o = OracleRun(w, oracle.FASGD, idx_s.size, np.ascontiguousarray(pool[:, idx_s]), th0[idx_s],
+                  c_push=c_push, seed=SEED)
+    pos = np.full(P, -1, np.int64)
+    pos[idx_s] = np.arange(idx_s.size)
+    counts = [0, 0]
+    for t in range(4):
+        c, s, j = t % 2, t % 2, max(0, t - 1)
+        gi, gv, m, (it, vt, nt) = _select_gpu(g.srv, c, g.pool[s], torch.from_numpy(vsnap[c]).cuda())
+        oi, ov = oracle.select(pool[s], vsnap[c], c_push, 1e-8, SEED, c, counts[c])
+        counts[c] += 1
+        assert 0.15 < m / P < 0.25
+        assert_bitwise(gi, oi, f"idx t={t}")
+        assert_bitwise(gv, ov, f"val t={t}")
+        g.srv.push_sparse(c, j, it, vt, n_dev=nt, n_max=P)
+        g.srv.apply_pending(1)
+        keep = pos[oi] >= 0
+        o.srv.push_sparse(c, j, pos[oi[keep]].astype(np.int32), ov[keep])
+        o.srv.apply_pending(1)
+    g.srv.sync()
+    gs = g.state()
+    compare_states([x[idx_s] for x in gs[:4]] + [gs[4]], o.state(), oracle.FASGD, "bfasgd 2^28")
+
+
+@pytest.mark.slow
 def test_select_max_p():
     """P = 2^31 - 1, the largest P int32 indices allow: c = 0 keeps every index
     (the last one is 2^31 - 2), c = inf keeps none, and at a 20% threshold every
