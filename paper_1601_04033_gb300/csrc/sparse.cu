@@ -109,6 +109,8 @@ cudaError_t launch_rule(const SparseArgs& a, int num_sms, cudaStream_t stream) {
     return launch_pdl(fasgd_sparse_kernel<RULE, EXACT>, (unsigned)want, kSparseThreads, 0, stream, a);
 }
 
+constexpr int kScatterUnroll = 8;
+
 // Client side of a B-FASGD fetch: theta[idx[i]] = val[i] for i < count.
 // Indices come from one compaction, so they are distinct and no two threads
 // write the same parameter; an index outside [0, P) is skipped and flagged.
@@ -124,21 +126,40 @@ __global__ void __launch_bounds__(kSparseThreads) fetch_scatter_kernel(const __g
             count = c < 0 ? 0 : a.count_max;
         }
     }
-    const int64_t stride = (int64_t)gridDim.x * kSparseThreads;
-    for (int64_t i = (int64_t)blockIdx.x * kSparseThreads + threadIdx.x; i < count; i += stride) {
-        const int32_t p = a.idx[i];
-        if (p < 0 || (int64_t)p >= a.P) {
-            if (a.err != nullptr) atomicOr(a.err, 2);
-            continue;
+    // kScatterUnroll entries per thread per step (consecutive lanes, coalesced
+    // list loads), every load of a step issued before its stores.
+    const int64_t span = (int64_t)kSparseThreads * kScatterUnroll;
+    for (int64_t base = (int64_t)blockIdx.x * span; base < count; base += (int64_t)gridDim.x * span) {
+        int32_t p[kScatterUnroll];
+        float x[kScatterUnroll];
+#pragma unroll
+        for (int k = 0; k < kScatterUnroll; ++k) {
+            const int64_t i = base + k * kSparseThreads + threadIdx.x;
+            p[k] = 0;
+            x[k] = 0.f;
+            if (i < count) {
+                p[k] = a.idx[i];
+                x[k] = a.val[i];
+            }
         }
-        a.theta[p] = a.val[i];
+#pragma unroll
+        for (int k = 0; k < kScatterUnroll; ++k) {
+            const int64_t i = base + k * kSparseThreads + threadIdx.x;
+            if (i >= count) continue;
+            if (p[k] < 0 || (int64_t)p[k] >= a.P) {
+                if (a.err != nullptr) atomicOr(a.err, 2);
+                continue;
+            }
+            a.theta[p[k]] = x[k];
+        }
     }
 }
 
 }  // namespace
 
 cudaError_t launch_scatter(const ScatterArgs& a, int num_sms, cudaStream_t stream) {
-    int64_t want = (a.count_max + kSparseThreads - 1) / kSparseThreads;
+    const int64_t per_block = (int64_t)kSparseThreads * kScatterUnroll;
+    int64_t want = (a.count_max + per_block - 1) / per_block;
     const int64_t cap = (int64_t)(num_sms > 0 ? num_sms : 1) * 8;
     if (want > cap) want = cap;
     if (want < 1) want = 1;
