@@ -103,6 +103,17 @@ def peaks():
         return FALLBACK_HBM_GBS, "fallback"
 
 
+def physical(roofline: dict) -> dict:
+    """Add the DRAM bandwidth the ncu traffic of one launch implies at the
+    live launch time, beside the algorithmic figure (when traffic is known)."""
+    t, ms = roofline.get("traffic"), roofline.get("launch_ms")
+    if t and ms:
+        gbs = t / (ms / 1e3) / 1e9
+        roofline["traffic_gbs"] = round(gbs, 1)
+        roofline["traffic_frac"] = round(gbs / roofline["peak"], 4)
+    return roofline
+
+
 def nominal(achieved: float) -> dict:
     """The same achieved bandwidth against the GB300's nominal HBM3e figure."""
     return {"nominal_peak": NOMINAL_HBM_GBS, "frac_nominal": round(achieved / NOMINAL_HBM_GBS, 4)}
@@ -809,7 +820,7 @@ def main():
                 "steps": args.steps, "warmup": args.warmup, "ms_per_step": res["ms_per_step"],
                 "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
                 "dtype": "f32", "data": "synthetic", "config": res["config"],
-                "roofline": res["roofline"], "cpu_baseline": cpu, "e2e": res["e2e"],
+                "roofline": physical(res["roofline"]), "cpu_baseline": cpu, "e2e": res["e2e"],
                 "clocks": res["clocks"], "gpu_launches": res["gpu_launches"],
                 "pushes_per_s": res["pushes_per_s"]}
         for k in ("hbm_gbs_step", "sent_fraction", "fetched_fraction", "sent_updates_per_s"):
