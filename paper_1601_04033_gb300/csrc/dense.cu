@@ -29,6 +29,8 @@
 // own copies in flight, and returns.  Elements are independent, so the
 // result does not depend on the grid or on which path handled an element.
 
+#include <atomic>
+
 #include "kernels.cuh"
 #include "twosum.cuh"
 #include "update.cuh"
@@ -368,13 +370,18 @@ cudaError_t launch_ch(const DenseArgs& a, int num_sms, cudaStream_t stream) {
     ring.stages = (kSmemBudget - 2 * kMaxStages * 8) / kStageBytes;
     if (ring.stages > kMaxStages) ring.stages = kMaxStages;
     const size_t smem = (size_t)ring.stages * kStageBytes + 2 * ring.stages * sizeof(uint64_t);
-    static bool configured = false;  // per instantiation
-    if (!configured) {
-        cudaError_t st = cudaFuncSetAttribute(fasgd_dense_kernel<RULE, ARITH, CH, SUMS>,
-                                              cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                              kSmemBudget);
+    // The shared-memory limit is a per-device attribute of the kernel: set it
+    // once per device (bit d of the mask) and instantiation.
+    static std::atomic<uint64_t> configured{0};
+    int dev = 0;
+    cudaError_t st = cudaGetDevice(&dev);
+    if (st != cudaSuccess) return st;
+    const uint64_t bit = dev < 64 ? 1ull << dev : 0;
+    if (bit == 0 || !(configured.load(std::memory_order_acquire) & bit)) {
+        st = cudaFuncSetAttribute(fasgd_dense_kernel<RULE, ARITH, CH, SUMS>,
+                                  cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBudget);
         if (st != cudaSuccess) return st;
-        configured = true;
+        configured.fetch_or(bit, std::memory_order_acq_rel);
     }
     const int64_t ntiles = a.P / kTile;
     int64_t grid = ntiles < num_sms ? ntiles : num_sms;  // one block per SM (shared-memory bound)

@@ -11,6 +11,8 @@
 // index and value loads are coalesced and four gathers per array are in
 // flight per thread.
 
+#include <atomic>
+
 #include "kernels.cuh"
 #include "pdl.cuh"
 #include "update.cuh"
@@ -93,12 +95,15 @@ __global__ void __launch_bounds__(kSparseThreads) fasgd_sparse_kernel(const __gr
 
 template <int RULE, bool EXACT>
 cudaError_t launch_rule(const SparseArgs& a, int num_sms, cudaStream_t stream) {
-    static int blocks_per_sm = 0;
+    // Resident blocks per SM, looked up once (the grid is only capped by it).
+    static std::atomic<int> cached{0};
+    int blocks_per_sm = cached.load(std::memory_order_relaxed);
     if (blocks_per_sm == 0) {
         cudaError_t st = cudaOccupancyMaxActiveBlocksPerMultiprocessor(
             &blocks_per_sm, fasgd_sparse_kernel<RULE, EXACT>, kSparseThreads, 0);
         if (st != cudaSuccess) return st;
         if (blocks_per_sm < 1) blocks_per_sm = 1;
+        cached.store(blocks_per_sm, std::memory_order_relaxed);
     }
     // Enough warps for the host-side bound on the count, at most one full wave.
     const int64_t per_block = (int64_t)kSparseThreads * kUnroll;
