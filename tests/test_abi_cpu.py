@@ -69,3 +69,62 @@ def test_host_side_argument_checks(binding):
     assert f.fasgd_sync(None) == f.EINVAL
     assert f.fasgd_timestamp(None) == -1 and f.fasgd_pending(None) == -1
     f.fasgd_destroy(None)
+
+
+HANDLELESS = {"bfasgd_fetch_apply", "fasgd_sim_quadratic_grad", "fasgd_sim_quadratic_loss",
+              "bfasgd_select_compact_noalloc", "fasgd_last_error", "fasgd_destroy",
+              "fasgd_create"}
+
+
+def test_every_handle_call_rejects_a_null_handle(binding):
+    """Every entry point that takes a handle returns EINVAL (or -1 for the
+    introspection calls) for NULL, before it reads any other argument."""
+    f = binding
+    for name, (res, argtypes) in f.SIGNATURES.items():
+        if name in HANDLELESS:
+            continue
+        args = [None if t in (ctypes.c_void_p,) or hasattr(t, "contents") or
+                t.__name__.startswith("LP_") else 0 for t in argtypes]
+        rc = getattr(f.LIB, name)(*args)
+        if res is ctypes.c_int64:
+            assert rc == -1, name
+        else:
+            assert rc == f.EINVAL, name
+
+
+def test_handleless_calls_check_their_arguments_on_the_host(binding):
+    f = binding
+    L = f.LIB
+    a16, a4 = 1 << 12, (1 << 12) + 4      # never dereferenced: rejected or a no-op first
+    # bfasgd_select_compact_noalloc(P, grad, v, c, eps_b, seed, client, push_no, idx, val, n, stream)
+    good = [1000, a16, a16, 1.0, 1e-8, 7, 0, 0, a16, a16, a16 + 64, None]
+    for k, bad in ((0, 0), (0, f.NOALLOC_PMAX + 1), (6, -1), (1, None), (1, a4), (2, None),
+                   (3, -1.0), (3, float("nan")), (4, float("inf")), (4, -1.0), (8, None),
+                   (9, None), (10, None), (10, a4)):
+        args = list(good)
+        args[k] = bad
+        assert L.bfasgd_select_compact_noalloc(*args) == f.EINVAL, (k, bad)
+        assert f.fasgd_last_error(None)
+    # bfasgd_fetch_apply(P, theta, idx, val, n_dev, n_max, stream, err)
+    good = [1000, a16, a16, a16, None, 0, None, None]
+    assert L.bfasgd_fetch_apply(*good) == f.OK       # nothing to apply: no device work
+    for k, bad in ((0, 0), (0, 1 << 31), (1, None), (5, -1), (5, 1001), (4, a4), (7, a4 + 2)):
+        args = list(good)
+        args[k] = bad
+        assert L.bfasgd_fetch_apply(*args) == f.EINVAL, (k, bad)
+    args = list(good)
+    args[5] = 10                                      # entries but no lists
+    args[2] = None
+    assert L.bfasgd_fetch_apply(*args) == f.EINVAL
+    # fasgd_sim_quadratic_grad(P, theta, h, star, sigma, seed, client, n, grad, stream)
+    good = [1000, a16, a16, a16, a16, 1, 0, 0, a16, None]
+    for k, bad in ((0, 0), (6, -1), (6, 1 << 30), (1, None), (2, a4), (4, None), (8, None)):
+        args = list(good)
+        args[k] = bad
+        assert L.fasgd_sim_quadratic_grad(*args) == f.EINVAL, (k, bad)
+    # fasgd_sim_quadratic_loss(P, theta, h, star, scratch, loss, stream)
+    good = [1000, a16, a16, a16, a16, a16 + 64, None]
+    for k, bad in ((0, 0), (1, None), (4, None), (4, a4), (5, None), (5, a4)):
+        args = list(good)
+        args[k] = bad
+        assert L.fasgd_sim_quadratic_loss(*args) == f.EINVAL, (k, bad)
