@@ -47,6 +47,7 @@ L2_BYTES = 129 * 1024 * 1024
 
 DENSE_KERNEL_SOURCES = ["paper_1601_04033_gb300/csrc/dense.cu",
                         "paper_1601_04033_gb300/csrc/update.cuh",
+                        "paper_1601_04033_gb300/csrc/wait.cuh",
                         "paper_1601_04033_gb300/csrc/kernels.cuh"]
 SPARSE_KERNEL_SOURCES = ["paper_1601_04033_gb300/csrc/select.cu",
                          "paper_1601_04033_gb300/csrc/sparse.cu",

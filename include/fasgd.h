@@ -376,6 +376,17 @@ FASGD_API int fasgd_set_fetch_counts(fasgd_t* h, const uint64_t* counts);
  */
 FASGD_API int fasgd_sync(fasgd_t* h);
 
+/*
+ * fasgd_selftest_wait_expiry -- exercise the failure path of the dense pass's
+ * copy pipeline (no counterpart in the paper): enqueue on the handle's
+ * stream one small kernel whose pipeline barrier never completes.  Its two
+ * bounded waits -- one thread and one whole warp, the forms the pass uses --
+ * each give up after about a second and raise device flag 8, so the next
+ * fasgd_sync returns FASGD_EDEVICE.  Changes no state; the handle stays
+ * usable.  Errors: EINVAL, ECUDA.
+ */
+FASGD_API int fasgd_selftest_wait_expiry(fasgd_t* h);
+
 /* Server timestamp T (pushes applied so far) and number of queued pushes. */
 FASGD_API int64_t fasgd_timestamp(const fasgd_t* h);
 FASGD_API int64_t fasgd_pending(const fasgd_t* h);

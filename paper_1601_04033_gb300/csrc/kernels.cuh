@@ -125,6 +125,8 @@ cudaError_t launch_sparse(const SparseArgs& a, int rule, bool exact, int num_sms
                           int64_t* launches);
 cudaError_t launch_select(const SelectArgs& a, cudaStream_t stream, int64_t* launches);
 cudaError_t launch_scatter(const ScatterArgs& a, int num_sms, cudaStream_t stream);
+// Self-test: bounded pipeline waits that can never complete (raise flag 8 in err).
+cudaError_t launch_wait_expiry(int32_t* err, cudaStream_t stream);
 cudaError_t launch_sim_grad(const SimGradArgs& a, int num_sms, cudaStream_t stream);
 cudaError_t launch_sim_loss(const SimLossArgs& a, cudaStream_t stream);
 

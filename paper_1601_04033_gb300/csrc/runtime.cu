@@ -1112,6 +1112,16 @@ int fasgd_sync(fasgd_t* h) {
     return FASGD_OK;
 }
 
+int fasgd_selftest_wait_expiry(fasgd_t* h) {
+    if (h == nullptr) return FASGD_EINVAL;
+    TraceRange trace("fasgd_selftest_wait_expiry");
+    DeviceGuard g(h->device);
+    cudaError_t st = fasgd::launch_wait_expiry(h->dev_err, h->stream);
+    if (st != cudaSuccess) return h->cuda_fail(st, "fasgd_selftest_wait_expiry");
+    ++h->launches;
+    return FASGD_OK;
+}
+
 int64_t fasgd_timestamp(const fasgd_t* h) { return h == nullptr ? -1 : h->T; }
 
 int64_t fasgd_pending(const fasgd_t* h) { return h == nullptr ? -1 : (int64_t)h->fifo.size(); }

@@ -45,6 +45,7 @@ SIGNATURES = {
     "fasgd_get_push_counts": (_i32, [_p, _p]),
     "fasgd_set_push_counts": (_i32, [_p, _p]),
     "fasgd_sync": (_i32, [_p]),
+    "fasgd_selftest_wait_expiry": (_i32, [_p]),
     "fasgd_timestamp": (_i64, [_p]),
     "fasgd_pending": (_i64, [_p]),
     "fasgd_kernel_launches": (_i64, [_p]),
@@ -220,6 +221,10 @@ def fasgd_set_push_counts(h, counts):
 
 def fasgd_sync(h):
     return LIB.fasgd_sync(h)
+
+
+def fasgd_selftest_wait_expiry(h):
+    return LIB.fasgd_selftest_wait_expiry(h)
 
 
 def fasgd_timestamp(h):
@@ -420,6 +425,10 @@ class Server:
 
     def sync(self):
         self._check(fasgd_sync(self.h))
+
+    def selftest_wait_expiry(self):
+        """Enqueue the pipeline-wait expiry self-test (the next sync reports EDEVICE)."""
+        self._check(fasgd_selftest_wait_expiry(self.h))
 
     @property
     def T(self) -> int:

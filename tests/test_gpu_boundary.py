@@ -113,3 +113,42 @@ def test_host_push_and_pull_match_device_path():
     assert e.value.code == f.EAGAIN
     b.srv.apply_pending(f.KMAX)
     b.srv.sync()
+
+
+def test_a_pipeline_wait_that_never_completes_is_reported():
+    """Failure detection without a fault: the dense pass's bounded pipeline
+    waits, run on a barrier nothing completes, give up after about a second,
+    raise flag 8, and fasgd_sync reports EDEVICE; the state is untouched and
+    the handle keeps working."""
+    import time
+    import torch
+    from paper_1601_04033_gb300 import fasgd
+    P = 10_000
+    srv = fasgd.Server(P, 2, 0.01, fasgd.FASGD)
+    srv.set_params(torch.linspace(-1, 1, P, device="cuda"))
+    g = torch.randn(P, device="cuda") * 0.01
+    srv.push(0, 0, g)
+    srv.apply_pending(1)
+    srv.sync()
+    before = [torch.empty(P, device="cuda") for _ in range(4)]
+    srv.get_state(*before)
+    launches = srv.launches
+    t0 = time.time()
+    srv.selftest_wait_expiry()
+    with pytest.raises(fasgd.FasgdError) as e:
+        srv.sync()
+    took = time.time() - t0
+    assert e.value.code == fasgd.EDEVICE
+    assert "flags 0x8 " in str(e.value)      # only the pipeline-wait flag
+    assert 0.9 < took < 60, took
+    assert srv.launches == launches + 1
+    after = [torch.empty(P, device="cuda") for _ in range(4)]
+    srv.get_state(*after)
+    for x, y in zip(before, after):
+        assert torch.equal(x, y)
+    srv.sync()                      # the flags were cleared
+    srv.push(1, 1, g)               # and the handle still applies pushes
+    srv.apply_pending(1)
+    srv.sync()
+    assert srv.T == 2
+    srv.close()
