@@ -787,8 +787,12 @@ def main():
                 "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
                 "ms_per_step": el * 1e3 / done, "higher_is_better": True, "scaling": "weak",
                 "vs_baseline": None, "dtype": "f32", "data": "synthetic",
-                "config": {"workload": w.name, "sample": f"first {P_s} parameters, K={w.K} "
-                           f"pushes per step", "oracle": "single-threaded C, fp32"},
+                "config": {"workload": w.name, "P_per_gpu": args.P or w.P,
+                           "P_total": (args.P or w.P) * args.gpus, "lambda": w.lam, "K": w.K,
+                           "variant": "fasgd", "alpha": w.alpha, "staleness": w.delay,
+                           "parallelism": f"param-shard{args.gpus}",
+                           "sample": f"first {P_s} parameters, K={w.K} pushes per step",
+                           "oracle": "single-threaded C, fp32"},
                 "cpu_baseline": {"value": rate, "unit": UNIT, "cores": 1, "kind": "oracle",
                                  "sample": f"{done} steps x K={w.K} pushes over {P_s} parameters"},
                 "e2e": {"value": rate, "unit": UNIT, "h2d_bytes_per_step": 0,
