@@ -196,24 +196,17 @@ uint32_t ora_draw(uint64_t seed, uint32_t client, uint64_t push_no, int64_t p)
  * Eq. 9 for one parameter, decided in fp32.  With a = fl(v + eps_b),
  * d = fl(a + c) and r = u / 2^24, and a, d > 0:
  *     r < 1 / (1 + c / a)  <=>  r < a / (a + c)  <=>  u * d < a * 2^24.
- * The product u * d (24 x 24 bits) is split without error into
- * prod + err (prod = fl(u*d), err = fma(u, d, -prod)), so the strict
- * comparison is exact: below when prod < A, or prod == A and err < 0.
+ * Both sides are formed in fp64, where they are exact: u has 24 bits and d
+ * a 24-bit significand, so u * d has at most 48; a * 2^24 is a power-of-two
+ * scaling, far inside fp64's exponent range.  (d = +inf never sends: the
+ * product is +inf, or NaN for u = 0, and neither is below a finite bound.)
  * Returns 1 to transmit, 0 to drop.
  */
 int ora_decide(uint32_t u, float v, float c, float eps_b)
 {
     float a = v + eps_b;
     float d = a + c;
-    float uf = (float)u;
-    float prod = uf * d;
-    float err = fmaf(uf, d, -prod);
-    float A = a * 16777216.0f;
-    if (prod < A)
-        return 1;
-    if (prod == A && err < 0.0f)
-        return 1;
-    return 0;
+    return (double)u * (double)d < (double)a * 16777216.0;
 }
 
 /*
@@ -267,10 +260,136 @@ void ora_fetch_apply(float *theta_client, int64_t count, const int32_t *idx, con
 }
 
 /*
+ * Exact means, rounded once to fp32 (the statistic of the per-message and
+ * per-tensor rules below).
+ *
+ * Every finite double is an integer multiple of 2^-1074 (its smallest
+ * subnormal), and so is every float, so a sum of them is an integer number
+ * of those units and can be formed with no rounding at all in a long
+ * fixed-point accumulator (a Kulisch accumulator): ORA_LIMBS little-endian
+ * 32-bit words, enough for 2^31 terms below 2^1024, one for the positive
+ * and one for the negative terms.  The mean is the exact quotient of that
+ * integer by the count, rounded to the nearest fp32 (ties to even).
+ */
+#define ORA_LIMBS 68
+
+typedef struct {
+    uint32_t pos[ORA_LIMBS], neg[ORA_LIMBS];
+    int nan, pinf, ninf;
+} ora_exact_sum;
+
+static void ora_sum_clear(ora_exact_sum *s)
+{
+    memset(s, 0, sizeof *s);
+}
+
+/* w += m * 2^shift (m < 2^53, shift < 2046) */
+static void ora_acc_add(uint32_t *w, uint64_t m, int shift)
+{
+    int i = shift / 32, bit = shift % 32;
+    uint64_t lo = (m & 0xFFFFFFFFu) << bit;         /* < 2^63 */
+    uint64_t hi = (m >> 32) << bit;                 /* < 2^52 */
+    uint64_t c = (uint64_t)w[i] + (lo & 0xFFFFFFFFu);
+    w[i] = (uint32_t)c;
+    c = (c >> 32) + (uint64_t)w[i + 1] + (lo >> 32) + (hi & 0xFFFFFFFFu);
+    w[i + 1] = (uint32_t)c;
+    c = (c >> 32) + (uint64_t)w[i + 2] + (hi >> 32);
+    w[i + 2] = (uint32_t)c;
+    c >>= 32;
+    for (int k = i + 3; c != 0 && k < ORA_LIMBS; k++) {
+        c += w[k];
+        w[k] = (uint32_t)c;
+        c >>= 32;
+    }
+}
+
+/* Adds x exactly: a finite double is m 2^(E-1075) for a normal encoding
+ * (E = biased exponent, m = 2^52 + fraction) and fraction 2^-1074 for a
+ * subnormal one, i.e. m units of 2^-1074 shifted left by max(E - 1, 0). */
+static void ora_sum_add(ora_exact_sum *s, double x)
+{
+    uint64_t bits;
+    memcpy(&bits, &x, sizeof bits);
+    int neg = (int)(bits >> 63);
+    int E = (int)((bits >> 52) & 0x7FF);
+    uint64_t F = bits & (((uint64_t)1 << 52) - 1);
+    if (E == 0x7FF) {                                /* inf or NaN: IEEE rules */
+        if (F != 0)
+            s->nan = 1;
+        else if (neg)
+            s->ninf = 1;
+        else
+            s->pinf = 1;
+        return;
+    }
+    uint64_t m = E == 0 ? F : F | ((uint64_t)1 << 52);
+    ora_acc_add(neg ? s->neg : s->pos, m, E == 0 ? 0 : E - 1);
+}
+
+static int ora_acc_cmp(const uint32_t *a, const uint32_t *b)
+{
+    for (int k = ORA_LIMBS - 1; k >= 0; k--)
+        if (a[k] != b[k])
+            return a[k] < b[k] ? -1 : 1;
+    return 0;
+}
+
+/* The sum divided by count (1 <= count < 2^32), rounded to the nearest
+ * float, ties to even. */
+static float ora_sum_mean(const ora_exact_sum *s, int64_t count)
+{
+    if (s->nan || (s->pinf && s->ninf) || count < 1)
+        return NAN;
+    if (s->pinf)
+        return INFINITY;
+    if (s->ninf)
+        return -INFINITY;
+    /* |sum| = big - small, with the sign of the larger accumulator */
+    int c = ora_acc_cmp(s->pos, s->neg);
+    const uint32_t *big = c >= 0 ? s->pos : s->neg, *small = c >= 0 ? s->neg : s->pos;
+    uint32_t q[ORA_LIMBS];
+    int64_t borrow = 0;
+    for (int k = 0; k < ORA_LIMBS; k++) {
+        int64_t d = (int64_t)big[k] - (int64_t)small[k] - borrow;
+        borrow = d < 0;
+        q[k] = (uint32_t)(d + (borrow ? ((int64_t)1 << 32) : 0));
+    }
+    /* q <- floor(|sum| / count), r = the remainder (schoolbook, top down) */
+    uint64_t r = 0;
+    for (int k = ORA_LIMBS - 1; k >= 0; k--) {
+        uint64_t cur = (r << 32) | q[k];
+        q[k] = (uint32_t)(cur / (uint64_t)count);
+        r = cur % (uint64_t)count;
+    }
+    /* Bit length L of q; the mean is (q + r / count) 2^-1074.  Its fp32
+     * spacing is 2^(L - 1098) in the normal range and 2^-149 below it: in
+     * units of 2^-1074, 2^shift with shift = max(L - 24, 925). */
+    int L = 0;
+    for (int k = ORA_LIMBS - 1; k >= 0 && L == 0; k--)
+        for (int bit = 31; bit >= 0; bit--)
+            if ((q[k] >> bit) & 1u) {
+                L = 32 * k + bit + 1;
+                break;
+            }
+    int shift = L - 24 > 925 ? L - 24 : 925;
+    uint64_t mant = 0;                          /* q >> shift: at most 24 bits */
+    for (int bit = shift + 23; bit >= shift; bit--)
+        mant = (mant << 1) | ((q[bit / 32] >> (bit % 32)) & 1u);
+    int guard = (q[(shift - 1) / 32] >> ((shift - 1) % 32)) & 1u;
+    int sticky = r != 0;
+    for (int bit = 0; bit < shift - 1 && !sticky; bit++)
+        sticky = (q[bit / 32] >> (bit % 32)) & 1u;
+    if (guard && (sticky || (mant & 1u)))
+        mant++;
+    float mag = ldexpf((float)mant, shift - 1074);   /* exact, or inf past FLT_MAX */
+    return c >= 0 ? mag : -mag;
+}
+
+/*
  * The paper's literal B-FASGD (Sec. 2.3): one decision per transmission
  * opportunity, with v the mean over all parameters of the server's moving
- * averages.  ora_mean_v returns that mean, summed in fp64 in index order and
- * rounded once to fp32; the decision is Eq. 9 in fp32 (ora_decide) with a
+ * averages.  ora_mean_v returns that mean: the exact sum of v divided by P,
+ * rounded once to fp32.  The decision is Eq. 9 in fp32 (ora_decide) with a
  * draw from the message domain: word 0 of Philox4x32-10 at counter
  * (2^32 - 1, client + 2^31 * stream, n low, n high), top 24 bits (the
  * per-parameter draws never reach that first counter word, since
@@ -278,10 +397,11 @@ void ora_fetch_apply(float *theta_client, int64_t count, const int32_t *idx, con
  */
 float ora_mean_v(int64_t P, const REAL *v)
 {
-    double s = 0.0;
+    ora_exact_sum s;
+    ora_sum_clear(&s);
     for (int64_t p = 0; p < P; p++)
-        s += (double)v[p];
-    return (float)(s / (double)P);
+        ora_sum_add(&s, (double)v[p]);
+    return ora_sum_mean(&s, P);
 }
 
 uint32_t ora_draw_message(uint64_t seed, uint32_t stream, uint32_t client, uint64_t n)
@@ -344,8 +464,8 @@ double ora_sim_loss(int64_t P, const float *theta, const float *h, const float *
  *
  *   tensors    contiguous ranges [o_t, o_t + s_t) that partition [0, P),
  *              o_0 = 0, o_{t+1} = o_t + s_t, s_t >= 1;
- *   statistic  vbar_t = the mean of v over tensor t (fp64 sum in index
- *              order, rounded once to fp32), as the per-message rule uses
+ *   statistic  vbar_t = the mean of v over tensor t (exact sum, rounded
+ *              once to fp32), as the per-message rule uses
  *              the mean over all parameters;
  *   decision   Eq. 9 per tensor: transmit tensor t iff
  *              u_t / 2^24 < 1 / (1 + c / (vbar_t + eps_b))   (ora_decide);
@@ -373,15 +493,16 @@ double ora_sim_loss(int64_t P, const float *theta, const float *h, const float *
  *              reading as the per-parameter path).
  */
 
-/* vbar_t for every tensor: fp64 sum over the tensor in index order, rounded once. */
+/* vbar_t for every tensor: the exact mean over the tensor, rounded once. */
 void ora_tensor_means(int32_t T, const int64_t *sizes, const REAL *v, float *vbar)
 {
     int64_t off = 0;
     for (int32_t t = 0; t < T; t++) {
-        double s = 0.0;
+        ora_exact_sum s;
+        ora_sum_clear(&s);
         for (int64_t p = off; p < off + sizes[t]; p++)
-            s += (double)v[p];
-        vbar[t] = (float)(s / (double)sizes[t]);
+            ora_sum_add(&s, (double)v[p]);
+        vbar[t] = ora_sum_mean(&s, sizes[t]);
         off += sizes[t];
     }
 }

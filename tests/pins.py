@@ -299,11 +299,14 @@ def check_dense_equals_full_sparse(libs: Libs):
 # Eq. 9: the fp32 send decision against exact rational arithmetic
 # --------------------------------------------------------------------------
 def _exact_decide(u, v, c, eps_b):
-    a = np.float32(np.float32(v) + np.float32(eps_b))
-    d = np.float32(a + np.float32(c))
-    if not (np.isfinite(a) and np.isfinite(d)):
+    with np.errstate(over="ignore"):
+        a = np.float32(np.float32(v) + np.float32(eps_b))
+        d = np.float32(a + np.float32(c))
+    if not np.isfinite(a):
         return None
-    # u/2^24 < a/d  <=>  u*d < a*2^24   (a, d > 0)
+    if np.isinf(d):              # u/2^24 < a/inf = 0 never holds
+        return False
+    # u/2^24 < a/d  <=>  u*d < a*2^24   (d > 0)
     return Fraction(int(u)) * Fraction(float(d)) < Fraction(float(a)) * (1 << 24)
 
 
@@ -321,6 +324,23 @@ def check_decide_exact(libs: Libs):
         d = float(np.float32(np.float32(a) + np.float32(c)))
         if rng.random() < 0.5:      # aim at the threshold: ties and near-ties
             u = int(np.clip(round(a * 2 ** 24 / d) + int(rng.integers(-2, 3)), 0, 2 ** 24 - 1))
+        else:
+            u = int(rng.integers(0, 2 ** 24))
+        want = _exact_decide(u, v, c, eps_b)
+        got = oracle.decide(u, v, c, eps_b, lib=libs.f32)
+        assert got == want, (u, v, c, eps_b)
+    # The whole fp32 range: a and c from subnormal to near FLT_MAX, c = 0 and
+    # c = +inf, draws aimed at the threshold.
+    for _ in range(4000):
+        v = float(np.float32(2.0 ** rng.uniform(-149, 127.9)))
+        r = rng.random()
+        c = 0.0 if r < 0.1 else float("inf") if r < 0.15 else float(np.float32(2.0 ** rng.uniform(-149, 127.9)))
+        eps_b = float(np.float32(rng.choice([0.0, 1e-8, 2.0 ** -140])))
+        with np.errstate(over="ignore"):
+            a = float(np.float32(np.float32(v) + np.float32(eps_b)))
+            d = float(np.float32(np.float32(a) + np.float32(c)))
+        if np.isfinite(d) and d > 0 and rng.random() < 0.7:
+            u = int(np.clip(int(Fraction(a) * (1 << 24) / Fraction(d)) + int(rng.integers(-2, 3)), 0, 2 ** 24 - 1))
         else:
             u = int(rng.integers(0, 2 ** 24))
         want = _exact_decide(u, v, c, eps_b)
@@ -503,6 +523,87 @@ def check_server_fetch_counters(libs: Libs):
     assert np.array_equal(a[0], b[0])
 
 
+# --------------------------------------------------------------------------
+# Exact means (the per-message and per-tensor statistics)
+# --------------------------------------------------------------------------
+def _exact_sum(x) -> Fraction:
+    """The exact sum of fp32 (or fp64) values: each is m 2^e with an integer
+    significand m, so grouping by exponent sums integers only."""
+    x = np.asarray(x, dtype=np.float64)
+    assert np.isfinite(x).all()
+    m, e = np.frexp(x)                       # x = m 2^e, 1/2 <= |m| < 1
+    mi = (m * 2.0 ** 53).astype(np.int64)    # exact: a double has 53 significant bits
+    total = 0
+    for ee in np.unique(e):                  # x = mi 2^(e - 53); units of 2^-1127
+        total += int(mi[e == ee].astype(object).sum()) << int(ee - 53 + 1127)
+    return Fraction(total, 1 << 1127)
+
+
+def _f32_nearest(q: Fraction) -> np.float32:
+    """The fp32 value nearest to the rational q, ties to the even
+    significand: q is compared exactly with a first guess and its two
+    neighbours (the guess, q rounded through fp64, is within one step)."""
+    guess = np.float32(float(q))
+    best = None
+    for x in (np.nextafter(guess, np.float32(-np.inf)), guess,
+              np.nextafter(guess, np.float32(np.inf))):
+        if not np.isfinite(x):
+            continue
+        key = (abs(Fraction(float(x)) - q), int(x.view(np.uint32)) & 1)
+        if best is None or key < best[0]:
+            best = (key, x)
+    return best[1]
+
+
+def _check_exact_means(libs: Libs, mean):
+    """mean(v, real) -> fp32: the exact mean of v rounded once, for more than
+    a million terms and at constructed rounding boundaries."""
+    rng = np.random.default_rng(47)
+    P = 1_000_003
+    v = (10 ** rng.uniform(-3, 3, P)).astype(np.float32)
+    v[rng.random(P) < 0.01] = 0.0
+    want = _f32_nearest(_exact_sum(v) / P)
+    for real in ("f32", "f64"):
+        assert mean(v, real) == want, real
+    # Values on an fp32 rounding boundary: (P - 2) copies of lo, z1 and z2
+    # with an exact sum of P (lo + up) / 2 + delta, up the float after lo.
+    # delta = 0 is a tie (to the even one of lo and up); delta = +-2^-149 puts
+    # the mean just above or below it, by far less than an fp64 sum of a
+    # million terms near 1.5 can resolve.
+    # With P = 2^20 the excess delta / P is a whole number of units of the
+    # exact quotient (no remainder); with P = 3 2^19 it is not.
+    tiny = np.float32(2.0 ** -149)
+    for P in (3 << 19, 1 << 20):
+        for lo in (np.float32(1.5), np.nextafter(np.float32(1.5), np.float32(2))):
+            up = np.nextafter(lo, np.float32(2))
+            gap = P * (Fraction(float(up)) - Fraction(float(lo))) / 2
+            z1 = np.float32(2 * Fraction(float(lo)) + gap)
+            assert Fraction(float(z1)) == 2 * Fraction(float(lo)) + gap
+            even = lo if int(lo.view(np.uint32)) % 2 == 0 else up
+            for delta, expect in ((np.float32(0.0), even), (tiny, up), (-tiny, lo)):
+                v = np.full(P, lo, dtype=np.float32)
+                v[P // 3] = z1
+                v[-1] = delta
+                assert _f32_nearest(_exact_sum(v) / P) == expect
+                for real in ("f32", "f64"):
+                    assert mean(v, real) == expect, (real, P, float(lo), float(delta))
+    P = 3 << 19
+    # In the fp64 build the terms are doubles: a term of 2^-1074 moves the
+    # mean by less than one unit of the exact quotient, so only the remainder
+    # of the division can tell that it is above the tie.
+    lo = np.float32(1.5)
+    up = np.nextafter(lo, np.float32(2))
+    v = np.full(P, float(lo))
+    v[P // 3] = float(np.float32(2 * Fraction(float(lo)) + P * (Fraction(float(up)) - Fraction(float(lo))) / 2))
+    v[-1] = 2.0 ** -1074
+    assert mean(v, "f64") == up
+    # Signs, zeros and subnormals: the exact mean of a mixed vector.
+    v = (rng.standard_normal(4099) * 10.0 ** rng.integers(-45, 3, 4099)).astype(np.float32)
+    for real in ("f32", "f64"):
+        assert mean(v, real) == _f32_nearest(_exact_sum(v) / v.size), real
+        assert mean(np.zeros(5, np.float32), real) == 0.0
+
+
 def check_message_path(libs: Libs):
     """The paper's literal B-FASGD (Sec. 2.3): one Eq. 9 decision per message
     against the mean of v; dropped pushes re-apply the client's cached
@@ -512,9 +613,9 @@ def check_message_path(libs: Libs):
     for real in ("f32", "f64"):
         for P in (1, 7, 1000, 4099):
             v = (10 ** rng.uniform(-2, 3, P)).astype(np.float32)
-            exact = Fraction(math.fsum(v.astype(np.float64))) / P
             got = oracle.mean_v(v, real, lib=libs.lib(real))
-            assert got == float(np.float32(float(exact))), (real, P)
+            assert np.float32(got) == _f32_nearest(_exact_sum(v) / P), (real, P)
+    _check_exact_means(libs, lambda v, real: np.float32(oracle.mean_v(v, real, lib=libs.lib(real))))
     # Message draws are their own domain (not the per-parameter draws).
     seed = 99
     same = sum(oracle.draw_message(seed, 0, 2, n, lib=libs.f32) ==
@@ -713,9 +814,8 @@ def check_tensor_means(libs: Libs):
         got = oracle.tensor_means(v, sizes, real, lib=libs.lib(real))
         off = np.concatenate([[0], np.cumsum(sizes)])
         for t in range(sizes.size):
-            seg = v[off[t]:off[t + 1]].astype(np.float64)
-            exact = Fraction(math.fsum(seg)) / int(sizes[t])
-            assert got[t] == np.float32(float(exact)), (real, t)
+            seg = v[off[t]:off[t + 1]]
+            assert got[t] == _f32_nearest(_exact_sum(seg) / int(sizes[t])), (real, t)
         assert got[0] == v[0]                          # one-element tensor: v itself
         const = np.repeat(np.float32([0.3, 7.0, 1e-3]), [5, 11, 3])
         assert np.array_equal(oracle.tensor_means(const, [5, 11, 3], real, lib=libs.lib(real)),
@@ -723,6 +823,14 @@ def check_tensor_means(libs: Libs):
     # One tensor over everything: the per-message statistic.
     v = (10 ** rng.uniform(-2, 3, 5000)).astype(np.float32)
     assert oracle.tensor_means(v, [5000], lib=libs.f32)[0] == oracle.mean_v(v, lib=libs.f32)
+
+    # The same constructions as the per-message statistic, each as the middle
+    # tensor of three (so the offsets matter too).
+    def middle(v, real):
+        sizes = [3, v.shape[0], 5]
+        w = np.concatenate([np.full(3, 7.0), np.asarray(v, dtype=np.float64), np.full(5, 1e-3)])
+        return oracle.tensor_means(w, sizes, real, lib=libs.lib(real))[1]
+    _check_exact_means(libs, middle)
 
 
 def check_budget_threshold(libs: Libs):

@@ -45,25 +45,39 @@ MUTANTS = {
     "fetch_uses_push_stream": ("return ora_select_stream(P, theta, v, c, eps_b, seed, 1,",
                                "return ora_select_stream(P, theta, v, c, eps_b, seed, 0,"),
     "fetch_apply_wrong_slot": ("theta_client[idx[i]] = val[i];", "theta_client[i] = val[i];"),
-    "mean_v_wrong_divisor": ("return (float)(s / (double)P);", "return (float)(s / (double)(P + 1));"),
-    "mean_v_first_only": ("s += (double)v[p];", "s = (double)v[p];"),
+    "mean_v_wrong_divisor": ("return ora_sum_mean(&s, P);", "return ora_sum_mean(&s, P + 1);"),
+    "mean_v_first_only": ("for (int64_t p = 0; p < P; p++)\n        ora_sum_add(&s, (double)v[p]);",
+                          "for (int64_t p = 0; p < 1; p++)\n        ora_sum_add(&s, (double)v[p]);"),
+    "mean_v_fp64_sequential": ("return ora_sum_mean(&s, P);",
+                               "{ double t = 0; for (int64_t p = 0; p < P; p++) t += (double)v[p];"
+                               " return (float)(t / (double)P); }"),
+    "mean_ties_away": ("if (guard && (sticky || (mant & 1u)))", "if (guard)"),
+    "mean_truncates": ("if (guard && (sticky || (mant & 1u)))\n        mant++;",
+                       "if (guard && (sticky || (mant & 1u)))\n        mant += 0;"),
+    "mean_drops_remainder": ("int sticky = r != 0;", "int sticky = 0;"),
+    "mean_drops_low_bits": ("sticky = (q[bit / 32] >> (bit % 32)) & 1u;", "sticky = 0;"),
+    "mean_ignores_sign": ("ora_acc_add(neg ? s->neg : s->pos, m,", "ora_acc_add(s->pos, m,"),
+    "mean_exponent_off_by_one": ("E == 0 ? 0 : E - 1", "E == 0 ? 0 : E"),
+    "mean_carry_dropped": ("c = (c >> 32) + (uint64_t)w[i + 2] + (hi >> 32);",
+                           "c = (uint64_t)w[i + 2] + (hi >> 32);"),
+    "decide_not_strict": ("< (double)a * 16777216.0", "<= (double)a * 16777216.0"),
+    "decide_product_in_fp32": ("(double)u * (double)d <", "(double)((float)u * d) <"),
+    "decide_threshold_scale": ("(double)a * 16777216.0", "(double)a * 8388608.0"),
+    "tensor_mean_divisor": ("vbar[t] = ora_sum_mean(&s, sizes[t]);",
+                            "vbar[t] = ora_sum_mean(&s, sizes[t] + 1);"),
+    "tensor_mean_no_offset": ("vbar[t] = ora_sum_mean(&s, sizes[t]);\n        off += sizes[t];",
+                              "vbar[t] = ora_sum_mean(&s, sizes[t]);"),
     "message_draw_collides": ("uint32_t ctr[4] = {0xFFFFFFFFu,", "uint32_t ctr[4] = {0u,"),
     "message_draw_ignores_stream": ("{0xFFFFFFFFu, client | (stream << 31),", "{0xFFFFFFFFu, client,"),
     "std_variant_inverts": ("REAL r = ora_sqrt(var + eps);\n        *v = beta", "REAL r = 1 / ora_sqrt(var + eps);\n        *v = beta"),
     "sim_noise_half_range": ("(1.0f / 8388608.0f) - 0.5f", "(1.0f / 16777216.0f) - 0.5f"),
     "sim_grad_sign": ("float d = theta[p] - star[p];\n        g[p]", "float d = star[p] - theta[p];\n        g[p]"),
     "sim_loss_no_half": ("return 0.5 * s;", "return s;"),
-    "decide_not_strict": ("prod == A && err < 0.0f", "prod == A && err <= 0.0f"),
-    "decide_ignores_err": ("if (prod == A && err < 0.0f)\n        return 1;\n", ""),
     "decide_drops_eps": ("float a = v + eps_b;", "float a = v;"),
     "select_val_index": ("val[m] = g[p];", "val[m] = g[m];"),
     "select_idx_off_by_one": ("idx[m] = (int32_t)p;", "idx[m] = (int32_t)(p + 1);"),
     "sparse_val_reversed": ("(REAL)val[i], coef,", "(REAL)val[count - 1 - i], coef,"),
     "sparse_no_order_check": ("if (i > 0 && idx[i] <= idx[i - 1])\n            return -1;\n", ""),
-    "tensor_mean_divisor": ("vbar[t] = (float)(s / (double)sizes[t]);",
-                            "vbar[t] = (float)(s / (double)(sizes[t] + 1));"),
-    "tensor_mean_no_offset": ("vbar[t] = (float)(s / (double)sizes[t]);\n        off += sizes[t];",
-                              "vbar[t] = (float)(s / (double)sizes[t]);"),
     "budget_term_scale": ("int shift = e - 24 + 32;", "int shift = e - 24 + 31;"),
     "budget_ignores_size": ("int64_t prod = size * M;", "int64_t prod = M;"),
     "budget_drops_eps": ("float a = vbar + eps_b;\n    if (!(a > 0.0f)",
