@@ -208,6 +208,10 @@ def gpu_identifier(torch) -> str:
         return str(torch.cuda.current_device())
 
 
+VARIANTS = {"asgd": streams.ASGD, "sasgd": streams.SASGD, "fasgd": streams.FASGD,
+            "fasgd-std": streams.FASGD_STD}
+
+
 def algorithmic_bytes_dense(P: int, K: int, fasgd_rule: bool) -> int:
     """theta (+ n, b, v) read and written once, K gradient slices read once."""
     state = 4 if fasgd_rule else 1
@@ -253,6 +257,23 @@ def oracle_rate(w: streams.Workload, P_sample: int, batches: int | None, seconds
 # ---------------------------------------------------------------------------
 # GPU arm
 # ---------------------------------------------------------------------------
+SMALL_P = 1 << 21   # dense workloads at or below this size also run the C driver
+
+
+def run_abi_latency(P: int, K: int, variant: int, steps: int) -> dict | None:
+    """The C timing driver of the ABI (abi_latency.c) on the same shape."""
+    from paper_1601_04033_gb300 import build
+    try:
+        exe = build.build_latency_driver()
+        out = subprocess.run([exe, str(P), str(K), str(steps), str(variant)], capture_output=True,
+                             text=True, timeout=300)
+    except Exception as e:      # reported, not fatal: the Python numbers stand alone
+        return {"error": str(e)[:200]}
+    if out.returncode != 0:
+        return {"error": out.stderr.strip()[-200:]}
+    return json.loads(out.stdout.strip().splitlines()[-1])
+
+
 def run_dense(args, w, world, rank, local):
     import torch
     from paper_1601_04033_gb300 import fasgd
@@ -260,7 +281,8 @@ def run_dense(args, w, world, rank, local):
     device = torch.device("cuda", local)
     torch.cuda.set_device(device)
     K, P = w.K, (args.P or w.P)
-    variant = streams.FASGD
+    variant = VARIANTS[args.variant]
+    fasgd_rule = variant in (streams.FASGD, streams.FASGD_STD)
     wr = shard_workload(w, rank)
     pool = streams.gradient_pool(wr, P, w.R)
     th0 = streams.theta0(wr, P)
@@ -294,6 +316,7 @@ def run_dense(args, w, world, rank, local):
     clocks.start()
     time.sleep(0.3)   # let the sampler take its first reading
     start.record(stream)
+    h0 = time.perf_counter()
     for i in range(args.steps):
         b = args.warmup + i
         cl, js, sl = batches[b]
@@ -302,6 +325,7 @@ def run_dense(args, w, world, rank, local):
         ev_a[i].record(stream)
         srv.apply_pending(K)
         ev_b[i].record(stream)
+    host_us = (time.perf_counter() - h0) * 1e6 / args.steps
     end.record(stream)
     torch.cuda.synchronize()
     clock_info = clocks.stop()
@@ -349,25 +373,36 @@ def run_dense(args, w, world, rank, local):
                "steps": args.e2e_steps, "ms_per_step": e_ms / args.e2e_steps}
     srv.sync()
     srv.close()
+    # Small passes are bound by call latency: time the same steps from C
+    # through the ABI (host cost of the calls, GPU time of an eager loop and
+    # of a graph replay of the same launches) to split it from the binding's.
+    abi_latency = None
+    if P <= SMALL_P and world == 1 and not args.no_abi_latency:
+        abi_latency = run_abi_latency(P, K, variant, max(args.steps, 1000))
 
     step_s = total_ms / 1e3 / args.steps
     value = P * world * K / step_s
-    alg = algorithmic_bytes_dense(P, K, True)
+    alg = algorithmic_bytes_dense(P, K, fasgd_rule)
     peak, peak_kind = peaks()
     achieved = alg / (kern_avg_ms / 1e3) / 1e9
+    tkey = w.name if not args.P else f"{w.name}-P{P}"
+    if args.variant != "fasgd":
+        tkey += "-" + ("sgd" if not fasgd_rule else args.variant)
     roofline = {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
                 "frac": round(achieved / peak, 4), "peak_source": peak_kind, **nominal(achieved),
-                "kernel": "fasgd_dense_kernel<FASGD> (bulk-copy ring)",
+                "kernel": "fasgd_dense_kernel<%s> (bulk-copy ring)"
+                          % ("FASGD" if variant == streams.FASGD else
+                             "FASGD_STD" if variant == streams.FASGD_STD else "SGD"),
                 "bytes_per_launch": alg, "launch_ms": round(kern_avg_ms, 5),
-                "traffic": profiled_traffic(w.name if not args.P else f"{w.name}-P{P}",
-                                            DENSE_KERNEL_SOURCES)}
+                "traffic": profiled_traffic(tkey, DENSE_KERNEL_SOURCES)}
     return {
         "value": value, "ms_per_step": total_ms / args.steps, "roofline": roofline,
         "clocks": clock_info, "e2e": e2e, "gpu_launches": launches,
         "pushes_per_s": world * K / step_s,
         "hbm_gbs_step": alg * world / step_s / 1e9,
+        "host_us_per_step": round(host_us, 3), "abi_latency": abi_latency,
         "config": {"workload": w.name, "P_per_gpu": P, "P_total": P * world, "lambda": w.lam,
-                   "K": K, "variant": "fasgd", "alpha": w.alpha, "staleness": w.delay,
+                   "K": K, "variant": args.variant, "alpha": w.alpha, "staleness": w.delay,
                    "gradient_pool_slots": w.R, "pushes_timed": K * args.steps,
                    "parallelism": f"param-shard{world}",
                    "arithmetic": "exact (IEEE sqrt/div, unfused)" if args.exact else
@@ -762,6 +797,11 @@ def main():
     ap.add_argument("--e2e-steps", type=int, default=40)
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-abi-latency", action="store_true",
+                    help="small dense workloads: skip the C driver timing")
+    ap.add_argument("--variant", choices=sorted(VARIANTS), default="fasgd",
+                    help="dense workloads: update rule (ASGD and SASGD move 8 + 4K bytes per "
+                         "parameter, the FASGD rules 32 + 4K)")
     ap.add_argument("--exact", action="store_true",
                     help="dense workloads: time the exact-arithmetic FASGD update")
     args = ap.parse_args()
@@ -782,14 +822,16 @@ def main():
         if rank != 0:
             return
         P_s = min(args.P or w.P, 1 << 20)
-        rate, done, el = oracle_rate(w, P_s, args.steps, None, warmup=args.warmup)
+        var = VARIANTS[args.variant] if mode == "dense" else streams.FASGD
+        rate, done, el = oracle_rate(w, P_s, args.steps, None, variant=var, warmup=args.warmup)
         line = {"impl": "reference", "metric": METRIC, "value": rate, "unit": UNIT,
                 "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
                 "ms_per_step": el * 1e3 / done, "higher_is_better": True, "scaling": "weak",
                 "vs_baseline": None, "dtype": "f32", "data": "synthetic",
                 "config": {"workload": w.name, "P_per_gpu": args.P or w.P,
                            "P_total": (args.P or w.P) * args.gpus, "lambda": w.lam, "K": w.K,
-                           "variant": "fasgd", "alpha": w.alpha, "staleness": w.delay,
+                           "variant": args.variant if mode == "dense" else "fasgd",
+                           "alpha": w.alpha, "staleness": w.delay,
                            "parallelism": f"param-shard{args.gpus}",
                            "sample": f"first {P_s} parameters, K={w.K} pushes per step",
                            "oracle": "single-threaded C, fp32"},
@@ -817,9 +859,11 @@ def main():
         if world == 1 and not args.no_cpu_baseline:
             P_s = min(res["config"]["P_per_gpu"], 1 << 22)
             wc = w if mode == "dense" else w.replace(K=1)
-            rate, done, el = oracle_rate(wc, P_s, None, args.cpu_seconds)
+            var = VARIANTS[args.variant] if mode == "dense" else streams.FASGD
+            rate, done, el = oracle_rate(wc, P_s, None, args.cpu_seconds, variant=var)
             cpu = {"value": rate, "unit": UNIT, "cores": 1, "kind": "oracle",
-                   "sample": f"{done} passes of K={wc.K} dense FASGD pushes over the first "
+                   "sample": f"{done} passes of K={wc.K} dense "
+                             f"{streams.VARIANT_NAMES[var].upper()} pushes over the first "
                              f"{P_s} parameters ({el:.1f} s)"}
         line = {"metric": METRIC, "value": res["value"], "unit": UNIT, "n_gpus": world,
                 "steps": args.steps, "warmup": args.warmup, "ms_per_step": res["ms_per_step"],
@@ -828,7 +872,8 @@ def main():
                 "roofline": physical(res["roofline"]), "cpu_baseline": cpu, "e2e": res["e2e"],
                 "clocks": res["clocks"], "gpu_launches": res["gpu_launches"],
                 "pushes_per_s": res["pushes_per_s"]}
-        for k in ("hbm_gbs_step", "sent_fraction", "fetched_fraction", "sent_updates_per_s"):
+        for k in ("hbm_gbs_step", "sent_fraction", "fetched_fraction", "sent_updates_per_s",
+                  "host_us_per_step", "abi_latency"):
             if k in res:
                 line[k] = res[k]
         print(json.dumps(line))

@@ -84,6 +84,32 @@ def build(force: bool = False, verbose: bool = False, extra_flags: list | None =
     return LIB
 
 
+DRIVER_SRC = os.path.join(PKG, "abi_latency.c")
+DRIVER = os.path.join(BUILD, "abi_latency")
+
+
+def build_latency_driver(force: bool = False) -> str:
+    """Build the C timing driver of the ABI (abi_latency.c) against
+    libfasgd.so and the CUDA runtime; returns the executable's path."""
+    lib = build()
+    if (not force and os.path.exists(DRIVER)
+            and os.path.getmtime(DRIVER) >= max(os.path.getmtime(DRIVER_SRC),
+                                                os.path.getmtime(lib))):
+        return DRIVER
+    os.makedirs(BUILD, exist_ok=True)
+    cuda = os.path.dirname(os.path.dirname(nvcc()))
+    tmp = DRIVER + f".tmp{os.getpid()}"
+    cmd = ["gcc", "-O2", "-std=c11", "-Wall", "-Wextra", DRIVER_SRC, f"-I{INCLUDE}",
+           f"-I{os.path.join(cuda, 'include')}", f"-L{PKG}", "-lfasgd",
+           f"-L{os.path.join(cuda, 'lib64')}", "-lcudart", f"-Wl,-rpath,{PKG}",
+           f"-Wl,-rpath,{os.path.join(cuda, 'lib64')}", "-o", tmp]
+    r = subprocess.run(cmd, capture_output=True, text=True)
+    if r.returncode != 0:
+        raise RuntimeError(f"abi_latency build failed:\n{r.stdout}\n{r.stderr}")
+    os.replace(tmp, DRIVER)
+    return DRIVER
+
+
 if __name__ == "__main__":
     import sys
     print(build(force="--force" in sys.argv, verbose=True,
