@@ -98,9 +98,11 @@ FASGD_API void fasgd_destroy(fasgd_t* h);
  * eps (Eq. 6 stabiliser), c_push and eps_b (Eq. 9 threshold and its
  * stabiliser) and the 64-bit seed of the B-FASGD draws.
  * Domain: 0 <= gamma <= 1, 0 <= beta < 1, eps and eps_b finite and >= 0,
- * c_push >= 0 (+inf allowed: nothing is sent).  The send decision needs
- * v_p + eps_b > 0 (eps_b > 0 guarantees it) and below 2^103 (so that
- * (v_p + eps_b) * 2^24 stays finite in fp32).
+ * c_push >= 0 (+inf allowed: nothing is sent).  The send decision is exact
+ * for every v_p >= 0 of any finite magnitude (subnormal to FLT_MAX) and
+ * every c_push >= 0; a parameter with v_p + eps_b = 0 is never sent, and
+ * (v_p + eps_b) + c_push must stay below 2^128 unless c_push = +inf (a
+ * finite sum that rounds to +inf in fp32 would read as "never sent").
  * Errors: EINVAL (outside the domain), EAGAIN (pushes pending).
  */
 FASGD_API int fasgd_set_hparams(fasgd_t* h, float gamma, float beta, float eps, float c_push,
@@ -179,6 +181,11 @@ FASGD_API int fasgd_push_sparse(fasgd_t* h, int32_t client, int64_t timestamp, c
  * keeps each element's theta, n, b, v in registers across them; each sparse
  * push is its own pass.  T increases by K.
  * Errors: EINVAL (K < 1 or K > FASGD_KMAX), EAGAIN (fewer than K pending), ECUDA.
+ * If a launch fails partway through the batch (ECUDA or ENOMEM), the pushes
+ * whose passes were already enqueued count as applied: they have left the
+ * queue and T has advanced by their number (the message says how many);
+ * the push that failed and the rest of the batch are still queued, with
+ * their draw counters unchanged, so retrying applies each push once.
  */
 FASGD_API int fasgd_apply_pending(fasgd_t* h, int32_t K);
 
@@ -412,10 +419,13 @@ FASGD_API int64_t fasgd_kernel_launches(const fasgd_t* h);
  * that every GPU which loads the library holds until the process exits.
  * The first call on a device looks up that array's device address (once per
  * device, with that device current); make that first call before any
- * stream capture.  All calls share the one array and the kernels rewrite
- * every scratch word before reading it, so nothing carries over between
- * calls -- but calls that overlap on the GPU (other streams, other host
- * threads) race on it and must be serialised by the caller.
+ * stream capture (a first call made while `stream` is capturing returns
+ * FASGD_EINVAL and does nothing).  The address is kept for the life of the
+ * process: after cudaDeviceReset on a device, do not call this entry point
+ * on that device again.  All calls share the one array and the kernels
+ * rewrite every scratch word before reading it, so nothing carries over
+ * between calls -- but calls that overlap on the GPU (other streams, other
+ * host threads) race on it and must be serialised by the caller.
  *
  * Arguments: P parameters, 1 <= P <= BFASGD_NOALLOC_PMAX (larger P is
  * rejected with FASGD_EINVAL and a message); grad and v: device fp32[P],

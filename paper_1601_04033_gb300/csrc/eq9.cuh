@@ -48,20 +48,39 @@ __device__ __forceinline__ Philox4 philox4x32_10(uint32_t c0, uint32_t c1, uint3
 }
 
 // Eq. 9 for one parameter: send iff u / 2^24 < 1 / (1 + c / a), a = fl(v + eps_b),
-// i.e. iff u * d < A with d = fl(a + c) and A = a * 2^24, decided exactly:
-// u * d = prod + err exactly (prod = fl(u * d), err = fma(u, d, -prod)), and
-// u * d < A  <=>  err < A - prod  <=>  err < fl(A - prod).  The last step is
-// exact: when A and prod are within a factor of two, A - prod is exact
-// (Sterbenz); otherwise |A - prod| > 2^-24 prod >= |err|, and rounding
-// A - prod keeps it on the same side of err.
-__device__ __forceinline__ uint32_t send_bit(uint32_t u, float v, float c, float eps_b) {
+// i.e. iff u * d < a * 2^24 with d = fl(a + c), decided exactly.
+//
+// The sign of u * d - a * 2^24 is the sign of one fused multiply-add: it
+// rounds the exact value once, rounding keeps the sign, and a nonzero
+// difference of these operands (all multiples of 2^-149) is never rounded to
+// zero.  So the test is fma(u, d, -A) < 0 with A = a * 2^24, once A is exact.
+// Two scalings cover every a >= 0 and c >= 0 (+inf included):
+//   SCALE_D = false, for c < kSendScaleC = 2^79:  fma(u, d, -(a * 2^24)).
+//     A is exact below a = 2^104; from there on d = a (c is below half an
+//     ulp of a), where u < 2^24 always holds, and the overflowed A = +inf
+//     still gives fma = -inf < 0.
+//   SCALE_D = true, for c >= 2^79:  fma(u, d * 2^-24, -a).  d >= c >= 2^79,
+//     so d * 2^-24 is exact; d = +inf gives +inf (u > 0) or NaN (u = 0),
+//     neither below 0: nothing is sent, as Eq. 9 says for c = +inf.
+// The host picks the form once per call from c (send_form).
+constexpr float kSendScaleC = 604462909807314587353088.0f;  // 2^79
+
+inline bool send_form(float c) { return c >= kSendScaleC; }
+
+template <bool SCALE_D>
+__device__ __forceinline__ bool send_test(uint32_t u, float v, float c, float eps_b) {
     const float a = __fadd_rn(v, eps_b);
     const float d = __fadd_rn(a, c);
     const float uf = (float)u;  // exact: u < 2^24
-    const float prod = __fmul_rn(uf, d);
-    const float err = __fmaf_rn(uf, d, -prod);
-    const float A = __fmul_rn(a, 16777216.0f);
-    return err < __fsub_rn(A, prod) ? 1u : 0u;
+    const float s = SCALE_D ? __fmaf_rn(uf, __fmul_rn(d, 5.9604644775390625e-8f), -a)
+                            : __fmaf_rn(uf, d, -__fmul_rn(a, 16777216.0f));
+    return s < 0.0f;
+}
+
+// The same test with the form chosen per call (single decisions).
+__device__ __forceinline__ uint32_t send_bit(uint32_t u, float v, float c, float eps_b) {
+    return (c >= kSendScaleC ? send_test<true>(u, v, c, eps_b) : send_test<false>(u, v, c, eps_b))
+               ? 1u : 0u;
 }
 
 }  // namespace fasgd

@@ -737,6 +737,24 @@ int fasgd_apply_pending(fasgd_t* h, int32_t K) {
                      : h->variant == FASGD_FASGD_STD ? fasgd::kRuleFasgdStd
                                                      : fasgd::kRuleSgd;
     const fasgd::StatParams sp = h->stat_params();
+    // Takes the first `done` pushes out of the queue (their passes are
+    // enqueued) and advances T past them.  A launch that fails partway keeps
+    // the batch's earlier pushes applied: they leave the queue, the failed
+    // push and the rest stay, so a retry applies each push exactly once.
+    auto retire = [h](int done) {
+        for (int i = 0; i < done; ++i) {
+            const int slot = h->fifo.front().stage;
+            if (slot >= 0) h->stage_busy[(size_t)slot] = 0;
+            h->fifo.pop_front();
+        }
+        h->T += done;
+    };
+    auto partial_fail = [h, K, &retire](cudaError_t st, const char* what, int done) {
+        retire(done);
+        return h->fail(st == cudaErrorMemoryAllocation ? FASGD_ENOMEM : FASGD_ECUDA,
+                       "fasgd_apply_pending: %s: %s (%d of %d pushes were applied and left the "
+                       "queue; T advanced by %d)", what, cudaGetErrorString(st), done, K, done);
+    };
     int k = 0;
     while (k < K) {
         const Push& first = h->fifo[(size_t)k];
@@ -776,12 +794,13 @@ int fasgd_apply_pending(fasgd_t* h, int32_t K) {
                     h->stage_seq[(size_t)slot] = h->pass_seq;
                 }
             }
-            if (st != cudaSuccess) return h->cuda_fail(st, "fasgd_apply_pending: dense pass");
+            if (st != cudaSuccess) return partial_fail(st, "dense pass", k);
             k += r;
         } else if (first.kind == kMessage) {
             // Decide against the mean of v now, refresh the client's cache
             // slot if the push is transmitted, then apply the slot.
             float* slot = h->grad_cache + (size_t)first.client * (size_t)h->cache_stride;
+            const uint64_t count0 = h->push_count[(size_t)first.client];
             cudaError_t st = h->launch_message(0, first.client, first.grad, slot, first.flag,
                                                h->c_push, &h->push_count);
             if (st == cudaSuccess) {
@@ -801,11 +820,17 @@ int fasgd_apply_pending(fasgd_t* h, int32_t K) {
                 st = fasgd::launch_dense(a, rule, h->exact, h->num_sms, h->stream, &h->launches);
                 h->msg_sums_valid = st == cudaSuccess;
             }
-            if (st != cudaSuccess) return h->cuda_fail(st, "fasgd_apply_pending: message push");
+            if (st != cudaSuccess) {
+                // A retry redraws the same decision against the same v (the
+                // pass did not run), so it refreshes the cache slot alike.
+                h->push_count[(size_t)first.client] = count0;
+                return partial_fail(st, "message push", k);
+            }
             k += 1;
         } else if (first.kind == kBudget) {
             // Decide every tensor against the statistics now, then update the
             // transmitted ones.
+            const uint64_t count0 = h->push_count[(size_t)first.client];
             cudaError_t st = h->launch_budget(0, first.client, first.budget, first.sent_out,
                                               first.c_out, first.count_out, h->push_count);
             if (st == cudaSuccess) {
@@ -814,7 +839,10 @@ int fasgd_apply_pending(fasgd_t* h, int32_t K) {
                 r.coef = h->coef(h->T + k - first.j);
                 st = fasgd::launch_tensor_apply(r, rule, h->exact, h->stream, &h->launches);
             }
-            if (st != cudaSuccess) return h->cuda_fail(st, "fasgd_apply_pending: budget push");
+            if (st != cudaSuccess) {
+                h->push_count[(size_t)first.client] = count0;   // a retry redraws the same decision
+                return partial_fail(st, "budget push", k);
+            }
             k += 1;
         } else {
             fasgd::SparseArgs a;
@@ -833,17 +861,12 @@ int fasgd_apply_pending(fasgd_t* h, int32_t K) {
             a.err = h->dev_err;
             if (first.n_max > 0 || first.n_dev != nullptr) {
                 cudaError_t st = fasgd::launch_sparse(a, rule, h->exact, h->num_sms, h->stream, &h->launches);
-                if (st != cudaSuccess) return h->cuda_fail(st, "fasgd_apply_pending: sparse pass");
+                if (st != cudaSuccess) return partial_fail(st, "sparse pass", k);
             }
             k += 1;
         }
     }
-    for (int i = 0; i < K; ++i) {
-        const int slot = h->fifo.front().stage;
-        if (slot >= 0) h->stage_busy[(size_t)slot] = 0;
-        h->fifo.pop_front();
-    }
-    h->T += K;
+    retire(K);
     return FASGD_OK;
 }
 

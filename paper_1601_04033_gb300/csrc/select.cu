@@ -41,7 +41,7 @@ __device__ __forceinline__ float4 load_quad(const float* x, int64_t e, int64_t P
     return make_float4(t[0], t[1], t[2], t[3]);
 }
 
-template <bool FULL>
+template <bool FULL, bool SCALE_D>
 __device__ __forceinline__ void mask_tile(const SelectArgs& a) {
     __shared__ int32_t warp_cnt[kWarps];
     const int lane = threadIdx.x & 31;
@@ -60,10 +60,10 @@ __device__ __forceinline__ void mask_tile(const SelectArgs& a) {
         uint32_t nib = 0;
         if (FULL || e < a.P) {
             const Philox4 r = philox4x32_10(e >> 2, a.client_word, a.push_lo, a.push_hi, a.round_key0, a.round_key1);
-            nib = send_bit(r.x[0] >> 8, v4[it].x, a.c, a.eps_b) |
-                  (send_bit(r.x[1] >> 8, v4[it].y, a.c, a.eps_b) << 1) |
-                  (send_bit(r.x[2] >> 8, v4[it].z, a.c, a.eps_b) << 2) |
-                  (send_bit(r.x[3] >> 8, v4[it].w, a.c, a.eps_b) << 3);
+            nib = (send_test<SCALE_D>(r.x[0] >> 8, v4[it].x, a.c, a.eps_b) ? 1u : 0u) |
+                  (send_test<SCALE_D>(r.x[1] >> 8, v4[it].y, a.c, a.eps_b) ? 2u : 0u) |
+                  (send_test<SCALE_D>(r.x[2] >> 8, v4[it].z, a.c, a.eps_b) ? 4u : 0u) |
+                  (send_test<SCALE_D>(r.x[3] >> 8, v4[it].w, a.c, a.eps_b) ? 8u : 0u);
             if (!FULL) {
                 const int64_t valid = a.P - e;  // parameters past P are never sent
                 if (valid < 4) nib &= (1u << valid) - 1u;
@@ -91,13 +91,15 @@ __device__ __forceinline__ void mask_tile(const SelectArgs& a) {
 }
 
 // Full tiles (all but perhaps the last) skip the per-quad bounds checks.
+// SCALE_D: the form of the Eq. 9 test for this call's c (send_form).
+template <bool SCALE_D>
 __global__ void __launch_bounds__(kSelectThreads) bfasgd_mask_kernel(const __grid_constant__ SelectArgs a) {
     pdl_wait();
     pdl_trigger();
     if ((int64_t)(blockIdx.x + 1) * kSelectTile <= a.P)
-        mask_tile<true>(a);
+        mask_tile<true, SCALE_D>(a);
     else
-        mask_tile<false>(a);
+        mask_tile<false, SCALE_D>(a);
 }
 
 constexpr int kScanThreads = 1024;
@@ -238,7 +240,9 @@ void select_key_schedule(SelectArgs& a, uint64_t seed) {
 }
 
 cudaError_t launch_select(const SelectArgs& a, cudaStream_t stream, int64_t* launches) {
-    cudaError_t st = launch_pdl(bfasgd_mask_kernel, a.ntiles, kSelectThreads, 0, stream, a);
+    cudaError_t st = send_form(a.c)
+                         ? launch_pdl(bfasgd_mask_kernel<true>, a.ntiles, kSelectThreads, 0, stream, a)
+                         : launch_pdl(bfasgd_mask_kernel<false>, a.ntiles, kSelectThreads, 0, stream, a);
     if (st != cudaSuccess) return st;
     ++*launches;
     st = launch_pdl(bfasgd_scan_kernel, 1, kScanThreads, 0, stream, a);
@@ -286,13 +290,24 @@ void* g_noalloc_addr[kMaxDevices] = {};
 
 // Device address of the static scratch on the current device, looked up once
 // per device.  Host code cannot use the symbol itself as a device pointer.
-cudaError_t noalloc_scratch(unsigned char** out) {
+// The look-up is a runtime call that does not belong in a stream capture:
+// if it is still to be made while `stream` is capturing, *capturing is set
+// and nothing is done.
+cudaError_t noalloc_scratch(cudaStream_t stream, unsigned char** out, bool* capturing) {
+    *capturing = false;
     int dev = 0;
     cudaError_t st = cudaGetDevice(&dev);
     if (st != cudaSuccess) return st;
     if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
     std::lock_guard<std::mutex> lock(g_noalloc_mutex);
     if (g_noalloc_addr[dev] == nullptr) {
+        cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+        st = cudaStreamIsCapturing(stream, &cs);
+        if (st != cudaSuccess) return st;
+        if (cs != cudaStreamCaptureStatusNone) {
+            *capturing = true;
+            return cudaSuccess;
+        }
         void* p = nullptr;
         st = cudaGetSymbolAddress(&p, g_noalloc_scratch);
         if (st != cudaSuccess) return st;
@@ -338,10 +353,15 @@ extern "C" int bfasgd_select_compact_noalloc(int64_t P, const float* grad, const
         return noalloc_fail(FASGD_EINVAL,
                             "bfasgd_select_compact_noalloc: need c >= 0 and finite eps_b >= 0");
     unsigned char* scratch = nullptr;
-    cudaError_t st = noalloc_scratch(&scratch);
+    bool capturing = false;
+    cudaError_t st = noalloc_scratch(static_cast<cudaStream_t>(stream), &scratch, &capturing);
     if (st != cudaSuccess)
         return noalloc_fail(FASGD_ECUDA, "bfasgd_select_compact_noalloc: cannot address the "
                                          "static scratch on this device");
+    if (capturing)
+        return noalloc_fail(FASGD_EINVAL,
+                            "bfasgd_select_compact_noalloc: the first call on a device looks up "
+                            "its static scratch and must come before any stream capture");
     fasgd::SelectArgs a;
     a.values = grad;
     a.v = v;

@@ -333,6 +333,47 @@ def test_select_at_the_threshold_bit_exact():
     assert_bitwise(gv, ov, "val at threshold")
 
 
+def test_select_threshold_over_the_whole_fp32_range():
+    """The exact Eq. 9 test away from ordinary magnitudes: thresholds placed at
+    each parameter's own draw (within an ulp) for c from subnormal to 2^110,
+    on both sides of the c = 2^79 switch between the kernel's two scalings,
+    and a above 2^104 (where a * 2^24 leaves the fp32 range) with small c,
+    where every parameter is sent.  Bit-exact against the oracle."""
+    import torch
+    P = 40_000
+    eps_b = 0.0
+    seed, client = 0xABCDEF, 3
+    u = np.array([oracle.draw(seed, client, 0, p) for p in range(P)], dtype=np.float64)
+    u = np.clip(u, 1, 2 ** 24 - 2)
+    nudge = np.random.default_rng(17).integers(-1, 2, P)
+    g = np.random.default_rng(18).standard_normal(P).astype(np.float32)
+    g_t = torch.from_numpy(g).cuda()
+    cases = []
+    for c in (2.0 ** -140, 2.0 ** -100, 3.0, 2.0 ** 78, 2.0 ** 79, 2.0 ** 80, 2.0 ** 110):
+        with np.errstate(over="ignore", under="ignore"):
+            a = np.minimum(c * u / (2.0 ** 24 - u), 3.0e38).astype(np.float32)
+        up = np.nextafter(a, np.float32(np.inf))
+        down = np.nextafter(a, np.float32(0))
+        v = np.where(nudge > 0, up, np.where(nudge < 0, down, a)).astype(np.float32)
+        cases.append((c, v, True))
+    big = (2.0 ** np.random.default_rng(19).uniform(104, 127.9, P)).astype(np.float32)
+    for c in (0.0, 1.0, 2.0 ** 78):
+        cases.append((c, big, False))
+    for k, (c, v, split) in enumerate(cases):
+        c32 = float(np.float32(c))
+        srv = _server(P, c=c32, seed=seed)
+        srv.set_hparams(0.95, 0.95, 1e-4, c32, eps_b, seed)
+        gi, gv, m, _ = _select_gpu(srv, client, g_t, torch.from_numpy(v).cuda())
+        oi, ov = oracle.select(g, v, c32, eps_b, seed, client, 0)
+        if split:
+            assert 0.1 * P < m < 0.9 * P, (c, m)
+        else:
+            assert m == P, (c, m)
+        assert_bitwise(gi, oi, f"idx c={c}")
+        assert_bitwise(gv, ov, f"val c={c}")
+        srv.close()
+
+
 def test_sparse_apply_divide_by_std_matches_dense_at_c0():
     import torch
     w = W["bfasgd-25m"]

@@ -102,41 +102,3 @@ def test_noalloc_sizes_in_turn_match_oracle():
         assert m == oi.size, (P, m, oi.size)
         assert np.array_equal(idx[:m].cpu().numpy(), oi)
         assert np.array_equal(val[:m].cpu().numpy().view(np.int32), ov.view(np.int32))
-
-
-def test_noalloc_graph_replays_match_eager():
-    """A captured call replayed on new inputs gives what an eager call with the
-    same counter gives: nothing a call depends on is left behind in the
-    scratch array or fixed in the captured launches beyond their arguments."""
-    import torch
-    f = _f()
-    P = 200_003
-    g = torch.zeros(P, device="cuda")
-    v = torch.ones(P, device="cuda")
-    gi, gv, gn = _outputs(P, "cuda")
-    ei, ev, en = _outputs(P, "cuda")
-    c, client, push_no = 12.0, 4, 9
-
-    def call(i, vv, nn, stream):
-        return f.bfasgd_select_compact_noalloc(P, g.data_ptr(), v.data_ptr(), c, EPS_B, SEED,
-                                               client, push_no, i.data_ptr(), vv.data_ptr(),
-                                               nn.data_ptr(), stream)
-
-    assert call(ei, ev, en, torch.cuda.current_stream().cuda_stream) == f.OK  # address look-up
-    torch.cuda.synchronize()
-    graph = torch.cuda.CUDAGraph()
-    with torch.cuda.graph(graph):
-        assert call(gi, gv, gn, torch.cuda.current_stream().cuda_stream) == f.OK
-    torch.cuda.synchronize()
-    for r in range(4):
-        gen = torch.Generator(device="cuda").manual_seed(r)
-        g.copy_(torch.randn(P, device="cuda", generator=gen) * 0.1)
-        v.copy_(torch.rand(P, device="cuda", generator=gen) * 100 + 0.1)
-        graph.replay()
-        torch.cuda.synchronize()
-        assert call(ei, ev, en, torch.cuda.current_stream().cuda_stream) == f.OK
-        torch.cuda.synchronize()
-        m = int(en.item())
-        assert int(gn.item()) == m and 0 < m < P, (r, int(gn.item()), m)
-        assert torch.equal(gi[:m], ei[:m])
-        assert torch.equal(gv[:m].view(torch.int32), ev[:m].view(torch.int32))
