@@ -18,6 +18,8 @@
 // global stores.  A stage holds up to 8 gradient slices; larger K runs as
 // several stages per tile (the state travels with the first one only).  The
 // last P mod 2048 parameters are handled by plain loads in the last block.
+// Passes with fewer tiles than SMs use a plain grid instead (one quad of
+// parameters per thread, fasgd_direct_kernel).
 //
 // With SUMS (one push, a.vsum set) the pass also leaves the float-float sum
 // of the new v over every 128-parameter chunk (one warp's share of a tile)
@@ -334,6 +336,81 @@ cudaError_t launch_ch(const DenseArgs& a, int num_sms, cudaStream_t stream) {
     return cudaGetLastError();
 }
 
+// ---- small passes ------------------------------------------------------------
+// With fewer tiles than SMs the ring cannot give every SM a tile: its few
+// blocks stage, compute and store one tile each, and the last then runs the
+// tail.  A plain grid with one quad of parameters per thread and all of a
+// thread's loads issued before its arithmetic makes one round trip to memory
+// instead.  Small working sets stay in L2 between passes, so the gradient
+// loads keep the default cache policy here.
+constexpr int kDirectThreads = 128;
+
+template <int RULE, int ARITH>
+__global__ void __launch_bounds__(kDirectThreads)
+fasgd_direct_kernel(const __grid_constant__ DenseArgs a) {
+    constexpr bool FAS = RULE != kRuleSgd;
+    constexpr bool STD = RULE == kRuleFasgdStd;
+    const int64_t nq = (a.P + 3) / 4;  // quads; the last may be partial
+    for (int64_t q = (int64_t)blockIdx.x * kDirectThreads + threadIdx.x; q < nq;
+         q += (int64_t)gridDim.x * kDirectThreads) {
+        const int64_t e = 4 * q;
+        if (e + 4 <= a.P) {
+            float4 th = *reinterpret_cast<const float4*>(a.theta + e);
+            float4 n = make_float4(0.f, 0.f, 0.f, 0.f), b = n, v = n;
+            if (FAS) {
+                n = *reinterpret_cast<const float4*>(a.n + e);
+                b = *reinterpret_cast<const float4*>(a.b + e);
+                v = *reinterpret_cast<const float4*>(a.v + e);
+            }
+            for (int k0 = 0; k0 < a.K; k0 += 8) {
+                float4 g[8];
+#pragma unroll
+                for (int j = 0; j < 8; ++j)
+                    if (k0 + j < a.K) g[j] = *reinterpret_cast<const float4*>(a.grad[k0 + j] + e);
+#pragma unroll
+                for (int j = 0; j < 8; ++j)
+                    if (k0 + j < a.K) update4<RULE, ARITH>(th, n, b, v, g[j], a.coef[k0 + j], a.sp);
+            }
+            *reinterpret_cast<float4*>(a.theta + e) = th;
+            if (FAS) {
+                *reinterpret_cast<float4*>(a.n + e) = n;
+                *reinterpret_cast<float4*>(a.b + e) = b;
+                *reinterpret_cast<float4*>(a.v + e) = v;
+            }
+        } else {
+            for (int64_t p = e; p < a.P; ++p) {
+                float th = a.theta[p], n = 0.f, b = 0.f, v = 0.f;
+                if (FAS) {
+                    n = a.n[p];
+                    b = a.b[p];
+                    v = a.v[p];
+                }
+                for (int k = 0; k < a.K; ++k) {
+                    if (FAS)
+                        rule_update<ARITH, STD>(th, n, b, v, a.grad[k][p], a.coef[k], a.sp);
+                    else
+                        sgd_update(th, a.grad[k][p], a.coef[k]);
+                }
+                a.theta[p] = th;
+                if (FAS) {
+                    a.n[p] = n;
+                    a.b[p] = b;
+                    a.v[p] = v;
+                }
+            }
+        }
+    }
+}
+
+template <int RULE, int ARITH>
+cudaError_t launch_direct(const DenseArgs& a, int num_sms, cudaStream_t stream) {
+    const int64_t nq = (a.P + 3) / 4;
+    int64_t grid = (nq + kDirectThreads - 1) / kDirectThreads;
+    if (grid > 8 * (int64_t)num_sms) grid = 8 * (int64_t)num_sms;
+    fasgd_direct_kernel<RULE, ARITH><<<(unsigned)grid, kDirectThreads, 0, stream>>>(a);
+    return cudaGetLastError();
+}
+
 template <int RULE, int ARITH>
 cudaError_t launch_rule(const DenseArgs& a, int num_sms, cudaStream_t stream) {
     if constexpr (RULE != kRuleSgd) {
@@ -342,6 +419,7 @@ cudaError_t launch_rule(const DenseArgs& a, int num_sms, cudaStream_t stream) {
             return launch_ch<RULE, ARITH, 1, true>(a, num_sms, stream);
         }
     }
+    if (a.P / kTile < num_sms) return launch_direct<RULE, ARITH>(a, num_sms, stream);
     // Gradient slices per stage: K rounded up to a power of two, at most 8.
     if (a.K > 4) return launch_ch<RULE, ARITH, 8>(a, num_sms, stream);
     if (a.K > 2) return launch_ch<RULE, ARITH, 4>(a, num_sms, stream);
