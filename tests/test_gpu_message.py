@@ -174,3 +174,29 @@ def test_full_size_25m_messages():
     os_ = o.state()
     compare_states([x[idx] for x in gs[:4]] + [gs[4]], [x[idx] for x in os_[:4]] + [os_[4]],
                    oracle.FASGD, "25M messages")
+
+
+@pytest.mark.slow
+def test_message_vbar_bits_at_25m():
+    """The per-message statistic (Sec. 2.3: the mean of v over every parameter)
+    at P = 25,000,000, bit for bit against the oracle's exact mean, on v
+    spread over six decades, with zeros mixed in, and on v of two adjacent
+    floats (a mean that sits between them)."""
+    import torch
+    from paper_1601_04033_gb300 import fasgd
+    P = 25_000_000
+    rng = np.random.default_rng(2525)
+    srv = fasgd.Server(P, 2, 0.001, fasgd.FASGD, seed=SEED)
+    zeros = torch.zeros(P, device="cuda")
+    lo = np.float32(0.3)
+    cases = [
+        (10 ** rng.uniform(-3, 3, P)).astype(np.float32),
+        np.where(rng.random(P) < 0.3, 0.0, 10 ** rng.uniform(-2, 2, P)).astype(np.float32),
+        np.where(rng.random(P) < 0.5, lo, np.nextafter(lo, np.float32(1))).astype(np.float32),
+    ]
+    for k, v in enumerate(cases):
+        srv.set_state(zeros, zeros, zeros, torch.from_numpy(v).cuda(), 0)
+        got = srv.message_vbar()
+        want = oracle.mean_v(v)
+        assert np.float32(got).view(np.uint32) == np.float32(want).view(np.uint32), (k, got, want)
+    srv.close()
