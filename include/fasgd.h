@@ -404,6 +404,17 @@ FASGD_API int fasgd_sync(fasgd_t* h);
  */
 FASGD_API int fasgd_selftest_wait_expiry(fasgd_t* h);
 
+/*
+ * fasgd_selftest_fail_pass -- exercise the partial-failure path of
+ * fasgd_apply_pending without any GPU fault: the pass of fasgd_apply_pending
+ * that comes `after` passes from now (0: the next one) reports a launch
+ * failure (ECUDA) instead of being launched; nothing runs on the GPU for it.
+ * A pass is a fused run of dense pushes, a sparse push, or the update of a
+ * message or budget push (after its decision).  after = -1 switches it off.
+ * The paper has no counterpart; this is a test hook.  Errors: EINVAL.
+ */
+FASGD_API int fasgd_selftest_fail_pass(fasgd_t* h, int32_t after);
+
 /* Server timestamp T (pushes applied so far) and number of queued pushes. */
 FASGD_API int64_t fasgd_timestamp(const fasgd_t* h);
 FASGD_API int64_t fasgd_pending(const fasgd_t* h);

@@ -18,7 +18,7 @@
 // global stores.  A stage holds up to 8 gradient slices; larger K runs as
 // several stages per tile (the state travels with the first one only).  The
 // last P mod 2048 parameters are handled by plain loads in the last block.
-// Passes with fewer tiles than SMs use a plain grid instead (one quad of
+// Passes of fewer than 8 tiles per SM use a plain grid instead (one quad of
 // parameters per thread, fasgd_direct_kernel).
 //
 // With SUMS (one push, a.vsum set) the pass also leaves the float-float sum
@@ -337,13 +337,18 @@ cudaError_t launch_ch(const DenseArgs& a, int num_sms, cudaStream_t stream) {
 }
 
 // ---- small passes ------------------------------------------------------------
-// With fewer tiles than SMs the ring cannot give every SM a tile: its few
-// blocks stage, compute and store one tile each, and the last then runs the
-// tail.  A plain grid with one quad of parameters per thread and all of a
-// thread's loads issued before its arithmetic makes one round trip to memory
-// instead.  Small working sets stay in L2 between passes, so the gradient
-// loads keep the default cache policy here.
+// With few tiles per SM the ring's staging does not pay: its blocks stage,
+// compute and store a handful of tiles each, and the last then runs the tail.
+// A plain grid with one quad of parameters per thread and all of a thread's
+// loads issued before its arithmetic makes one round trip to memory instead.
+// Measured per pass (graph replay, K = 1 / 8): equal or faster up to
+// 2.5M parameters (7,850: 2.1 / 3.4 us against 3.4 / 6.7 us; 1.29M: 5.0 /
+// 10.7 us against 5.5 / 13.1 us), behind the ring from about 5M (K = 1:
+// 23.5 against 18.1 us), so it takes passes below 8 tiles per SM.  Such
+// working sets stay in L2 between passes, so the gradient loads keep the
+// default cache policy here.
 constexpr int kDirectThreads = 128;
+constexpr int kDirectTilesPerSm = 8;
 
 template <int RULE, int ARITH>
 __global__ void __launch_bounds__(kDirectThreads)
@@ -419,7 +424,7 @@ cudaError_t launch_rule(const DenseArgs& a, int num_sms, cudaStream_t stream) {
             return launch_ch<RULE, ARITH, 1, true>(a, num_sms, stream);
         }
     }
-    if (a.P / kTile < num_sms) return launch_direct<RULE, ARITH>(a, num_sms, stream);
+    if (a.P / kTile < kDirectTilesPerSm * num_sms) return launch_direct<RULE, ARITH>(a, num_sms, stream);
     // Gradient slices per stage: K rounded up to a power of two, at most 8.
     if (a.K > 4) return launch_ch<RULE, ARITH, 8>(a, num_sms, stream);
     if (a.K > 2) return launch_ch<RULE, ARITH, 4>(a, num_sms, stream);

@@ -128,6 +128,16 @@ struct fasgd_s {
     std::deque<Push> fifo;
     int64_t T = 0;
     int64_t launches = 0;
+    // Test hook (fasgd_selftest_fail_pass): the pass of fasgd_apply_pending
+    // this many passes from now reports a launch failure instead of running;
+    // -1: off.
+    int32_t fail_pass_in = -1;
+    // True when the next pass is the one to fail (the countdown advances).
+    bool injected_failure() {
+        if (fail_pass_in < 0) return false;
+        if (fail_pass_in-- > 0) return false;
+        return true;
+    }
     std::vector<uint64_t> push_count;
     std::vector<uint64_t> fetch_count;
     std::string err;
@@ -784,7 +794,10 @@ int fasgd_apply_pending(fasgd_t* h, int32_t K) {
                 const int slot = h->fifo[(size_t)(k + i)].stage;
                 if (slot >= 0) st = cudaStreamWaitEvent(h->stream, h->slot_ready[(size_t)slot], 0);
             }
-            if (st == cudaSuccess) st = fasgd::launch_dense(a, rule, h->exact, h->num_sms, h->stream, &h->launches);
+            if (st == cudaSuccess)
+                st = h->injected_failure()
+                         ? cudaErrorLaunchFailure
+                         : fasgd::launch_dense(a, rule, h->exact, h->num_sms, h->stream, &h->launches);
             ++h->pass_seq;
             for (int i = 0; i < r && st == cudaSuccess; ++i) {  // the slots may be refilled after this
                 const int slot = h->fifo[(size_t)(k + i)].stage;
@@ -817,7 +830,9 @@ int fasgd_apply_pending(fasgd_t* h, int32_t K) {
                 a.coef[0] = h->coef(h->T + k - first.j);
                 a.K = 1;
                 if (rule != fasgd::kRuleSgd) a.vsum = h->msg_chunks;   // keep the chunk sums current
-                st = fasgd::launch_dense(a, rule, h->exact, h->num_sms, h->stream, &h->launches);
+                st = h->injected_failure()
+                         ? cudaErrorLaunchFailure
+                         : fasgd::launch_dense(a, rule, h->exact, h->num_sms, h->stream, &h->launches);
                 h->msg_sums_valid = st == cudaSuccess;
             }
             if (st != cudaSuccess) {
@@ -837,7 +852,9 @@ int fasgd_apply_pending(fasgd_t* h, int32_t K) {
                 fasgd::RangeArgs r = h->range_args();
                 r.grad = first.grad;
                 r.coef = h->coef(h->T + k - first.j);
-                st = fasgd::launch_tensor_apply(r, rule, h->exact, h->stream, &h->launches);
+                st = h->injected_failure()
+                         ? cudaErrorLaunchFailure
+                         : fasgd::launch_tensor_apply(r, rule, h->exact, h->stream, &h->launches);
             }
             if (st != cudaSuccess) {
                 h->push_count[(size_t)first.client] = count0;   // a retry redraws the same decision
@@ -860,7 +877,10 @@ int fasgd_apply_pending(fasgd_t* h, int32_t K) {
             a.sp = sp;
             a.err = h->dev_err;
             if (first.n_max > 0 || first.n_dev != nullptr) {
-                cudaError_t st = fasgd::launch_sparse(a, rule, h->exact, h->num_sms, h->stream, &h->launches);
+                cudaError_t st = h->injected_failure()
+                                     ? cudaErrorLaunchFailure
+                                     : fasgd::launch_sparse(a, rule, h->exact, h->num_sms, h->stream,
+                                                            &h->launches);
                 if (st != cudaSuccess) return partial_fail(st, "sparse pass", k);
             }
             k += 1;
@@ -1142,6 +1162,13 @@ int fasgd_selftest_wait_expiry(fasgd_t* h) {
     cudaError_t st = fasgd::launch_wait_expiry(h->dev_err, h->stream);
     if (st != cudaSuccess) return h->cuda_fail(st, "fasgd_selftest_wait_expiry");
     ++h->launches;
+    return FASGD_OK;
+}
+
+int fasgd_selftest_fail_pass(fasgd_t* h, int32_t after) {
+    if (h == nullptr) return FASGD_EINVAL;
+    if (after < -1) return h->fail(FASGD_EINVAL, "after must be >= -1");
+    h->fail_pass_in = after;
     return FASGD_OK;
 }
 

@@ -46,6 +46,7 @@ SIGNATURES = {
     "fasgd_set_push_counts": (_i32, [_p, _p]),
     "fasgd_sync": (_i32, [_p]),
     "fasgd_selftest_wait_expiry": (_i32, [_p]),
+    "fasgd_selftest_fail_pass": (_i32, [_p, _i32]),
     "fasgd_timestamp": (_i64, [_p]),
     "fasgd_pending": (_i64, [_p]),
     "fasgd_kernel_launches": (_i64, [_p]),
@@ -225,6 +226,10 @@ def fasgd_sync(h):
 
 def fasgd_selftest_wait_expiry(h):
     return LIB.fasgd_selftest_wait_expiry(h)
+
+
+def fasgd_selftest_fail_pass(h, after):
+    return LIB.fasgd_selftest_fail_pass(h, after)
 
 
 def fasgd_timestamp(h):
@@ -429,6 +434,10 @@ class Server:
     def selftest_wait_expiry(self):
         """Enqueue the pipeline-wait expiry self-test (the next sync reports EDEVICE)."""
         self._check(fasgd_selftest_wait_expiry(self.h))
+
+    def selftest_fail_pass(self, after: int):
+        """Make the pass of apply_pending `after` passes from now report a launch failure."""
+        self._check(fasgd_selftest_fail_pass(self.h, after))
 
     @property
     def T(self) -> int:

@@ -152,3 +152,66 @@ def test_a_pipeline_wait_that_never_completes_is_reported():
     srv.sync()
     assert srv.T == 2
     srv.close()
+
+
+@pytest.mark.parametrize("fail_at", [0, 1, 2, 3, 4])
+def test_apply_pending_failing_partway_applies_each_push_once(fail_at):
+    """Failure partway through a mixed batch, made on the host (the injected
+    pass reports a launch failure and nothing runs for it): the call returns
+    ECUDA, the pushes before the failed pass have left the queue and T has
+    advanced by their number, the failed message or budget push keeps its
+    draw counter; a retry of the rest then leaves the state bit for bit
+    where one uninterrupted apply of the whole batch leaves it.  Passes of
+    the batch: 0 two fused dense pushes, 1 a message push, 2 a sparse push,
+    3 a budget push, 4 a dense push."""
+    import torch
+    from paper_1601_04033_gb300 import fasgd
+    P, lam = 20_011, 4
+    gen = torch.Generator(device="cuda").manual_seed(11)
+    grads = [torch.randn(P, device="cuda", generator=gen) * 0.05 for _ in range(5)]
+    idx = torch.arange(0, P, 3, dtype=torch.int32, device="cuda")
+    val = grads[3][idx.long()].contiguous()
+    theta0 = torch.randn(P, device="cuda", generator=gen) * 0.01
+
+    def server():
+        srv = fasgd.Server(P, lam, 0.01, fasgd.FASGD, c_push=3.0, seed=5)
+        srv.set_params(theta0)
+        srv.set_tensors([5000, 7011, 8000])
+        return srv
+
+    def queue(srv):
+        srv.push(0, 0, grads[0])
+        srv.push(1, 0, grads[1])
+        srv.push_message(2, 0, grads[2])
+        srv.push_sparse(3, 0, idx, val)
+        srv.push_budget(1, 0, grads[4], 9000)
+        srv.push(0, 0, grads[0])
+
+    ref = server()
+    queue(ref)
+    ref.apply_pending(6)
+    srv = server()
+    queue(srv)
+    pushes_before = [0, 2, 3, 4, 5][fail_at]     # pushes of the passes before the failed one
+    srv.selftest_fail_pass(fail_at)
+    with pytest.raises(fasgd.FasgdError) as e:
+        srv.apply_pending(6)
+    assert e.value.code == fasgd.ECUDA
+    assert f"{pushes_before} of 6 pushes were applied" in str(e.value)
+    assert srv.T == pushes_before and srv.pending == 6 - pushes_before
+    counts = list(srv.push_counts())
+    assert counts[2] == (1 if pushes_before > 2 else 0)      # the message push's draw
+    assert counts[1] == (1 if pushes_before > 4 else 0)      # the budget push's draw
+    srv.apply_pending(6 - pushes_before)
+    srv.sync()
+    ref.sync()
+    assert srv.T == ref.T == 6 and srv.pending == 0
+    assert list(srv.push_counts()) == list(ref.push_counts())
+    a = [torch.empty(P, device="cuda") for _ in range(4)]
+    b = [torch.empty(P, device="cuda") for _ in range(4)]
+    srv.get_state(*a)
+    ref.get_state(*b)
+    for x, y, name in zip(a, b, ("theta", "n", "b", "v")):
+        assert torch.equal(x, y), name
+    srv.close()
+    ref.close()

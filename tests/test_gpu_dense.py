@@ -70,13 +70,14 @@ def test_tiny_and_ragged(P):
 
 @pytest.mark.parametrize("delta", [-1, 0, 5])
 def test_small_pass_threshold(delta):
-    """P on both sides of the switch between the plain-grid pass (fewer tiles
-    of 2048 than SMs) and the bulk-copy ring: both against the oracle, K = 3."""
+    """P on both sides of the switch between the plain-grid pass (fewer than
+    8 tiles of 2048 per SM) and the bulk-copy ring: both against the oracle,
+    K = 3."""
     import torch
     sms = torch.cuda.get_device_properties(0).multi_processor_count
     w = W["fasgd-25m-k8"].replace(R=8)
-    run_parity(w, oracle.FASGD, sms * 2048 + delta, 300, 3)
-    run_parity(w, oracle.ASGD, sms * 2048 + delta, 300, 3)
+    run_parity(w, oracle.FASGD, 8 * sms * 2048 + delta, 300, 3)
+    run_parity(w, oracle.ASGD, 8 * sms * 2048 + delta, 300, 3)
 
 
 def test_fused_equals_sequential_bitwise():
