@@ -6,7 +6,9 @@ every T that is a multiple of lcm(100, K), to the end of the stream.
 
 At P = 25M and 2^28 the oracle runs on sampled parameters alone: the update
 is elementwise, so that sub-problem is exact.  The B-FASGD stream compares
-every push's list bit for bit and the whole state every 100 pushes."""
+every push's list bit for bit and the whole state every 100 pushes; the
+per-message and per-tensor rules (Sec. 2.3 and Sec. 5) compare every
+decision and the state every 100 pushes over the same 10,000-push stream."""
 
 import math
 
@@ -115,3 +117,70 @@ def test_bfasgd_full_stream():
             compare_states(g.state(), o.state(), oracle.FASGD, f"bfasgd full stream T={t + 1}")
     g.srv.sync()
     assert 0.17 < sent / (P * w.pushes) < 0.23
+
+
+def test_message_rule_full_stream():
+    """The paper's literal per-message B-FASGD (Sec. 2.3) over the B-FASGD
+    workload's whole 10,000-push stream (lambda = 64, Poisson(8) staleness)
+    at P = 100,003: every decision equal to the oracle's, the state within
+    the bound every 100 pushes."""
+    import torch
+    w = W["bfasgd-message-25m"].replace(R=8)
+    P = 100_003
+    pool = streams.gradient_pool(w, P)
+    th0 = streams.theta0(w, P)
+    seed = 0x3E55A6E
+    g = GpuRun(w, oracle.FASGD, P, pool, th0, c_push=40.0, seed=seed)
+    o = OracleRun(w, oracle.FASGD, P, pool, th0, c_push=40.0, seed=seed)
+    ps = streams.push_stream(w, w.pushes, 1)
+    flags = torch.full((w.pushes,), -1, dtype=torch.int32, device="cuda")
+    for t in range(w.pushes):
+        cl, js, sl = ps.batch(t)
+        c, j, s = int(cl[0]), int(js[0]), int(sl[0])
+        g.srv.push_message(c, j, g.pool[s], sent_dev=flags[t:t + 1])
+        g.srv.apply_pending(1)
+        o.srv.push_message(c, j, pool[s])
+        o.srv.apply_pending(1)
+        if (t + 1) % 100 == 0:
+            compare_states(g.state(), o.state(), oracle.FASGD, f"message stream T={t + 1}")
+            got = flags[:t + 1].cpu().numpy()
+            want = np.array(o.srv.message_log, dtype=np.int32)
+            assert np.array_equal(got, want), f"decisions differ by T={t + 1}"
+    assert 0 < int(flags.sum()) < w.pushes
+
+
+def test_budget_rule_full_stream():
+    """Per-tensor B-FASGD under a 20 % budget over the workload's whole
+    10,000-push stream at P = 100,003 in 17 tensors (fast arithmetic): every
+    push's decisions and count equal to the oracle's, its threshold within
+    1e-5, the state within the bound every 100 pushes."""
+    import torch
+    w = W["bfasgd-tensor-25m"].replace(R=8)
+    P = 100_003
+    sizes = streams.tensor_sizes(5, P, 17)
+    pool = streams.gradient_pool(w, P)
+    th0 = streams.theta0(w, P)
+    seed = 0xB0D6E7
+    g = GpuRun(w, oracle.FASGD, P, pool, th0, seed=seed)
+    o = OracleRun(w, oracle.FASGD, P, pool, th0, seed=seed)
+    g.srv.set_tensors(sizes)
+    o.srv.set_tensors(sizes)
+    sent = torch.zeros(len(sizes), dtype=torch.uint8, device="cuda")
+    cth = torch.zeros(1, dtype=torch.float32, device="cuda")
+    cnt = torch.zeros(1, dtype=torch.int64, device="cuda")
+    budget = P // 5
+    ps = streams.push_stream(w, w.pushes, 1)
+    for t in range(w.pushes):
+        cl, js, sl = ps.batch(t)
+        c, j, s = int(cl[0]), int(js[0]), int(sl[0])
+        g.srv.push_budget(c, j, g.pool[s], budget, sent, cth, cnt)
+        g.srv.apply_pending(1)
+        o.srv.push_budget(c, j, pool[s], budget)
+        o.srv.apply_pending(1)
+        osent, oc, om = o.srv.budget_log[-1]
+        assert np.array_equal(sent.cpu().numpy(), osent), f"decisions differ at push {t}"
+        assert int(cnt.item()) == om, t
+        gc = float(cth.item())
+        assert gc == oc or abs(gc - oc) <= 1e-5 * abs(oc), (t, gc, oc)
+        if (t + 1) % 100 == 0:
+            compare_states(g.state(), o.state(), oracle.FASGD, f"budget stream T={t + 1}")
