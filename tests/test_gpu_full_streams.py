@@ -184,3 +184,37 @@ def test_budget_rule_full_stream():
         assert gc == oc or abs(gc - oc) <= 1e-5 * abs(oc), (t, gc, oc)
         if (t + 1) % 100 == 0:
             compare_states(g.state(), o.state(), oracle.FASGD, f"budget stream T={t + 1}")
+
+
+def test_budget_rule_full_stream_exact_mode_bitwise():
+    """The same per-tensor rule in exact arithmetic (fasgd_set_exact) over the
+    whole 10,000-push stream at P = 300,007 in 160 tensors: v is then the
+    same on both sides, so every push's tensor means, threshold c, decisions
+    and count equal the oracle's bit for bit, and so does the final state."""
+    import torch
+    w = W["bfasgd-tensor-25m"].replace(R=8)
+    P = 300_007
+    sizes = streams.tensor_sizes(5, P, 160)
+    pool = streams.gradient_pool(w, P)
+    th0 = streams.theta0(w, P)
+    seed = 0xB0D6E7
+    g = GpuRun(w, oracle.FASGD, P, pool, th0, seed=seed, exact=True)
+    o = OracleRun(w, oracle.FASGD, P, pool, th0, seed=seed)
+    g.srv.set_tensors(sizes)
+    o.srv.set_tensors(sizes)
+    sent = torch.zeros(len(sizes), dtype=torch.uint8, device="cuda")
+    cth = torch.zeros(1, dtype=torch.float32, device="cuda")
+    cnt = torch.zeros(1, dtype=torch.int64, device="cuda")
+    ps = streams.push_stream(w, w.pushes, 1)
+    for t in range(w.pushes):
+        cl, js, sl = ps.batch(t)
+        c, j, s = int(cl[0]), int(js[0]), int(sl[0])
+        g.srv.push_budget(c, j, g.pool[s], P // 5, sent, cth, cnt)
+        g.srv.apply_pending(1)
+        o.srv.push_budget(c, j, pool[s], P // 5)
+        o.srv.apply_pending(1)
+        osent, oc, om = o.srv.budget_log[-1]
+        assert np.array_equal(sent.cpu().numpy(), osent), f"decisions differ at push {t}"
+        assert int(cnt.item()) == om, t
+        assert np.float32(cth.item()).view(np.uint32) == np.float32(oc).view(np.uint32), t
+    compare_states(g.state(), o.state(), oracle.FASGD, "exact budget stream", exact=True)
