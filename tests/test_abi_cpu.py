@@ -128,3 +128,10 @@ def test_handleless_calls_check_their_arguments_on_the_host(binding):
         args = list(good)
         args[k] = bad
         assert L.fasgd_sim_quadratic_loss(*args) == f.EINVAL, (k, bad)
+
+
+def test_c_callers_compile_and_link():
+    """The header is plain C: the C timing driver of the ABI (abi_latency.c)
+    compiles as C11 and links against the library."""
+    exe = build.build_latency_driver(force=True)
+    assert os.path.exists(exe) and os.access(exe, os.X_OK)
