@@ -409,7 +409,8 @@ FASGD_API int fasgd_selftest_wait_expiry(fasgd_t* h);
  * fasgd_apply_pending without any GPU fault: the pass of fasgd_apply_pending
  * that comes `after` passes from now (0: the next one) reports a launch
  * failure (ECUDA) instead of being launched; nothing runs on the GPU for it.
- * A pass is a fused run of dense pushes, a sparse push, or the update of a
+ * A pass is a fused run of dense pushes, a sparse push (one whose list is
+ * known to be empty launches nothing and is not counted), or the update of a
  * message or budget push (after its decision).  after = -1 switches it off.
  * The paper has no counterpart; this is a test hook.  Errors: EINVAL.
  */
