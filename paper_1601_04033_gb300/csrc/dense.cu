@@ -41,11 +41,17 @@
 namespace fasgd {
 namespace {
 
-constexpr int kConsumers = 512;                 // consumer threads per block
-constexpr int kTile = 4 * kConsumers;           // parameters per tile
-constexpr int kThreads = kConsumers + 32;       // + one producer warp
+// Ring geometry per consumer count CONS (threads that compute; 512 or 256):
+// tiles of 4 CONS parameters, CONS + 32 threads per block (one producer
+// warp), 512 / CONS blocks per SM sharing 220 KB of shared memory.
+template <int CONS> struct Geom {
+    static constexpr int kTile = 4 * CONS;
+    static constexpr int kThreads = CONS + 32;
+    static constexpr int kBlocksPerSm = 512 / CONS;
+    static constexpr int kSmemBudget = 220 * 1024 / kBlocksPerSm;   // ring + barriers, per block
+};
+constexpr int kTile = Geom<512>::kTile;         // the reference tile (2048 parameters)
 constexpr int kMaxStages = 8;
-constexpr int kSmemBudget = 220 * 1024;         // ring + barriers, per block
 
 // ---- bulk async copy (the mbarrier wrappers and bounded waits: wait.cuh) ----
 // 1-D bulk copy global -> shared (16-byte aligned, size a multiple of 16),
@@ -76,13 +82,13 @@ __device__ __forceinline__ void update4(float4& th, float4& n, float4& b, float4
     }
 }
 
-// Parameters [begin, P) with plain loads, by the consumer threads of one
-// block; begin is a multiple of 4.
-template <int RULE, int ARITH>
+// Parameters [begin, P) with plain loads, by the CONS consumer threads of
+// one block; begin is a multiple of 4.
+template <int RULE, int ARITH, int CONS>
 __device__ void apply_range_direct(const DenseArgs& a, int64_t begin, int tid) {
     constexpr bool FAS = RULE != kRuleSgd;
     const int64_t end_q = a.P & ~int64_t(3);
-    for (int64_t e = begin + 4 * (int64_t)tid; e < end_q; e += 4 * (int64_t)kConsumers) {
+    for (int64_t e = begin + 4 * (int64_t)tid; e < end_q; e += 4 * (int64_t)CONS) {
         float4 th = *reinterpret_cast<const float4*>(a.theta + e);
         float4 n = make_float4(0.f, 0.f, 0.f, 0.f), b = n, v = n;
         if (FAS) {
@@ -126,14 +132,14 @@ __device__ void apply_range_direct(const DenseArgs& a, int64_t begin, int tid) {
 }
 
 // The SUMS form of the tail: parameters [begin, P) chunk by chunk, consumer
-// warp w taking chunks begin/128 + w, + 16, ...; lane l updates parameters
-// 4l .. 4l + 3 of the chunk (guarded at P) and the warp forms the chunk's sum
-// of the new v in registers.  begin is a multiple of 2048.
-template <int RULE, int ARITH>
+// warp w taking chunks begin/128 + w, + CONS/32, ...; lane l updates
+// parameters 4l .. 4l + 3 of the chunk (guarded at P) and the warp forms the
+// chunk's sum of the new v in registers.  begin is a multiple of 128.
+template <int RULE, int ARITH, int CONS>
 __device__ void apply_range_chunks(const DenseArgs& a, int64_t begin, int tid) {
     const int warp = tid >> 5, lane = tid & 31;
     const int64_t nch = (a.P + kVsumChunk - 1) / kVsumChunk;
-    for (int64_t c = begin / kVsumChunk + warp; c < nch; c += kConsumers / 32) {
+    for (int64_t c = begin / kVsumChunk + warp; c < nch; c += CONS / 32) {
         const int64_t e = c * kVsumChunk + 4 * lane;
         float th[4] = {0.f, 0.f, 0.f, 0.f}, n[4] = {0.f, 0.f, 0.f, 0.f};
         float b[4] = {0.f, 0.f, 0.f, 0.f}, v[4] = {0.f, 0.f, 0.f, 0.f};
@@ -173,12 +179,15 @@ struct Ring {
 
 // RULE: kRuleSgd / kRuleFasgd / kRuleFasgdStd; ARITH: kArithApprox /
 // kArithApproxFtz / kArithExact (see update.cuh); CH: gradient slices per stage;
-// SUMS: also leave the chunk sums of the new v (FASGD rules, K = 1).
-template <int RULE, int ARITH, int CH, bool SUMS>
-__global__ void __launch_bounds__(kThreads, 1)
+// SUMS: also leave the chunk sums of the new v (FASGD rules, K = 1); CONS:
+// consumer threads per block (the ring geometry, Geom).
+template <int RULE, int ARITH, int CH, bool SUMS, int CONS>
+__global__ void __launch_bounds__(Geom<CONS>::kThreads, Geom<CONS>::kBlocksPerSm)
 fasgd_dense_kernel(const __grid_constant__ DenseArgs a, const Ring ring, const int64_t ntiles) {
     constexpr bool FAS = RULE != kRuleSgd;
     constexpr int kState = FAS ? 4 : 1;              // theta (, n, b, v)
+    constexpr int kTile = Geom<CONS>::kTile;
+    constexpr int kConsumers = CONS;
     constexpr int kStageFloats = (kState + CH) * kTile;
     extern __shared__ __align__(128) unsigned char smem[];
     float* buf = reinterpret_cast<float*>(smem);
@@ -301,19 +310,20 @@ fasgd_dense_kernel(const __grid_constant__ DenseArgs a, const Ring ring, const i
     // Parameters after the last full tile.
     if (ok && blockIdx.x == gridDim.x - 1) {
         if (SUMS)
-            apply_range_chunks<RULE, ARITH>(a, ntiles * kTile, tid);
+            apply_range_chunks<RULE, ARITH, CONS>(a, ntiles * kTile, tid);
         else
-            apply_range_direct<RULE, ARITH>(a, ntiles * kTile, tid);
+            apply_range_direct<RULE, ARITH, CONS>(a, ntiles * kTile, tid);
     }
 }
 
-template <int RULE, int ARITH, int CH, bool SUMS = false>
+template <int RULE, int ARITH, int CH, bool SUMS = false, int CONS = 512>
 cudaError_t launch_ch(const DenseArgs& a, int num_sms, cudaStream_t stream) {
+    using G = Geom<CONS>;
     constexpr int kState = RULE != kRuleSgd ? 4 : 1;
-    constexpr int kStageBytes = (kState + CH) * kTile * 4;
+    constexpr int kStageBytes = (kState + CH) * G::kTile * 4;
     Ring ring;
     ring.chunks = (a.K + CH - 1) / CH;
-    ring.stages = (kSmemBudget - 2 * kMaxStages * 8) / kStageBytes;
+    ring.stages = (G::kSmemBudget - 2 * kMaxStages * 8) / kStageBytes;
     if (ring.stages > kMaxStages) ring.stages = kMaxStages;
     const size_t smem = (size_t)ring.stages * kStageBytes + 2 * ring.stages * sizeof(uint64_t);
     // The shared-memory limit is a per-device attribute of the kernel: set it
@@ -324,15 +334,18 @@ cudaError_t launch_ch(const DenseArgs& a, int num_sms, cudaStream_t stream) {
     if (st != cudaSuccess) return st;
     const uint64_t bit = dev < 64 ? 1ull << dev : 0;
     if (bit == 0 || !(configured.load(std::memory_order_acquire) & bit)) {
-        st = cudaFuncSetAttribute(fasgd_dense_kernel<RULE, ARITH, CH, SUMS>,
-                                  cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBudget);
+        st = cudaFuncSetAttribute(fasgd_dense_kernel<RULE, ARITH, CH, SUMS, CONS>,
+                                  cudaFuncAttributeMaxDynamicSharedMemorySize, G::kSmemBudget);
         if (st != cudaSuccess) return st;
         configured.fetch_or(bit, std::memory_order_acq_rel);
     }
-    const int64_t ntiles = a.P / kTile;
-    int64_t grid = ntiles < num_sms ? ntiles : num_sms;  // one block per SM (shared-memory bound)
+    const int64_t ntiles = a.P / G::kTile;
+    // kBlocksPerSm blocks per SM (shared-memory bound), never more than there are tiles.
+    const int64_t slots = (int64_t)G::kBlocksPerSm * num_sms;
+    int64_t grid = ntiles < slots ? ntiles : slots;
     if (grid < 1) grid = 1;
-    fasgd_dense_kernel<RULE, ARITH, CH, SUMS><<<(unsigned)grid, kThreads, smem, stream>>>(a, ring, ntiles);
+    fasgd_dense_kernel<RULE, ARITH, CH, SUMS, CONS>
+        <<<(unsigned)grid, G::kThreads, smem, stream>>>(a, ring, ntiles);
     return cudaGetLastError();
 }
 
@@ -426,6 +439,11 @@ cudaError_t launch_rule(const DenseArgs& a, int num_sms, cudaStream_t stream) {
     }
     if (a.P / kTile < kDirectTilesPerSm * num_sms) return launch_direct<RULE, ARITH>(a, num_sms, stream);
     // Gradient slices per stage: K rounded up to a power of two, at most 8.
+    // K > 8 takes several stages per tile: two blocks of 256 consumers per SM
+    // keep more stages in flight there (P = 50M, K = 16: 686.8 against
+    // 704.0 us per pass); up to K = 8 one block of 512 is faster (226.8
+    // against 232.1 us at P = 25M, K = 8).
+    if (a.K > 8) return launch_ch<RULE, ARITH, 8, false, 256>(a, num_sms, stream);
     if (a.K > 4) return launch_ch<RULE, ARITH, 8>(a, num_sms, stream);
     if (a.K > 2) return launch_ch<RULE, ARITH, 4>(a, num_sms, stream);
     if (a.K > 1) return launch_ch<RULE, ARITH, 2>(a, num_sms, stream);

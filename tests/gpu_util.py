@@ -139,3 +139,41 @@ def run_parity(w, variant, P, n_pushes, K, check_every=None, real="f32", **hp):
             checks += 1
     assert checks > 0
     return g, o
+
+
+def ring_P(extra: int = 500_017) -> int:
+    """A parameter count the bulk-copy ring (not the plain-grid pass) handles
+    on this GPU: 8 tiles of 2048 per SM, plus a ragged remainder."""
+    torch = torch_cuda()
+    return 8 * torch.cuda.get_device_properties(0).multi_processor_count * 2048 + extra
+
+
+def run_parity_sampled(w, variant, P, n_pushes, K, count=20_000, **hp):
+    """Like run_parity, but the oracle runs on `count` sampled parameters only
+    (the update is elementwise, so that sub-problem is exact); compared at
+    every T multiple of lcm(100, K)."""
+    torch = torch_cuda()
+    every = 100 * K // math.gcd(100, K)
+    pool = streams.gradient_pool(w, P)
+    th0 = streams.theta0(w, P)
+    ps = streams.push_stream(w, n_pushes, K)
+    idx = streams.sample_indices(P, count)
+    g = GpuRun(w, variant, P, pool, th0, **hp)
+    o = OracleRun(w, variant, idx.size, np.ascontiguousarray(pool[:, idx]), th0[idx], **hp)
+    del pool
+    idx_t = torch.from_numpy(idx).cuda()
+    full = [torch.empty(P, device="cuda") for _ in range(4)]
+    checks = 0
+    for b in range(n_pushes // K):
+        batch = ps.batch(b)
+        g.push_batch(*batch)
+        o.push_batch(*batch)
+        if ((b + 1) * K) % every == 0:
+            T = g.srv.get_state(*full)
+            gs = [x[idx_t].cpu().numpy() for x in full] + [T]
+            compare_states(gs, o.state(), variant, f"{w.name} var={variant} P={P} K={K} T={T} "
+                           "(sampled)", exact=bool(hp.get("exact", False)))
+            checks += 1
+    assert checks > 0
+    g.srv.sync()
+    return checks

@@ -5,7 +5,7 @@ import pytest
 
 import oracle
 from gpu_util import (GpuRun, OracleRun, assert_bitwise, assert_close, compare_states,
-                      run_parity)
+                      ring_P, run_parity, run_parity_sampled)
 from paper_1601_04033_gb300 import streams
 
 pytestmark = pytest.mark.gpu
@@ -66,6 +66,36 @@ def test_tiny_and_ragged(P):
     w = W["fasgd-7850"]
     for variant in (oracle.ASGD, oracle.FASGD):
         run_parity(w, variant, P, 100, 4, check_every=100)
+
+
+@pytest.mark.parametrize("K", [2, 3, 5, 13, 16, 32])
+def test_ring_pass_k_values(K):
+    """The bulk-copy ring at every chunk width (K up to 8: one stage per tile
+    and one block of 512 consumers per SM; K > 8: several stages per tile and
+    two blocks of 256 per SM), FASGD against the oracle on sampled
+    parameters, over lcm(100, K) pushes."""
+    w = W["fasgd-25m-k8"].replace(R=max(2 * K, 16))
+    run_parity_sampled(w, oracle.FASGD, ring_P(), 100 * K // np.gcd(100, K), K)
+
+
+@pytest.mark.parametrize("variant", [oracle.FASGD, oracle.FASGD_STD])
+@pytest.mark.parametrize("K,eps", [(1, 1e-4), (8, 1e-4), (13, 1e-4), (8, 0.0)])
+def test_ring_exact_mode_is_bitwise(variant, K, eps):
+    """Exact arithmetic on the ring (both geometries): theta, n, b and v equal
+    the oracle's fp32 sequence bit for bit on sampled parameters."""
+    w = W["fasgd-25m-k8"].replace(R=max(2 * K, 16))
+    run_parity_sampled(w, variant, ring_P(), 100 * K // np.gcd(100, K), K, eps=eps, exact=True)
+
+
+@pytest.mark.parametrize("variant,K,eps", [(oracle.FASGD_STD, 8, 1e-4), (oracle.FASGD, 16, 0.0),
+                                           (oracle.SASGD, 16, 1e-4)])
+def test_ring_other_rules(variant, K, eps):
+    """The ring with the divide-by-std rule, the subnormal-preserving MUFU
+    forms (eps = 0) and SASGD, against the oracle on sampled parameters."""
+    w = W["fasgd-25m-k8"].replace(R=max(2 * K, 16))
+    if variant == oracle.FASGD_STD:
+        w = w.replace(alpha=w.alpha * 1e-3)
+    run_parity_sampled(w, variant, ring_P(), 100 * K // np.gcd(100, K), K, eps=eps)
 
 
 @pytest.mark.parametrize("delta", [-1, 0, 5])
