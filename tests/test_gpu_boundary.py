@@ -215,3 +215,141 @@ def test_apply_pending_failing_partway_applies_each_push_once(fail_at):
         assert torch.equal(x, y), name
     srv.close()
     ref.close()
+
+
+@pytest.mark.parametrize("seed", [1, 2, 3])
+def test_random_protocol_against_oracle(seed):
+    """A random interleaving of every kind of call a server sees -- dense
+    pushes from device and from pinned host memory, caller sparse lists,
+    B-FASGD selects pushed as lists, per-message and per-tensor pushes,
+    applies of random K (some with a launch failure injected partway and
+    then retried), per-parameter, per-message and per-tensor fetches, and
+    checkpoint round trips -- against the oracle driven the same way, in
+    exact arithmetic: every list, decision and count bit for bit as it
+    happens, and the state, timestamp and draw counters bit for bit at the end."""
+    import torch
+    from paper_1601_04033_gb300 import fasgd
+    rng = np.random.default_rng(seed)
+    P, lam, R = 12_007, 4, 6
+    w = streams.WORKLOADS["bfasgd-tensor-25m"].replace(lam=lam, R=R)
+    sizes = streams.tensor_sizes(seed, P, 7)
+    pool = streams.gradient_pool(w, P)
+    th0 = streams.theta0(w, P)
+    hp = (0.95, 0.95, 1e-4, 2.0, 1e-8, 77 + seed)
+    srv = fasgd.Server(P, lam, 0.01, fasgd.FASGD)
+    srv.set_exact(True)
+    srv.set_hparams(*hp)
+    srv.set_fetch_threshold(1.5)
+    srv.set_params(torch.from_numpy(th0).cuda())
+    srv.set_tensors(sizes)
+    o = oracle.OracleServer(P, lam, 0.01, oracle.FASGD)
+    o.set_hparams(*hp)
+    o.set_fetch_threshold(1.5)
+    o.set_params(th0)
+    o.set_tensors(sizes)
+    _, dpool = fasgd.aligned_vectors(pool)
+    hpool = torch.from_numpy(pool).pin_memory()
+    keep = []                                   # device lists borrowed until applied
+    idx = torch.empty(P, dtype=torch.int32, device="cuda")
+    val = torch.empty(P, dtype=torch.float32, device="cuda")
+    cnt = torch.empty(1, dtype=torch.int64, device="cuda")
+    flag = torch.empty(1, dtype=torch.int32, device="cuda")
+    sent = torch.zeros(len(sizes), dtype=torch.uint8, device="cuda")
+    cdev = torch.zeros(1, dtype=torch.float32, device="cuda")
+    kinds = ["dense", "host", "list", "select", "message", "budget", "apply", "apply",
+             "fetch", "fetch_message", "fetch_budget", "checkpoint"]
+    for step in range(400):
+        kind = kinds[rng.integers(len(kinds))] if srv.pending < 20 else "apply"
+        c = int(rng.integers(lam))
+        T = srv.T
+        assert T == o.T and srv.pending == len(o.fifo), step
+        j = int(rng.integers(max(0, T - 5), T + 1))
+        s = int(rng.integers(R))
+        if kind == "dense":
+            srv.push(c, j, dpool[s])
+            o.push(c, j, pool[s])
+        elif kind == "host":
+            srv.push_host(c, j, hpool[s])
+            o.push(c, j, pool[s])
+        elif kind == "list":
+            li = np.sort(rng.choice(P, int(rng.integers(0, P // 3)), replace=False)).astype(np.int32)
+            lv = (rng.standard_normal(li.size) * 0.05).astype(np.float32)
+            di, dv = torch.from_numpy(li).cuda(), torch.from_numpy(lv).cuda()
+            keep.append((di, dv))
+            srv.push_sparse(c, j, di, dv)
+            o.push_sparse(c, j, li, lv)
+        elif kind == "select":
+            li, lv, lc = torch.empty_like(idx), torch.empty_like(val), torch.empty_like(cnt)
+            keep.append((li, lv, lc))
+            srv.select_compact(c, dpool[s], li, lv, lc)
+            oi, ov = o.select_compact(c, pool[s])
+            m = int(lc.item())
+            assert m == oi.size, step
+            assert_bitwise(li[:m].cpu().numpy(), oi, f"select idx {step}")
+            assert_bitwise(lv[:m].cpu().numpy(), ov, f"select val {step}")
+            srv.push_sparse(c, j, li, lv, n_dev=lc, n_max=P)
+            o.push_sparse(c, j, oi, ov)
+        elif kind == "message":
+            srv.push_message(c, j, dpool[s])
+            o.push_message(c, j, pool[s])
+        elif kind == "budget":
+            budget = int(rng.integers(0, P + 100))
+            srv.push_budget(c, j, dpool[s], budget)
+            o.push_budget(c, j, pool[s], budget)
+        elif kind == "apply":
+            if srv.pending == 0:
+                continue
+            K = int(rng.integers(1, min(srv.pending, 32) + 1))
+            T0 = srv.T
+            if rng.random() < 0.3:
+                srv.selftest_fail_pass(int(rng.integers(0, 3)))
+            try:
+                srv.apply_pending(K)
+            except fasgd.FasgdError as e:
+                assert e.code == fasgd.ECUDA
+                srv.selftest_fail_pass(-1)
+                done = srv.T - T0
+                assert srv.pending == len(o.fifo) - done
+                srv.apply_pending(K - done)
+            srv.selftest_fail_pass(-1)
+            o.apply_pending(K)
+        elif kind == "fetch":
+            srv.fetch_compact(c, idx, val, cnt)
+            oi, ov = o.fetch_compact(c)
+            m = int(cnt.item())
+            assert m == oi.size, step
+            assert_bitwise(idx[:m].cpu().numpy(), oi, f"fetch idx {step}")
+            assert_bitwise(val[:m].cpu().numpy(), ov, f"fetch val {step}")
+        elif kind == "fetch_message":
+            copy = torch.full((P,), 7.0, device="cuda")
+            srv.fetch_message(c, copy, fetched_dev=flag)
+            ocopy = np.full(P, 7.0, np.float32)
+            ok = o.fetch_message(c, ocopy)
+            assert int(flag.item()) == int(ok), step
+            assert_bitwise(copy.cpu().numpy(), ocopy, f"fetched copy {step}")
+        elif kind == "fetch_budget":
+            budget = int(rng.integers(0, P + 100))
+            copy = torch.full((P,), 7.0, device="cuda")
+            srv.fetch_budget(c, copy, budget, sent_dev=sent, c_dev=cdev)
+            ocopy = np.full(P, 7.0, np.float32)
+            osent, oc, _ = o.fetch_budget(c, ocopy, budget)
+            assert np.array_equal(sent.cpu().numpy(), osent), step
+            assert np.float32(cdev.item()).view(np.uint32) == np.float32(oc).view(np.uint32), step
+            assert_bitwise(copy.cpu().numpy(), ocopy, f"budget fetch copy {step}")
+        elif kind == "checkpoint" and srv.pending == 0:
+            st = [torch.empty(P, device="cuda") for _ in range(4)]
+            Tc = srv.get_state(*st)
+            srv.set_state(*st, Tc)
+    while srv.pending:
+        K = min(srv.pending, 32)
+        srv.apply_pending(K)
+        o.apply_pending(K)
+    srv.sync()
+    assert srv.T == o.T
+    assert list(srv.push_counts()) == o.push_count
+    assert list(srv.fetch_counts()) == o.fetch_count
+    out = [torch.empty(P, device="cuda") for _ in range(4)]
+    srv.get_state(*out)
+    for x, y, name in zip(out, o.state()[:4], ("theta", "n", "b", "v")):
+        assert_bitwise(x.cpu().numpy(), y.astype(np.float32), f"final {name}")
+    srv.close()
