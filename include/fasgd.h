@@ -131,7 +131,15 @@ FASGD_API int fasgd_set_hparams(fasgd_t* h, float gamma, float beta, float eps, 
  */
 FASGD_API int fasgd_set_exact(fasgd_t* h, int32_t exact);
 
-/* Stream every later call is enqueued on (a cudaStream_t; NULL = legacy default stream). */
+/*
+ * Stream every later call is enqueued on (a cudaStream_t; NULL = legacy
+ * default stream).  Work the handle already enqueued on the previous stream
+ * comes before anything it enqueues on the new one: the call records an event
+ * on the previous stream and makes the new stream wait for it (so neither
+ * stream may be in a stream capture that the other is not part of).
+ * Errors: EINVAL, EAGAIN (pushes pending), ECUDA (the event could not be
+ * recorded or waited on; the stream is not changed).
+ */
 FASGD_API int fasgd_set_stream(fasgd_t* h, void* stream);
 
 /*

@@ -125,6 +125,7 @@ struct fasgd_s {
     cudaStream_t pull_stream = nullptr;   // pulls run beside the next host copies
     cudaEvent_t order_ev = nullptr;
     cudaEvent_t pull_done_ev = nullptr;
+    cudaEvent_t switch_ev = nullptr;      // orders a new stream after the previous one
     std::deque<Push> fifo;
     int64_t T = 0;
     int64_t launches = 0;
@@ -363,6 +364,8 @@ struct fasgd_s {
         slot_free.clear();
         if (order_ev) cudaEventDestroy(order_ev);
         if (pull_done_ev) cudaEventDestroy(pull_done_ev);
+        if (switch_ev) cudaEventDestroy(switch_ev);
+        switch_ev = nullptr;
         if (copy_stream) cudaStreamDestroy(copy_stream);
         if (pull_stream) cudaStreamDestroy(pull_stream);
         order_ev = pull_done_ev = nullptr;
@@ -481,7 +484,17 @@ int fasgd_set_exact(fasgd_t* h, int32_t exact) {
 int fasgd_set_stream(fasgd_t* h, void* stream) {
     if (h == nullptr) return FASGD_EINVAL;
     if (!h->fifo.empty()) return h->fail(FASGD_EAGAIN, "pushes are pending");
-    h->stream = static_cast<cudaStream_t>(stream);
+    const cudaStream_t s = static_cast<cudaStream_t>(stream);
+    if (s == h->stream) return FASGD_OK;
+    // What the handle enqueued on the previous stream (passes, selects,
+    // copies, pulls) comes before anything it enqueues on the new one.
+    DeviceGuard g(h->device);
+    cudaError_t st = cudaSuccess;
+    if (h->switch_ev == nullptr) st = cudaEventCreateWithFlags(&h->switch_ev, cudaEventDisableTiming);
+    if (st == cudaSuccess) st = cudaEventRecord(h->switch_ev, h->stream);
+    if (st == cudaSuccess) st = cudaStreamWaitEvent(s, h->switch_ev, 0);
+    if (st != cudaSuccess) return h->cuda_fail(st, "fasgd_set_stream");
+    h->stream = s;
     return FASGD_OK;
 }
 
@@ -651,14 +664,21 @@ int bfasgd_set_tensors(fasgd_t* h, int32_t T, const int64_t* sizes) {
     if (st == cudaSuccess) st = cudaMalloc(reinterpret_cast<void**>(&h->t_vbar), (size_t)T * sizeof(float));
     if (st == cudaSuccess) st = cudaMalloc(reinterpret_cast<void**>(&h->t_dirty), (size_t)T);
     if (st == cudaSuccess) st = cudaMalloc(reinterpret_cast<void**>(&h->t_cprev), 2 * sizeof(long long));
-    if (st == cudaSuccess) st = cudaMemset(h->t_dirty, 1, (size_t)T);
-    if (st == cudaSuccess) st = cudaMemset(h->t_cprev, 0xff, 2 * sizeof(long long));   // none yet
+    // The tables are written on the handle's stream, ahead of the decisions
+    // that read them; the stream is drained before the host tables go away.
+    if (st == cudaSuccess) st = cudaMemsetAsync(h->t_dirty, 1, (size_t)T, h->stream);
     if (st == cudaSuccess)
-        st = cudaMemcpy(h->t_items, items.data(), ni * sizeof(fasgd::TensorItem), cudaMemcpyHostToDevice);
+        st = cudaMemsetAsync(h->t_cprev, 0xff, 2 * sizeof(long long), h->stream);   // none yet
     if (st == cudaSuccess)
-        st = cudaMemcpy(h->t_item_begin, begin.data(), begin.size() * sizeof(int32_t), cudaMemcpyHostToDevice);
+        st = cudaMemcpyAsync(h->t_items, items.data(), ni * sizeof(fasgd::TensorItem),
+                             cudaMemcpyHostToDevice, h->stream);
     if (st == cudaSuccess)
-        st = cudaMemcpy(h->t_sizes, sz.data(), sz.size() * sizeof(int32_t), cudaMemcpyHostToDevice);
+        st = cudaMemcpyAsync(h->t_item_begin, begin.data(), begin.size() * sizeof(int32_t),
+                             cudaMemcpyHostToDevice, h->stream);
+    if (st == cudaSuccess)
+        st = cudaMemcpyAsync(h->t_sizes, sz.data(), sz.size() * sizeof(int32_t),
+                             cudaMemcpyHostToDevice, h->stream);
+    if (st == cudaSuccess) st = cudaStreamSynchronize(h->stream);
     if (st != cudaSuccess) {
         h->free_tensors();
         return h->cuda_fail(st, "bfasgd_set_tensors");

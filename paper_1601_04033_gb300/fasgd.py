@@ -319,6 +319,11 @@ class Server:
             raise FasgdError(rc, fasgd_last_error(self.h))
         return rc
 
+    def set_stream(self, stream):
+        """Enqueue every later call on `stream` (a torch CUDA stream)."""
+        self._check(fasgd_set_stream(self.h, stream.cuda_stream))
+        self.stream = stream
+
     def close(self):
         if getattr(self, "h", None):
             fasgd_destroy(self.h)

@@ -353,3 +353,39 @@ def test_random_protocol_against_oracle(seed):
     for x, y, name in zip(out, o.state()[:4], ("theta", "n", "b", "v")):
         assert_bitwise(x.cpu().numpy(), y.astype(np.float32), f"final {name}")
     srv.close()
+
+
+def test_set_stream_orders_the_previous_streams_work():
+    """fasgd_set_stream: a fused pass of 8 pushes at P = 25M enqueued on one
+    stream, a switch to a second stream and a one-push pass enqueued there at
+    once leave the state of the nine pushes applied in order -- bit for bit
+    the state of the same calls on one stream.  (Were the second stream not
+    ordered after the first, its pass would read theta, n, b, v while the
+    first pass still writes them.)"""
+    import torch
+    from paper_1601_04033_gb300 import fasgd
+    P, K = 25_000_000, 8
+    gen = torch.Generator(device="cuda").manual_seed(11)
+    grads = torch.randn(K + 1, P, device="cuda", generator=gen) * 0.01
+    th0 = torch.randn(P, device="cuda", generator=gen) * 0.01
+    torch.cuda.synchronize()
+
+    def run(switch):
+        first, second = torch.cuda.Stream(), torch.cuda.Stream()
+        srv = fasgd.Server(P, 4, 0.001, fasgd.FASGD, stream=first)
+        srv.set_params(th0)
+        for k in range(K):
+            srv.push(k % 4, 0, grads[k])
+        srv.apply_pending(K)
+        if switch:
+            srv.set_stream(second)
+        srv.push(0, K, grads[K])
+        srv.apply_pending(1)
+        srv.sync()
+        out = [torch.empty(P, device="cuda") for _ in range(4)]
+        assert srv.get_state(*out) == K + 1
+        srv.close()
+        return out
+
+    for x, y in zip(run(False), run(True)):
+        assert torch.equal(x, y)
