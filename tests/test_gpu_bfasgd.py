@@ -394,3 +394,48 @@ def test_sparse_apply_divide_by_std_matches_dense_at_c0():
     for x, y, name in zip(a.state()[:4], b.state()[:4], ("theta", "n", "b", "v")):
         assert_bitwise(x, y, name)
     compare_states(a.state(), o.state(), oracle.FASGD_STD, "std variant")
+
+
+def _mid_sizes():
+    """About 5M parameters (~600 tiles of 8,192): a whole number of tiles,
+    partial last tiles of 1 and 4,099 parameters, one short of a tile
+    boundary, and a size whose tile count is no multiple of the SM count."""
+    at = 608 * 8192
+    return [at - 1, at, at + 1, at + 4099, at + 97 * 8192 + 12_345]
+
+
+@pytest.mark.parametrize("which", range(5))
+def test_select_mid_sizes_bit_exact(which):
+    """Push and fetch selects at about 5M parameters against the oracle, for
+    thresholds in both forms of the Eq. 9 test (c below and above 2^79) and two
+    calls of each stream."""
+    import torch
+    P = _mid_sizes()[which]
+    rng = np.random.default_rng(P)
+    g = (rng.standard_normal(P) * 0.1).astype(np.float32)
+    for lo, hi, cs in ((-1, 2, (0.0, 5.0, float("inf"))), (28, 34, (1e30,))):
+        v = (10 ** rng.uniform(lo, hi, P)).astype(np.float32)
+        g_t, v_t = torch.from_numpy(g).cuda(), torch.from_numpy(v).cuda()
+        for c in cs:
+            srv = _server(P, c=c)
+            srv.set_fetch_threshold(c)
+            srv.set_params(g_t)             # fetches compact theta = g
+            for call in range(2):
+                gi, gv, m, _ = _select_gpu(srv, 5, g_t, v_t)
+                oi, ov = oracle.select(g, v, np.float32(c), 1e-8, SEED, 5, call)
+                assert m == oi.size, (P, c, call, m, oi.size)
+                if 0.0 < c < float("inf"):
+                    assert 0 < m < P
+                assert_bitwise(gi, oi, f"push idx P={P} c={c}")
+                assert_bitwise(gv, ov, f"push val P={P} c={c}")
+                idx = torch.empty(P, dtype=torch.int32, device="cuda")
+                val = torch.empty(P, dtype=torch.float32, device="cuda")
+                n = torch.empty(1, dtype=torch.int64, device="cuda")
+                srv.fetch_compact(5, idx, val, n, v=v_t)
+                fm = int(n.item())
+                fi, fv = oracle.fetch_select(g, v, np.float32(c), 1e-8, SEED, 5, call)
+                assert fm == fi.size, (P, c, call, fm, fi.size)
+                assert_bitwise(idx[:fm].cpu().numpy(), fi, f"fetch idx P={P} c={c}")
+                assert_bitwise(val[:fm].cpu().numpy(), fv, f"fetch val P={P} c={c}")
+            srv.sync()
+            srv.close()
