@@ -332,8 +332,10 @@ __global__ void __launch_bounds__(kTensorResolveThreads) budget_resolve_kernel(c
                                 (!w_interp || (span << m) <= w_prev_span);
             long long nc;
             if (interp) {
-                const double f = (double)(w_elo - a.limit) / (double)(w_elo - w_ehi);  // in (0, 1]
-                long long xs = nlo + (long long)(f * (double)span);
+                // f in (0, 1] only guides where the candidates go, so fp32
+                // does (fp64 is a slow pipe here, on the round's critical path).
+                const float f = (float)(w_elo - a.limit) / (float)(w_elo - w_ehi);
+                long long xs = nlo + (long long)(f * (float)span);
                 xs = xs <= nlo ? nlo + 1 : (xs >= nhi ? nhi - 1 : xs);
                 const int h = (1 << (m - 1)) - 1;
                 const int j = lane - h;

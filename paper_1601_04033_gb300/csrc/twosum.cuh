@@ -75,7 +75,9 @@ __device__ __forceinline__ float2 chunk_sum4(float4 v) {
 // about 2^-43 (relative) of a rounding boundary.
 __device__ __forceinline__ float ff_div_int(float h, float l, int32_t s) {
     const float sh = __int2float_rn(s);
-    const float sl = __ll2float_rn((long long)s - __float2ll_rn(sh));
+    // s - sh is an integer of magnitude at most 64 (sh may round up to 2^31,
+    // so the difference is taken modulo 2^32 in unsigned arithmetic).
+    const float sl = __int2float_rn((int32_t)((uint32_t)s - __float2uint_rn(sh)));
     const float q0 = __fdiv_rn(h, sh);
     const float e1 = __fmaf_rn(-q0, sh, h);
     const float r = __fsub_rn(__fadd_rn(e1, l), __fmul_rn(q0, sl));
