@@ -217,16 +217,18 @@ def test_apply_pending_failing_partway_applies_each_push_once(fail_at):
     ref.close()
 
 
-@pytest.mark.parametrize("seed", [1, 2, 3])
-def test_random_protocol_against_oracle(seed):
+@pytest.mark.parametrize("variant,seed", [("FASGD", 1), ("FASGD", 2), ("FASGD", 3),
+                                          ("SASGD", 4), ("ASGD", 5), ("FASGD_STD", 6)])
+def test_random_protocol_against_oracle(variant, seed):
     """A random interleaving of every kind of call a server sees -- dense
     pushes from device and from pinned host memory, caller sparse lists,
     B-FASGD selects pushed as lists, per-message and per-tensor pushes,
     applies of random K (some with a launch failure injected partway and
     then retried), per-parameter, per-message and per-tensor fetches, and
     checkpoint round trips -- against the oracle driven the same way, in
-    exact arithmetic: every list, decision and count bit for bit as it
-    happens, and the state, timestamp and draw counters bit for bit at the end."""
+    exact arithmetic, for each update rule: every list, decision and count bit
+    for bit as it happens, and the state, timestamp and draw counters bit for
+    bit at the end."""
     import torch
     from paper_1601_04033_gb300 import fasgd
     rng = np.random.default_rng(seed)
@@ -236,13 +238,14 @@ def test_random_protocol_against_oracle(seed):
     pool = streams.gradient_pool(w, P)
     th0 = streams.theta0(w, P)
     hp = (0.95, 0.95, 1e-4, 2.0, 1e-8, 77 + seed)
-    srv = fasgd.Server(P, lam, 0.01, fasgd.FASGD)
+    alpha = 1e-5 if variant == "FASGD_STD" else 0.01   # the divide-by-std steps are ~1/std^2 larger
+    srv = fasgd.Server(P, lam, alpha, getattr(fasgd, variant))
     srv.set_exact(True)
     srv.set_hparams(*hp)
     srv.set_fetch_threshold(1.5)
     srv.set_params(torch.from_numpy(th0).cuda())
     srv.set_tensors(sizes)
-    o = oracle.OracleServer(P, lam, 0.01, oracle.FASGD)
+    o = oracle.OracleServer(P, lam, alpha, getattr(oracle, variant))
     o.set_hparams(*hp)
     o.set_fetch_threshold(1.5)
     o.set_params(th0)
