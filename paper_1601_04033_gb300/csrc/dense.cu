@@ -26,6 +26,10 @@
 // in a.vsum, formed in registers, so the next per-message decision needs no
 // pass over v (message.cu forms the same chunk sums from v, bit for bit).
 //
+// Both kernels are launched as programmatic dependents (pdl.cuh): a pass is
+// scheduled while the kernel before it on the stream drains, sets up its
+// barriers, and waits (griddepcontrol.wait) before it touches memory.
+//
 // Every wait on an mbarrier is bounded (about one second of wall clock);
 // on expiry the block sets flag 8 of the error word, waits (bounded) for its
 // own copies in flight, and returns.  Elements are independent, so the
@@ -34,6 +38,7 @@
 #include <atomic>
 
 #include "kernels.cuh"
+#include "pdl.cuh"
 #include "twosum.cuh"
 #include "update.cuh"
 #include "wait.cuh"
@@ -204,6 +209,8 @@ fasgd_dense_kernel(const __grid_constant__ DenseArgs a, const Ring ring, const i
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
     __syncthreads();
+    pdl_wait();      // the kernel before this one on the stream is complete
+    pdl_trigger();
 
     if (warp == kConsumerWarps) {
         // ---------------- producer: one elected lane ----------------
@@ -344,9 +351,8 @@ cudaError_t launch_ch(const DenseArgs& a, int num_sms, cudaStream_t stream) {
     const int64_t slots = (int64_t)G::kBlocksPerSm * num_sms;
     int64_t grid = ntiles < slots ? ntiles : slots;
     if (grid < 1) grid = 1;
-    fasgd_dense_kernel<RULE, ARITH, CH, SUMS, CONS>
-        <<<(unsigned)grid, G::kThreads, smem, stream>>>(a, ring, ntiles);
-    return cudaGetLastError();
+    return launch_pdl(fasgd_dense_kernel<RULE, ARITH, CH, SUMS, CONS>, (unsigned)grid,
+                      G::kThreads, smem, stream, a, ring, ntiles);
 }
 
 // ---- small passes ------------------------------------------------------------
@@ -368,6 +374,8 @@ __global__ void __launch_bounds__(kDirectThreads)
 fasgd_direct_kernel(const __grid_constant__ DenseArgs a) {
     constexpr bool FAS = RULE != kRuleSgd;
     constexpr bool STD = RULE == kRuleFasgdStd;
+    pdl_wait();
+    pdl_trigger();
     const int64_t nq = (a.P + 3) / 4;  // quads; the last may be partial
     for (int64_t q = (int64_t)blockIdx.x * kDirectThreads + threadIdx.x; q < nq;
          q += (int64_t)gridDim.x * kDirectThreads) {
@@ -425,8 +433,7 @@ cudaError_t launch_direct(const DenseArgs& a, int num_sms, cudaStream_t stream) 
     const int64_t nq = (a.P + 3) / 4;
     int64_t grid = (nq + kDirectThreads - 1) / kDirectThreads;
     if (grid > 8 * (int64_t)num_sms) grid = 8 * (int64_t)num_sms;
-    fasgd_direct_kernel<RULE, ARITH><<<(unsigned)grid, kDirectThreads, 0, stream>>>(a);
-    return cudaGetLastError();
+    return launch_pdl(fasgd_direct_kernel<RULE, ARITH>, (unsigned)grid, kDirectThreads, 0, stream, a);
 }
 
 template <int RULE, int ARITH>
