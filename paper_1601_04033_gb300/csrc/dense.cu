@@ -25,6 +25,11 @@
 // of the new v over every 128-parameter chunk (one warp's share of a tile)
 // in a.vsum, formed in registers, so the next per-message decision needs no
 // pass over v (message.cu forms the same chunk sums from v, bit for bit).
+// A SUMS pass of a per-message push also takes the push's Eq. 9 decision
+// itself (a.msg: every block's warp 0 combines the statistic's partials in
+// the decision kernel's order, message_decide) and, if the push is
+// transmitted, applies the pushed gradient while copying it into the
+// client's cache slot; if dropped it applies the slot.
 //
 // Both kernels are launched as programmatic dependents (pdl.cuh): a pass is
 // scheduled while the kernel before it on the stream drains, sets up its
@@ -38,6 +43,7 @@
 #include <atomic>
 
 #include "kernels.cuh"
+#include "message.cuh"
 #include "pdl.cuh"
 #include "twosum.cuh"
 #include "update.cuh"
@@ -136,12 +142,14 @@ __device__ void apply_range_direct(const DenseArgs& a, int64_t begin, int tid) {
     }
 }
 
-// The SUMS form of the tail: parameters [begin, P) chunk by chunk, consumer
-// warp w taking chunks begin/128 + w, + CONS/32, ...; lane l updates
-// parameters 4l .. 4l + 3 of the chunk (guarded at P) and the warp forms the
+// The SUMS form of the tail (one push): parameters [begin, P) chunk by
+// chunk, consumer warp w taking chunks begin/128 + w, + CONS/32, ...; lane l
+// updates parameters 4l .. 4l + 3 of the chunk (guarded at P) with gradient
+// g0, copying it to copy_to unless that is null, and the warp forms the
 // chunk's sum of the new v in registers.  begin is a multiple of 128.
 template <int RULE, int ARITH, int CONS>
-__device__ void apply_range_chunks(const DenseArgs& a, int64_t begin, int tid) {
+__device__ void apply_range_chunks(const DenseArgs& a, int64_t begin, int tid, const float* g0,
+                                   float* copy_to) {
     const int warp = tid >> 5, lane = tid & 31;
     const int64_t nch = (a.P + kVsumChunk - 1) / kVsumChunk;
     for (int64_t c = begin / kVsumChunk + warp; c < nch; c += CONS / 32) {
@@ -156,13 +164,14 @@ __device__ void apply_range_chunks(const DenseArgs& a, int64_t begin, int tid) {
                 b[j] = a.b[e + j];
                 v[j] = a.v[e + j];
             }
-        for (int k = 0; k < a.K; ++k)
 #pragma unroll
-            for (int j = 0; j < 4; ++j)
-                if (e + j < a.P)
-                    rule_update<ARITH, RULE == kRuleFasgdStd>(th[j], n[j], b[j], v[j],
-                                                              __ldcs(a.grad[k] + e + j),
-                                                              a.coef[k], a.sp);
+        for (int j = 0; j < 4; ++j)
+            if (e + j < a.P) {
+                const float g = __ldcs(g0 + e + j);
+                if (copy_to != nullptr) copy_to[e + j] = g;
+                rule_update<ARITH, RULE == kRuleFasgdStd>(th[j], n[j], b[j], v[j], g, a.coef[0],
+                                                          a.sp);
+            }
 #pragma unroll
         for (int j = 0; j < 4; ++j)
             if (e + j < a.P) {
@@ -211,6 +220,32 @@ fasgd_dense_kernel(const __grid_constant__ DenseArgs a, const Ring ring, const i
     __syncthreads();
     pdl_wait();      // the kernel before this one on the stream is complete
     pdl_trigger();
+    // A message push decided here (SUMS, a.msg.partial set): warp 0 takes the
+    // decision, every thread reads it.  Transmitted: apply the pushed gradient
+    // and copy it into the client's cache slot; dropped: apply the slot.
+    const float* g0 = a.grad[0];
+    float* copy_to = nullptr;
+    if constexpr (SUMS) {
+        __shared__ uint32_t s_send;
+        if (a.msg.partial != nullptr) {
+            if (warp == 0) {
+                float vbar;
+                const uint32_t send = message_decide(a.msg.partial, a.msg.nblocks, a.P, a.msg.c,
+                                                     a.msg.eps_b, a.msg.round_key0,
+                                                     a.msg.round_key1, a.msg.client_word,
+                                                     a.msg.n_lo, a.msg.n_hi, &vbar);
+                if (lane == 0) {
+                    s_send = send;
+                    if (blockIdx.x == 0 && a.msg.flag_out != nullptr) *a.msg.flag_out = (int32_t)send;
+                }
+            }
+            __syncthreads();
+            if (s_send) {
+                g0 = a.msg.src;
+                copy_to = a.msg.slot;
+            }
+        }
+    }
 
     if (warp == kConsumerWarps) {
         // ---------------- producer: one elected lane ----------------
@@ -240,7 +275,8 @@ fasgd_dense_kernel(const __grid_constant__ DenseArgs a, const Ring ring, const i
                     }
                     float* gs = st + kState * kTile;
                     for (int j = 0; j < ng; ++j)
-                        bulk_load(gs + j * kTile, a.grad[k0 + j] + off, kTile * 4, &full[s]);
+                        bulk_load(gs + j * kTile, (k0 + j == 0 ? g0 : a.grad[k0 + j]) + off,
+                                  kTile * 4, &full[s]);
                     issued |= 1u << s;
                     issued_phase = (issued_phase & ~(1u << s)) | (ph << s);
                     if (++s == ring.stages) {
@@ -283,6 +319,8 @@ fasgd_dense_kernel(const __grid_constant__ DenseArgs a, const Ring ring, const i
                 for (int j = 0; j < CH; ++j) g[j] = gs[j * (kTile / 4) + tid];
                 __syncwarp();
                 if (lane == 0) mbar_arrive(&empty[s]);  // inputs are in registers
+                if (SUMS && copy_to != nullptr)          // a transmitted message refreshes its slot
+                    reinterpret_cast<float4*>(copy_to + t * kTile)[tid] = g[0];
 #pragma unroll
                 for (int j = 0; j < CH; ++j) update4<RULE, ARITH>(th, n, b, v, g[j], a.coef[k0 + j], a.sp);
             } else {               // the last, partial chunk
@@ -317,7 +355,7 @@ fasgd_dense_kernel(const __grid_constant__ DenseArgs a, const Ring ring, const i
     // Parameters after the last full tile.
     if (ok && blockIdx.x == gridDim.x - 1) {
         if (SUMS)
-            apply_range_chunks<RULE, ARITH, CONS>(a, ntiles * kTile, tid);
+            apply_range_chunks<RULE, ARITH, CONS>(a, ntiles * kTile, tid, g0, copy_to);
         else
             apply_range_direct<RULE, ARITH, CONS>(a, ntiles * kTile, tid);
     }

@@ -22,6 +22,22 @@ struct StatParams {
     float eps;
 };
 
+// A per-message push decided inside its pass (with vsum, FASGD rules): the
+// pass first takes the push's Eq. 9 decision from the statistic's partials
+// (message_decide); if transmitted it applies src and copies it into slot
+// (the client's gradient cache slot, which is also grad[0]), else it applies
+// grad[0] as it stands.  partial == null: no decision, grad[0] is applied.
+struct PassMessage {
+    const float2* partial;          // nblocks float-float partial sums of v
+    int32_t nblocks;
+    float c, eps_b;
+    uint32_t round_key0[10], round_key1[10];
+    uint32_t client_word, n_lo, n_hi;
+    const float* src;               // the pushed gradient, fp32[P], 16-byte aligned
+    float* slot;                    // == grad[0]
+    int32_t* flag_out;              // may be null: 1 transmitted, 0 dropped
+};
+
 // One fused pass over the parameters applying K dense pushes in order.
 struct DenseArgs {
     float* theta;
@@ -36,6 +52,7 @@ struct DenseArgs {
     int32_t* err;                   // device error flags (bit 3: a pipeline wait expired)
     float2* vsum;                   // if set (K = 1, FASGD rules): the float-float sum of
                                     // the new v over every 128-parameter chunk
+    PassMessage msg;                // with vsum only
 };
 // Parameters per chunk of the per-message statistic's partial sums.
 constexpr int kVsumChunk = 128;

@@ -19,7 +19,11 @@
 // launch and every GPU.  For a push, src is the client's gradient and dst its
 // slot of the server's gradient cache (the pass that follows reads the
 // slot, so a dropped push re-applies the client's last sent gradient); for a
-// fetch, src is theta and dst the client's copy.
+// fetch, src is theta and dst the client's copy.  Under the FASGD rules a
+// push skips kernel 2: the pass that applies it takes the same decision
+// (message_decide, message.cuh) and refreshes the slot as it streams
+// (dense.cu); kernel 2 serves fetches, the statistic query and ASGD/SASGD
+// pushes.
 
 #include "eq9.cuh"
 #include "kernels.cuh"
@@ -106,24 +110,11 @@ __global__ void __launch_bounds__(kMsgThreads) message_resolve_kernel(const __gr
     pdl_wait();
     pdl_trigger();
     if (threadIdx.x < 32) {
-        const int lane = threadIdx.x;
-        float h = 0.f, l = 0.f;
-        // Lane l adds partials l, l + 32, ... in order, eight loads in flight.
-        for (int b = lane; b < a.nblocks; b += 8 * 32) {
-            float2 x[8];
-#pragma unroll
-            for (int k = 0; k < 8; ++k)
-                if (b + 32 * k < a.nblocks) x[k] = a.partial[b + 32 * k];
-#pragma unroll
-            for (int k = 0; k < 8; ++k)
-                if (b + 32 * k < a.nblocks) ff_add(h, l, x[k].x, x[k].y);
-        }
-        ff_warp_sum(h, l);
-        if (lane == 0) {
-            const float vbar = ff_div_int(h, l, (int32_t)a.P);
-            const Philox4 r = philox4x32_10(0xFFFFFFFFu, a.client_word, a.n_lo, a.n_hi,
-                                            a.round_key0, a.round_key1);
-            const uint32_t send = send_bit(r.x[0] >> 8, vbar, a.c, a.eps_b);
+        float vbar;
+        const uint32_t send = message_decide(a.partial, a.nblocks, a.P, a.c, a.eps_b,
+                                             a.round_key0, a.round_key1, a.client_word, a.n_lo,
+                                             a.n_hi, &vbar);
+        if (threadIdx.x == 0) {
             s_send = send;
             if (blockIdx.x == 0 && a.flag_out != nullptr) *a.flag_out = (int32_t)send;
             if (blockIdx.x == 0 && a.vbar_out != nullptr) *a.vbar_out = vbar;
@@ -149,11 +140,16 @@ int32_t message_partial_blocks(int64_t P) {
     return (int32_t)b;
 }
 
+cudaError_t launch_message_partials(const MessageArgs& a, cudaStream_t stream, int64_t* launches) {
+    const cudaError_t st = launch_pdl(vbar_partial_kernel, a.nblocks, kMsgThreads, 0, stream, a);
+    if (st == cudaSuccess) ++*launches;
+    return st;
+}
+
 cudaError_t launch_message(const MessageArgs& a, int num_sms, cudaStream_t stream,
                            int64_t* launches) {
-    cudaError_t st = launch_pdl(vbar_partial_kernel, a.nblocks, kMsgThreads, 0, stream, a);
+    cudaError_t st = launch_message_partials(a, stream, launches);
     if (st != cudaSuccess) return st;
-    ++*launches;
     int64_t grid = ((a.P >> 2) + kMsgThreads - 1) / kMsgThreads;
     const int64_t cap = (int64_t)(num_sms > 0 ? num_sms : 1) * 8;
     if (grid > cap) grid = cap;

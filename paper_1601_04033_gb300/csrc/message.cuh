@@ -1,7 +1,9 @@
 // Internal interface of the per-message B-FASGD kernels (message.cu) for the
 // host runtime.  Not part of the public C ABI.
 #pragma once
+#include "eq9.cuh"
 #include "kernels.cuh"
+#include "twosum.cuh"
 
 namespace fasgd {
 
@@ -33,5 +35,39 @@ int32_t message_partial_blocks(int64_t P);
 
 cudaError_t launch_message(const MessageArgs& a, int num_sms, cudaStream_t stream,
                            int64_t* launches);
+// The partials only (vbar_partial_kernel): for a decision the pass that
+// follows takes itself (message_decide).
+cudaError_t launch_message_partials(const MessageArgs& a, cudaStream_t stream, int64_t* launches);
+
+// The decision of one message from the nblocks partials vbar_partial_kernel
+// left, taken by one whole warp: lane l adds partials l, l + 32, ... in
+// order (eight loads in flight), then a fixed float-float shuffle tree,
+// vbar = fl32(sum / P) (ff_div_int), u = word 0 of Philox4x32-10 at counter
+// (2^32-1, client_word, n_lo, n_hi), the exact Eq. 9 test.  Every caller
+// forms the same bits.  Returns the decision (1: transmitted) in every lane
+// and vbar in *vbar.
+__device__ __forceinline__ uint32_t message_decide(const float2* partial, int32_t nblocks,
+                                                   int64_t P, float c, float eps_b,
+                                                   const uint32_t (&rk0)[10],
+                                                   const uint32_t (&rk1)[10],
+                                                   uint32_t client_word, uint32_t n_lo,
+                                                   uint32_t n_hi, float* vbar) {
+    const int lane = threadIdx.x & 31;
+    float h = 0.f, l = 0.f;
+    for (int b = lane; b < nblocks; b += 8 * 32) {
+        float2 x[8];
+#pragma unroll
+        for (int k = 0; k < 8; ++k)
+            if (b + 32 * k < nblocks) x[k] = partial[b + 32 * k];
+#pragma unroll
+        for (int k = 0; k < 8; ++k)
+            if (b + 32 * k < nblocks) ff_add(h, l, x[k].x, x[k].y);
+    }
+    ff_warp_sum(h, l);
+    const float vb = ff_div_int(h, l, (int32_t)P);
+    const Philox4 r = philox4x32_10(0xFFFFFFFFu, client_word, n_lo, n_hi, rk0, rk1);
+    *vbar = vb;
+    return send_bit(r.x[0] >> 8, vb, c, eps_b);
+}
 
 }  // namespace fasgd

@@ -282,11 +282,11 @@ struct fasgd_s {
         return st;
     }
 
-    // One per-message decision of `stream_id` for `client` (advancing its
-    // counter), copying src -> dst if transmitted.
-    cudaError_t launch_message(uint32_t stream_id, int32_t client, const float* src, float* dst,
-                               int32_t* flag, float c, std::vector<uint64_t>* counter,
-                               float* vbar_out = nullptr) {
+    // Arguments of one per-message decision of `stream_id` for `client`, its
+    // n-th message of that stream, copying src -> dst if transmitted.
+    fasgd::MessageArgs message_args(uint32_t stream_id, int32_t client, const float* src,
+                                    float* dst, int32_t* flag, float c, uint64_t n,
+                                    float* vbar_out) const {
         fasgd::MessageArgs a;
         std::memset(&a, 0, sizeof a);
         a.v = v;
@@ -298,7 +298,6 @@ struct fasgd_s {
         a.c = c;
         a.eps_b = eps_b;
         fasgd::philox_key_schedule(seed, a.round_key0, a.round_key1);
-        const uint64_t n = counter != nullptr ? (*counter)[(size_t)client] : 0;
         a.client_word = (uint32_t)client | (stream_id << 31);
         a.n_lo = (uint32_t)n;
         a.n_hi = (uint32_t)(n >> 32);
@@ -306,6 +305,16 @@ struct fasgd_s {
         a.dst = dst;
         a.flag_out = flag;
         a.vbar_out = vbar_out;
+        return a;
+    }
+
+    // One per-message decision of `stream_id` for `client` (advancing its
+    // counter), copying src -> dst if transmitted.
+    cudaError_t launch_message(uint32_t stream_id, int32_t client, const float* src, float* dst,
+                               int32_t* flag, float c, std::vector<uint64_t>* counter,
+                               float* vbar_out = nullptr) {
+        const uint64_t n = counter != nullptr ? (*counter)[(size_t)client] : 0;
+        const fasgd::MessageArgs a = message_args(stream_id, client, src, dst, flag, c, n, vbar_out);
         cudaError_t st = fasgd::launch_message(a, num_sms, stream, &launches);
         if (st == cudaSuccess) {
             msg_sums_valid = true;
@@ -831,28 +840,59 @@ int fasgd_apply_pending(fasgd_t* h, int32_t K) {
             k += r;
         } else if (first.kind == kMessage) {
             // Decide against the mean of v now, refresh the client's cache
-            // slot if the push is transmitted, then apply the slot.
+            // slot if the push is transmitted, then apply the slot.  Under the
+            // FASGD rules the pass itself takes the decision from the
+            // statistic's partials and, if transmitted, applies the pushed
+            // gradient while copying it into the slot.
             float* slot = h->grad_cache + (size_t)first.client * (size_t)h->cache_stride;
             const uint64_t count0 = h->push_count[(size_t)first.client];
-            cudaError_t st = h->launch_message(0, first.client, first.grad, slot, first.flag,
-                                               h->c_push, &h->push_count);
-            if (st == cudaSuccess) {
-                fasgd::DenseArgs a;
-                std::memset(&a, 0, sizeof a);
-                a.theta = h->theta;
-                a.n = h->n;
-                a.b = h->b;
-                a.v = h->v;
-                a.P = h->P;
-                a.sp = sp;
-                a.err = h->dev_err;
-                a.grad[0] = slot;
-                a.coef[0] = h->coef(h->T + k - first.j);
-                a.K = 1;
-                if (rule != fasgd::kRuleSgd) a.vsum = h->msg_chunks;   // keep the chunk sums current
-                st = h->injected_failure()
-                         ? cudaErrorLaunchFailure
-                         : fasgd::launch_dense(a, rule, h->exact, h->num_sms, h->stream, &h->launches);
+            fasgd::DenseArgs a;
+            std::memset(&a, 0, sizeof a);
+            a.theta = h->theta;
+            a.n = h->n;
+            a.b = h->b;
+            a.v = h->v;
+            a.P = h->P;
+            a.sp = sp;
+            a.err = h->dev_err;
+            a.grad[0] = slot;
+            a.coef[0] = h->coef(h->T + k - first.j);
+            a.K = 1;
+            cudaError_t st;
+            if (rule != fasgd::kRuleSgd) {
+                const fasgd::MessageArgs m =
+                    h->message_args(0, first.client, first.grad, slot, first.flag, h->c_push,
+                                    count0, nullptr);
+                st = fasgd::launch_message_partials(m, h->stream, &h->launches);
+                if (st == cudaSuccess) {
+                    a.vsum = h->msg_chunks;   // keep the chunk sums current
+                    a.msg.partial = m.partial;
+                    a.msg.nblocks = m.nblocks;
+                    a.msg.c = m.c;
+                    a.msg.eps_b = m.eps_b;
+                    std::memcpy(a.msg.round_key0, m.round_key0, sizeof a.msg.round_key0);
+                    std::memcpy(a.msg.round_key1, m.round_key1, sizeof a.msg.round_key1);
+                    a.msg.client_word = m.client_word;
+                    a.msg.n_lo = m.n_lo;
+                    a.msg.n_hi = m.n_hi;
+                    a.msg.src = first.grad;
+                    a.msg.slot = slot;
+                    a.msg.flag_out = first.flag;
+                    st = h->injected_failure()
+                             ? cudaErrorLaunchFailure
+                             : fasgd::launch_dense(a, rule, h->exact, h->num_sms, h->stream,
+                                                   &h->launches);
+                    if (st == cudaSuccess) h->push_count[(size_t)first.client] = count0 + 1;
+                }
+                h->msg_sums_valid = st == cudaSuccess;
+            } else {
+                st = h->launch_message(0, first.client, first.grad, slot, first.flag, h->c_push,
+                                       &h->push_count);
+                if (st == cudaSuccess)
+                    st = h->injected_failure()
+                             ? cudaErrorLaunchFailure
+                             : fasgd::launch_dense(a, rule, h->exact, h->num_sms, h->stream,
+                                                   &h->launches);
                 h->msg_sums_valid = st == cudaSuccess;
             }
             if (st != cudaSuccess) {
