@@ -51,7 +51,7 @@ def assert_bitwise(gpu, ora, what):
     assert bad.size == 0, f"{what}: {bad.size} elements differ, first at {bad[:5]}"
 
 
-class GpuRun:
+class CudaRun:
     """A CUDA-path server fed from a device-resident gradient pool."""
 
     def __init__(self, w: streams.Workload, variant: int, P: int, pool: np.ndarray,
@@ -125,7 +125,7 @@ def run_parity(w, variant, P, n_pushes, K, check_every=None, real="f32", **hp):
     pool = streams.gradient_pool(w, P)
     th0 = streams.theta0(w, P)
     ps = streams.push_stream(w, n_pushes, K)
-    g = GpuRun(w, variant, P, pool, th0, **hp)
+    g = CudaRun(w, variant, P, pool, th0, **hp)
     o = OracleRun(w, variant, P, pool, th0, real=real, **hp)
     checks = 0
     for b in range(n_pushes // K):
@@ -158,7 +158,7 @@ def run_parity_sampled(w, variant, P, n_pushes, K, count=20_000, **hp):
     th0 = streams.theta0(w, P)
     ps = streams.push_stream(w, n_pushes, K)
     idx = streams.sample_indices(P, count)
-    g = GpuRun(w, variant, P, pool, th0, **hp)
+    g = CudaRun(w, variant, P, pool, th0, **hp)
     o = OracleRun(w, variant, idx.size, np.ascontiguousarray(pool[:, idx]), th0[idx], **hp)
     del pool
     idx_t = torch.from_numpy(idx).cuda()

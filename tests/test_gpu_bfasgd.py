@@ -4,7 +4,7 @@ import numpy as np
 import pytest
 
 import oracle
-from gpu_util import (GpuRun, OracleRun, assert_bitwise, assert_close, compare_states)
+from gpu_util import (CudaRun, OracleRun, assert_bitwise, assert_close, compare_states)
 from paper_1601_04033_gb300 import streams
 from paper_1601_04033_gb300.calibrate import calibrate_c
 
@@ -57,7 +57,7 @@ def test_select_uses_live_v_when_v_is_null():
     w = W["bfasgd-25m"]
     pool = streams.gradient_pool(w, P, 4)
     th0 = streams.theta0(w, P)
-    g = GpuRun(w, oracle.FASGD, P, pool, th0, c_push=2.0, seed=SEED)
+    g = CudaRun(w, oracle.FASGD, P, pool, th0, c_push=2.0, seed=SEED)
     g.push_batch([0, 1], [0, 0], [0, 1])
     v_live = g.state()[3]
     gi, gv, m, _ = _select_gpu(g.srv, 3, g.pool[2])
@@ -75,7 +75,7 @@ def _bfasgd_stream(P, n_pushes, w, c_target=0.2, check_every=100):
     vsnap = [streams.client_v_snapshot(w, c, P) for c in range(lam)]
     c_push = calibrate_c(vsnap[0], c_target)
     ps = streams.push_stream(w, n_pushes, 1)
-    g = GpuRun(w, oracle.FASGD, P, pool, th0, c_push=c_push, seed=SEED)
+    g = CudaRun(w, oracle.FASGD, P, pool, th0, c_push=c_push, seed=SEED)
     o = OracleRun(w, oracle.FASGD, P, pool, th0, c_push=c_push, seed=SEED)
     vsnap_t = [torch.from_numpy(v).cuda() for v in vsnap]
     sent = 0
@@ -112,8 +112,8 @@ def test_bfasgd_c0_equals_dense_bitwise():
     pool = streams.gradient_pool(w, P, 8)
     th0 = streams.theta0(w, P)
     ps = streams.push_stream(w.replace(R=8), 40, 1)
-    a = GpuRun(w, oracle.FASGD, P, pool, th0)
-    b = GpuRun(w, oracle.FASGD, P, pool, th0, c_push=0.0, seed=SEED)
+    a = CudaRun(w, oracle.FASGD, P, pool, th0)
+    b = CudaRun(w, oracle.FASGD, P, pool, th0, c_push=0.0, seed=SEED)
     for t in range(40):
         cl, js, sl = ps.batch(t)
         a.push_batch(cl, js, sl)
@@ -130,7 +130,7 @@ def test_empty_list_leaves_state():
     w = W["bfasgd-25m"]
     P = 4099
     pool = streams.gradient_pool(w, P, 2)
-    g = GpuRun(w, oracle.FASGD, P, pool, streams.theta0(w, P), c_push=float("inf"))
+    g = CudaRun(w, oracle.FASGD, P, pool, streams.theta0(w, P), c_push=float("inf"))
     g.push_batch([0], [0], [0])
     before = g.state()
     _, _, m, (idx, val, n) = _select_gpu(g.srv, 1, g.pool[1])
@@ -203,7 +203,7 @@ def test_bfasgd_full_size_25m_sampled():
     vsnap = [streams.client_v_snapshot(w, c, P) for c in range(3)]
     c_push = calibrate_c(vsnap[0], 0.2)
     idx_s = streams.sample_indices(P, 20_000)
-    g = GpuRun(w, oracle.FASGD, P, pool, th0, c_push=c_push, seed=SEED)
+    g = CudaRun(w, oracle.FASGD, P, pool, th0, c_push=c_push, seed=SEED)
     o = OracleRun(w, oracle.FASGD, idx_s.size, np.ascontiguousarray(pool[:, idx_s]), th0[idx_s],
                   c_push=c_push, seed=SEED)
     pos = np.full(P, -1, np.int64)
@@ -239,7 +239,7 @@ def test_bfasgd_full_size_2_28_sampled():
     vsnap = [streams.client_v_snapshot(w, c, P) for c in range(2)]
     c_push = calibrate_c(vsnap[0][:: P // (1 << 22)], 0.2)
     idx_s = streams.sample_indices(P, 20_000)
-    g = GpuRun(w, oracle.FASGD, P, pool, th0, c_push=c_push, seed=SEED)
+    g = CudaRun(w, oracle.FASGD, P, pool, th0, c_push=c_push, seed=SEED)
     o = OracleRun(w, oracle.FASGD, idx_s.size, np.ascontiguousarray(pool[:, idx_s]), th0[idx_s],
                   c_push=c_push, seed=SEED)
     pos = np.full(P, -1, np.int64)
@@ -381,8 +381,8 @@ def test_sparse_apply_divide_by_std_matches_dense_at_c0():
     pool = streams.gradient_pool(w, P, 4)
     th0 = streams.theta0(w, P)
     ps = streams.push_stream(w.replace(R=4), 25, 1)
-    a = GpuRun(w, oracle.FASGD_STD, P, pool, th0)
-    b = GpuRun(w, oracle.FASGD_STD, P, pool, th0, c_push=0.0, seed=SEED)
+    a = CudaRun(w, oracle.FASGD_STD, P, pool, th0)
+    b = CudaRun(w, oracle.FASGD_STD, P, pool, th0, c_push=0.0, seed=SEED)
     o = OracleRun(w, oracle.FASGD_STD, P, pool, th0)
     for t in range(25):
         cl, js, sl = ps.batch(t)

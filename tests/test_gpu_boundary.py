@@ -4,7 +4,7 @@ import numpy as np
 import pytest
 
 import oracle
-from gpu_util import GpuRun, assert_bitwise
+from gpu_util import CudaRun, assert_bitwise
 from paper_1601_04033_gb300 import streams
 
 pytestmark = pytest.mark.gpu
@@ -91,8 +91,8 @@ def test_host_push_and_pull_match_device_path():
     pool = streams.gradient_pool(w, P, 8)
     th0 = streams.theta0(w, P)
     ps = streams.push_stream(w.replace(R=8, K=4), 40, 4)
-    a = GpuRun(w, oracle.FASGD, P, pool, th0)
-    b = GpuRun(w, oracle.FASGD, P, pool, th0)
+    a = CudaRun(w, oracle.FASGD, P, pool, th0)
+    b = CudaRun(w, oracle.FASGD, P, pool, th0)
     host_pool = torch.from_numpy(pool).pin_memory()
     out = torch.empty(P, dtype=torch.float32).pin_memory()
     for k in range(10):

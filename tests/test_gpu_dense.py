@@ -4,7 +4,7 @@ import numpy as np
 import pytest
 
 import oracle
-from gpu_util import (GpuRun, OracleRun, assert_bitwise, assert_close, compare_states,
+from gpu_util import (CudaRun, OracleRun, assert_bitwise, assert_close, compare_states,
                       ring_P, run_parity, run_parity_sampled)
 from paper_1601_04033_gb300 import streams
 
@@ -48,7 +48,7 @@ def test_against_fp64_oracle(variant):
     pool = streams.gradient_pool(w, P)
     th0 = streams.theta0(w, P)
     ps = streams.push_stream(w, 300, 1)
-    g = GpuRun(w, variant, P, pool, th0)
+    g = CudaRun(w, variant, P, pool, th0)
     o = OracleRun(w, variant, P, pool, th0, real="f64")
     for b in range(300):
         cl, js, sl = ps.batch(b)
@@ -117,8 +117,8 @@ def test_fused_equals_sequential_bitwise():
     pool = streams.gradient_pool(w, P)
     th0 = streams.theta0(w, P)
     ps = streams.push_stream(w, 64, 8)
-    a = GpuRun(w, oracle.FASGD, P, pool, th0)
-    b = GpuRun(w, oracle.FASGD, P, pool, th0)
+    a = CudaRun(w, oracle.FASGD, P, pool, th0)
+    b = CudaRun(w, oracle.FASGD, P, pool, th0)
     for k in range(8):
         cl, js, sl = ps.batch(k)
         a.push_batch(cl, js, sl)                 # one fused pass of 8
@@ -140,12 +140,12 @@ def test_checkpoint_restore_bitwise():
     pool = streams.gradient_pool(w, P)
     th0 = streams.theta0(w, P)
     ps = streams.push_stream(w, 120, 4)
-    a = GpuRun(w, oracle.FASGD, P, pool, th0)
+    a = CudaRun(w, oracle.FASGD, P, pool, th0)
     for k in range(15):
         a.push_batch(*ps.batch(k))
     mid = [torch.empty(P, device="cuda") for _ in range(4)]
     T = a.srv.get_state(*mid)
-    b = GpuRun(w, oracle.FASGD, P, pool, np.zeros(P, np.float32))
+    b = CudaRun(w, oracle.FASGD, P, pool, np.zeros(P, np.float32))
     b.srv.set_state(*mid, T)
     for k in range(15, 30):
         a.push_batch(*ps.batch(k))
@@ -164,7 +164,7 @@ def test_full_size_25m_k8_sampled():
     pool = streams.gradient_pool(w, P)
     th0 = streams.theta0(w, P)
     ps = streams.push_stream(w, 200, 8)
-    g = GpuRun(w, oracle.FASGD, P, pool, th0)
+    g = CudaRun(w, oracle.FASGD, P, pool, th0)
     for b in range(25):
         g.push_batch(*ps.batch(b))
     gs = g.state()
@@ -186,7 +186,7 @@ def test_full_size_268m_k16_sampled():
     pool = streams.gradient_pool(w, P)
     th0 = streams.theta0(w, P)
     ps = streams.push_stream(w, 64, 16)
-    g = GpuRun(w, oracle.FASGD, P, pool, th0)
+    g = CudaRun(w, oracle.FASGD, P, pool, th0)
     for b in range(4):
         g.push_batch(*ps.batch(b))
     idx = streams.sample_indices(P, 20_000)
@@ -253,7 +253,7 @@ def test_fast_arithmetic_outside_its_envelope(variant, hp):
     pool = streams.gradient_pool(w, P)
     th0 = streams.theta0(w, P)
     ps = streams.push_stream(w, n, K)
-    g = GpuRun(w, variant, P, pool, th0, **hp)
+    g = CudaRun(w, variant, P, pool, th0, **hp)
     o = OracleRun(w, variant, P, pool, th0, **hp)
     peak = np.abs(th0.astype(np.float64))
     for b in range(n):

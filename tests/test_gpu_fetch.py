@@ -5,7 +5,7 @@ import numpy as np
 import pytest
 
 import oracle
-from gpu_util import GpuRun, OracleRun, assert_bitwise, assert_close, compare_states
+from gpu_util import CudaRun, OracleRun, assert_bitwise, assert_close, compare_states
 from paper_1601_04033_gb300 import streams
 from paper_1601_04033_gb300.calibrate import calibrate_c
 
@@ -121,7 +121,7 @@ def test_bfasgd_round_trip_against_oracle():
     vs = [streams.client_v_snapshot(w, c, P) for c in range(w.lam)]
     c_push = calibrate_c(vs[0], 0.2)
     c_fetch = calibrate_c(vs[0], 0.1)
-    g = GpuRun(w, oracle.FASGD, P, pool, th0, c_push=c_push, seed=SEED)
+    g = CudaRun(w, oracle.FASGD, P, pool, th0, c_push=c_push, seed=SEED)
     o = OracleRun(w, oracle.FASGD, P, pool, th0, c_push=c_push, seed=SEED)
     g.srv.set_fetch_threshold(c_fetch)
     o.srv.set_fetch_threshold(c_fetch)

@@ -16,7 +16,7 @@ import numpy as np
 import pytest
 
 import oracle
-from gpu_util import GpuRun, OracleRun, assert_bitwise, compare_states, run_parity
+from gpu_util import CudaRun, OracleRun, assert_bitwise, compare_states, run_parity
 from paper_1601_04033_gb300 import streams
 from paper_1601_04033_gb300.calibrate import calibrate_c
 
@@ -43,7 +43,7 @@ def _sampled_stream(w, P, n_pushes, K, R=None):
     th0 = streams.theta0(wr, P)
     ps = streams.push_stream(wr, n_pushes, K)
     idx = streams.sample_indices(P, 20_000)
-    g = GpuRun(wr, oracle.FASGD, P, pool, th0)
+    g = CudaRun(wr, oracle.FASGD, P, pool, th0)
     o = OracleRun(wr, oracle.FASGD, idx.size, np.ascontiguousarray(pool[:, idx]), th0[idx])
     del pool
     idx_t = torch.from_numpy(idx).cuda()
@@ -92,7 +92,7 @@ def test_bfasgd_full_stream():
     c_push = calibrate_c(vsnap[0], 0.2)
     seed = 0xC0FFEE_1234_5678
     ps = streams.push_stream(w, w.pushes, 1)
-    g = GpuRun(w, oracle.FASGD, P, pool, th0, c_push=c_push, seed=seed)
+    g = CudaRun(w, oracle.FASGD, P, pool, th0, c_push=c_push, seed=seed)
     o = OracleRun(w, oracle.FASGD, P, pool, th0, c_push=c_push, seed=seed)
     vsnap_t = [torch.from_numpy(v).cuda() for v in vsnap]
     idx = torch.empty(P, dtype=torch.int32, device="cuda")
@@ -130,7 +130,7 @@ def test_message_rule_full_stream():
     pool = streams.gradient_pool(w, P)
     th0 = streams.theta0(w, P)
     seed = 0x3E55A6E
-    g = GpuRun(w, oracle.FASGD, P, pool, th0, c_push=40.0, seed=seed)
+    g = CudaRun(w, oracle.FASGD, P, pool, th0, c_push=40.0, seed=seed)
     o = OracleRun(w, oracle.FASGD, P, pool, th0, c_push=40.0, seed=seed)
     ps = streams.push_stream(w, w.pushes, 1)
     flags = torch.full((w.pushes,), -1, dtype=torch.int32, device="cuda")
@@ -161,7 +161,7 @@ def test_budget_rule_full_stream():
     pool = streams.gradient_pool(w, P)
     th0 = streams.theta0(w, P)
     seed = 0xB0D6E7
-    g = GpuRun(w, oracle.FASGD, P, pool, th0, seed=seed)
+    g = CudaRun(w, oracle.FASGD, P, pool, th0, seed=seed)
     o = OracleRun(w, oracle.FASGD, P, pool, th0, seed=seed)
     g.srv.set_tensors(sizes)
     o.srv.set_tensors(sizes)
@@ -198,7 +198,7 @@ def test_budget_rule_full_stream_exact_mode_bitwise():
     pool = streams.gradient_pool(w, P)
     th0 = streams.theta0(w, P)
     seed = 0xB0D6E7
-    g = GpuRun(w, oracle.FASGD, P, pool, th0, seed=seed, exact=True)
+    g = CudaRun(w, oracle.FASGD, P, pool, th0, seed=seed, exact=True)
     o = OracleRun(w, oracle.FASGD, P, pool, th0, seed=seed)
     g.srv.set_tensors(sizes)
     o.srv.set_tensors(sizes)

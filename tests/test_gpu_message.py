@@ -5,7 +5,7 @@ import numpy as np
 import pytest
 
 import oracle
-from gpu_util import GpuRun, OracleRun, assert_bitwise, compare_states
+from gpu_util import CudaRun, OracleRun, assert_bitwise, compare_states
 from paper_1601_04033_gb300 import streams
 
 pytestmark = pytest.mark.gpu
@@ -19,7 +19,7 @@ def _run_pair(P, n_push, c_push, lam=3, variant=oracle.FASGD):
     pool = streams.gradient_pool(w, P)
     th0 = streams.theta0(w, P)
     ps = streams.push_stream(w, n_push, 1)
-    g = GpuRun(w, variant, P, pool, th0, c_push=c_push, seed=SEED)
+    g = CudaRun(w, variant, P, pool, th0, c_push=c_push, seed=SEED)
     o = OracleRun(w, variant, P, pool, th0, c_push=c_push, seed=SEED)
     flags = torch.full((n_push,), -1, dtype=torch.int32, device="cuda")
     for t in range(n_push):
@@ -50,10 +50,10 @@ def test_message_c0_equals_dense_and_cinf_applies_zeros():
     pool = streams.gradient_pool(w, P)
     th0 = streams.theta0(w, P)
     ps = streams.push_stream(w, 30, 1)
-    a = GpuRun(w, oracle.FASGD, P, pool, th0, c_push=0.0, seed=SEED)
-    b = GpuRun(w, oracle.FASGD, P, pool, th0)
-    z = GpuRun(w, oracle.FASGD, P, pool, th0, c_push=float("inf"), seed=SEED)
-    zb = GpuRun(w, oracle.FASGD, P, np.zeros_like(pool), th0)
+    a = CudaRun(w, oracle.FASGD, P, pool, th0, c_push=0.0, seed=SEED)
+    b = CudaRun(w, oracle.FASGD, P, pool, th0)
+    z = CudaRun(w, oracle.FASGD, P, pool, th0, c_push=float("inf"), seed=SEED)
+    zb = CudaRun(w, oracle.FASGD, P, np.zeros_like(pool), th0)
     for t in range(30):
         cl, js, sl = ps.batch(t)
         c, j, s = int(cl[0]), int(js[0]), int(sl[0])
@@ -142,7 +142,7 @@ def test_full_size_25m_messages():
     P = w.P
     pool = streams.gradient_pool(w, P)
     th0 = streams.theta0(w, P)
-    g = GpuRun(w, oracle.FASGD, P, pool, th0, c_push=2.0, seed=SEED)
+    g = CudaRun(w, oracle.FASGD, P, pool, th0, c_push=2.0, seed=SEED)
     o = OracleRun(w, oracle.FASGD, P, pool, th0, c_push=2.0, seed=SEED)
     g.srv.set_fetch_threshold(4.0)
     o.srv.set_fetch_threshold(4.0)
