@@ -979,7 +979,113 @@ def check_budget_server(libs: Libs):
     assert a.fetch_count == [0, 3, 0]
 
 
-ALL_CHECKS = [
+# --------------------------------------------------------------------------
+# Protocol: batches in arrival order, draws keyed by the right stream and count
+# --------------------------------------------------------------------------
+def check_batched_apply_order(libs: Libs):
+    """Sec. 2.1: queued pushes are applied in arrival order, push k of a batch
+    at server timestamp T + k.  Batches of 1 to 5 pushes with mixed staleness
+    equal the fp64 series form with tau_k = T + k - j_k; the same pushes in
+    reverse arrival order do not."""
+    rng = np.random.default_rng(71)
+    P = 5
+    theta0 = (rng.standard_normal(P) * 0.01).astype(np.float32)
+    gamma, beta, eps, alpha = 0.8, 0.6, 1e-3, 0.05
+    sizes = [3, 1, 4, 2, 5]
+    batches, T = [], 0
+    for k in sizes:
+        batch = []
+        for _ in range(k):
+            g = (rng.standard_normal(P) * rng.choice([0.01, 0.5, 2.0])).astype(np.float32)
+            batch.append((T - min(int(rng.integers(0, 4)), T), g))
+        batches.append(batch)
+        T += k
+
+    def events(order):
+        out, T = [], 0
+        for batch in batches:
+            for k, (j, g) in enumerate(order(batch)):
+                out.append((T + k - j, {p: float(g[p]) for p in range(P)}))
+            T += len(batch)
+        return out
+
+    for variant in (SASGD, FASGD):
+        G, B = float(np.float32(gamma)), float(np.float32(beta))
+        E, A = float(np.float32(eps)), float(np.float32(alpha))
+        ref = _series_reference(variant, theta0, events(lambda b: b), A, G, B, E)
+        rev = _series_reference(variant, theta0, events(lambda b: b[::-1]), A, G, B, E)
+        assert _rel(rev[0], ref[0]) > 1e-6          # the order is visible in theta
+        s = _server(libs, "f64", P, variant, alpha=alpha, gamma=gamma, beta=beta, eps=eps)
+        s.set_params(theta0)
+        for batch in batches:
+            for c, (j, g) in enumerate(batch):
+                s.push(c % s.lam, j, g)
+            s.apply_pending(len(batch))
+        assert s.T == T and not s.fifo
+        for name, got, r in zip(("theta", "n", "b", "v"), s.state()[:4], ref):
+            bound = 1e-12 * (np.abs(r) + np.max(np.abs(r)) + 1e-30)
+            assert np.all(np.abs(got - r) <= bound), (variant, name)
+
+
+def check_fetch_draws_keyed_by_fetch_count(libs: Libs):
+    """A client's n-th per-parameter fetch is decided with the draws of its
+    n-th fetch (stream 1), whatever pushes it selected in between: two
+    servers in the same state, one of which selects three pushes between its
+    fetches, return the same fetch lists; and fetch and push lists of the
+    same count differ (separate streams)."""
+    rng = np.random.default_rng(83)
+    P = 4096
+    theta0 = (rng.standard_normal(P) * 0.01).astype(np.float32)
+    g = (rng.standard_normal(P) * 0.1).astype(np.float32)
+
+    def server():
+        s = _server(libs, "f32", P, FASGD, lam=3, c_push=1.0, seed=555)
+        s.set_params(theta0)
+        s.push(0, 0, g)
+        s.apply_pending(1)
+        s.set_fetch_threshold(1.0)
+        return s
+
+    a, b = server(), server()
+    fa = [a.fetch_compact(2) for _ in range(2)]
+    pushes = [b.select_compact(2, g) for _ in range(3)]
+    fb = [b.fetch_compact(2)]
+    b.select_compact(2, g)
+    fb.append(b.fetch_compact(2))
+    for (ia, va), (ib, vb) in zip(fa, fb):
+        assert np.array_equal(ia, ib) and np.array_equal(va, vb)
+    assert 0 < fa[0][0].size < P
+    assert not np.array_equal(fa[0][0], pushes[0][0])
+
+
+def check_tensor_streams_separate(libs: Libs):
+    """Per-tensor rule: a client's n-th budget fetch and its n-th budget push,
+    decided against the same statistics and budget, draw from separate
+    streams -- over 64 tensors their decisions differ."""
+    rng = np.random.default_rng(89)
+    sizes = rng.integers(1, 40, 64)
+    P = int(sizes.sum())
+    g = (rng.standard_normal(P) * 0.1).astype(np.float32)
+
+    def server():
+        s = _server(libs, "f32", P, FASGD, lam=2, seed=777, eps_b=1e-3)
+        s.set_tensors(sizes)
+        s.push(0, 0, g)
+        s.apply_pending(1)
+        return s
+
+    a, b = server(), server()
+    copy = np.zeros(P, np.float32)
+    sent_fetch, c_fetch, _ = a.fetch_budget(1, copy, P // 2)
+    b.push_budget(1, b.T, g, P // 2)
+    b.apply_pending(1)
+    sent_push, c_push, _ = b.budget_log[-1]
+    assert c_fetch == c_push                      # same statistics, same budget
+    assert 0 < int(sent_fetch.sum()) < sizes.size
+    assert not np.array_equal(sent_fetch, sent_push)
+
+
+ALL_CHECKS = [  # quick pins first: a mutant stops at the first pin it fails
     check_hand_trace,
     check_constant_gradient_closed_form,
     check_std_variant_closed_form,
@@ -994,11 +1100,14 @@ ALL_CHECKS = [
     check_sparse_leaves_unsent_untouched,
     check_fetch_path,
     check_server_fetch_counters,
-    check_message_path,
     check_sim_objective,
-    check_tensor_means,
     check_budget_threshold,
     check_tensor_decisions,
     check_budget_server,
+    check_batched_apply_order,
+    check_fetch_draws_keyed_by_fetch_count,
+    check_tensor_streams_separate,
     check_protocol_errors,
+    check_tensor_means,
+    check_message_path,
 ]

@@ -1,0 +1,102 @@
+"""Planted mistakes in the oracle's protocol layer are caught by the pins (no GPU).
+
+``test_oracle_mutants.py`` plants slips in the C source of the elementwise
+rules.  This file does the same for the Python layer of ``oracle/__init__.py``
+that turns them into the server of Sec. 2.1-2.3: the FIFO of pushes, the
+staleness tau = T - j a push finds, the per-client push and fetch counters
+that key the draws, the per-message gradient cache and the per-tensor
+decisions.  Each mutant is the module's source with one plausible slip,
+loaded as a separate module; the pins then run against it (``pins.oracle``
+is pointed at the mutant for the test) and at least one must fail.
+"""
+
+import types
+
+import pytest
+
+import oracle
+import pins
+
+PY_MUTANTS = {
+    # protocol order and staleness (Sec. 2.1)
+    "fifo_last_first": ("kind, client, j, payload = self.fifo.pop(0)",
+                        "kind, client, j, payload = self.fifo.pop()"),
+    "tau_off_by_one": ("tau = self.T - j", "tau = self.T - j + 1"),
+    "future_timestamp_accepted": ("if not 0 <= j <= self.T:", "if not 0 <= j <= self.T + 1:"),
+    # per-message rule (Sec. 2.3): counter, stream, cache, statistic
+    "message_push_counter_stuck": (
+        "                n = self.push_count[client]\n"
+        "                self.push_count[client] += 1\n"
+        "                u = draw_message(self.seed, 0, client, n)",
+        "                n = self.push_count[client]\n"
+        "                u = draw_message(self.seed, 0, client, n)"),
+    "message_push_fetch_stream": ("u = draw_message(self.seed, 0, client, n)",
+                                  "u = draw_message(self.seed, 1, client, n)"),
+    "message_drop_applies_new": ("                if sent:\n"
+                                 "                    self.cache[client] = payload.copy()",
+                                 "                self.cache[client] = payload.copy()"),
+    "message_cache_one_slot": ("self.cache[client] = payload.copy()",
+                               "self.cache[0] = payload.copy()"),
+    "message_mean_of_theta": ("                vbar = mean_v(self.v, self.real)\n"
+                              "                sent = decide(",
+                              "                vbar = mean_v(self.theta, self.real)\n"
+                              "                sent = decide("),
+    "fetch_message_counter_stuck": (
+        "        n = self.fetch_count[client]\n"
+        "        self.fetch_count[client] += 1\n"
+        "        u = draw_message(self.seed, 1, client, n)",
+        "        n = self.fetch_count[client]\n"
+        "        u = draw_message(self.seed, 1, client, n)"),
+    "fetch_message_always_copies": ("        if ok:\n            theta_client[:] = self.theta",
+                                    "        if True:\n            theta_client[:] = self.theta"),
+    # per-parameter rule: the counters that key the draws
+    "select_counter_stuck": ("        self.push_count[client] += 1\n        return out",
+                             "        return out"),
+    "fetch_compact_push_counter": ("self.seed, client, self.fetch_count[client],",
+                                   "self.seed, client, self.push_count[client],"),
+    # per-tensor rule under a budget
+    "budget_push_counter_stuck": (
+        "                n = self.push_count[client]\n"
+        "                self.push_count[client] += 1\n"
+        "                sent, cb, m = self._budget_decide(0, client, n, budget)",
+        "                n = self.push_count[client]\n"
+        "                sent, cb, m = self._budget_decide(0, client, n, budget)"),
+    "budget_fetch_push_stream": ("sent, c, m = self._budget_decide(1, client, n, budget)",
+                                 "sent, c, m = self._budget_decide(0, client, n, budget)"),
+    "budget_fetch_copies_all": ("for t in np.flatnonzero(sent):",
+                                "for t in range(sent.size):"),
+}
+
+
+def _load_mutant(name, old, new):
+    src = open(oracle.__file__).read()
+    assert src.count(old) == 1, f"mutant {name}: pattern not (uniquely) in the oracle module"
+    mod = types.ModuleType(f"oracle_protocol_mutant_{name}")
+    mod.__file__ = oracle.__file__
+    exec(compile(src.replace(old, new, 1), oracle.__file__, "exec"), mod.__dict__)
+    return mod
+
+
+@pytest.mark.parametrize("name", sorted(PY_MUTANTS))
+def test_protocol_mutant_is_caught(monkeypatch, name):
+    old, new = PY_MUTANTS[name]
+    mutant = _load_mutant(name, old, new)
+    monkeypatch.setattr(pins, "oracle", mutant)
+    libs = pins.real_libs()
+    caught = None
+    for check in pins.ALL_CHECKS:   # the first pin that fails catches the mutant
+        try:
+            check(libs)
+        except Exception as e:      # any failure of a pin counts as a catch
+            caught = f"{check.__name__}: {type(e).__name__}"
+            break
+    assert caught is not None, f"protocol mutant {name} passed every pin"
+
+
+def test_unmutated_module_passes_every_pin(monkeypatch):
+    """The harness itself: the module loaded the same way, unchanged, passes."""
+    monkeypatch.setattr(pins, "oracle", _load_mutant("none", "ASGD, SASGD, FASGD, FASGD_STD = 0, 1, 2, 3",
+                                                     "ASGD, SASGD, FASGD, FASGD_STD = 0, 1, 2, 3"))
+    libs = pins.real_libs()
+    for check in pins.ALL_CHECKS:
+        check(libs)
