@@ -733,6 +733,68 @@ def check_sim_objective(libs: Libs):
     assert np.array_equal(sim.srv.theta.view(np.uint32), ref.view(np.uint32))
 
 
+def check_sim_protocol(libs: Libs):
+    """The closed-loop simulation with several clients, restated plainly:
+    every client keeps a copy of the parameters and the server timestamp it
+    was taken at; a dispatcher batch of clients computes gradients at their
+    copies (noise drawn per client and gradient count), pushes them with
+    those timestamps, the server applies the batch in order (push k at
+    T + k: tau = T + k - j), and the clients of the batch then refresh.  A
+    full refresh, and the per-parameter, per-message and per-tensor refreshes
+    at the thresholds or budgets that fetch everything or nothing, reproduce
+    the restatement bit for bit under ASGD and SASGD.  (A per-parameter or
+    per-tensor refresh stamps the copy with T whatever it transmitted; a
+    per-message refresh only when it fetches.)"""
+    import oracle.sim as osim
+    rng = np.random.default_rng(97)
+    P, lam, seed = 37, 3, 11
+    obj = ((10 ** rng.uniform(-1, 0.5, P)).astype(np.float32),
+           (rng.standard_normal(P) * 0.1).astype(np.float32),
+           (10 ** rng.uniform(-3, -1, P)).astype(np.float32))
+    th0 = (rng.standard_normal(P) * 0.1).astype(np.float32)
+    schedule = [[0], [1], [0, 2], [1, 2, 0], [2], [0, 1], [1], [2, 0]]
+    a32 = np.float32(0.05)
+
+    def restated(variant, copy_refresh, stamp_refresh):
+        theta, T = th0.copy(), 0
+        copies = [th0.copy() for _ in range(lam)]
+        stamp, count = [0] * lam, [0] * lam
+        for batch in schedule:
+            pushes = []
+            for c in batch:
+                pushes.append((stamp[c], oracle.sim_grad(copies[c], *obj, seed, c, count[c],
+                                                         lib=libs.f32)))
+                count[c] += 1
+            for k, (j, g) in enumerate(pushes):
+                tau = T + k - j
+                coef = a32 if variant == ASGD else np.float32(float(a32) / max(tau, 1))
+                theta = (theta - coef * g).astype(np.float32)
+            T += len(batch)
+            for c in batch:
+                if copy_refresh:
+                    copies[c] = theta.copy()
+                if stamp_refresh:
+                    stamp[c] = T
+        return theta
+
+    inf = float("inf")
+    cases = [("full", {}, True, True),
+             ("param", {"c_fetch": 0.0}, True, True), ("param", {"c_fetch": inf}, False, True),
+             ("message", {"c_fetch": 0.0}, True, True), ("message", {"c_fetch": inf}, False, False),
+             ("budget", {"fetch_budget": P, "tensor_sizes": [10, 27]}, True, True),
+             ("budget", {"fetch_budget": 0, "tensor_sizes": [10, 27]}, False, True)]
+    for variant in (ASGD, SASGD):
+        for fetch, kw, copy_refresh, stamp_refresh in cases:
+            sim = osim.OracleSimulation(P, lam, float(a32), variant, objective=obj, theta0=th0,
+                                        seed=seed, fetch=fetch, lib=libs.f32, **kw)
+            sim.run(schedule)
+            want = restated(variant, copy_refresh, stamp_refresh)
+            assert np.array_equal(sim.srv.theta.view(np.uint32), want.view(np.uint32)), (
+                variant, fetch, kw)
+    # the restatement itself sees the staleness: SASGD differs from ASGD here
+    assert not np.array_equal(restated(ASGD, True, True), restated(SASGD, True, True))
+
+
 def check_protocol_errors(libs: Libs):
     s = _server(libs, "f32", 4, FASGD, lam=2)
     g = np.zeros(4, np.float32)
@@ -1107,6 +1169,7 @@ ALL_CHECKS = [  # quick pins first: a mutant stops at the first pin it fails
     check_batched_apply_order,
     check_fetch_draws_keyed_by_fetch_count,
     check_tensor_streams_separate,
+    check_sim_protocol,
     check_protocol_errors,
     check_tensor_means,
     check_message_path,

@@ -100,3 +100,52 @@ def test_unmutated_module_passes_every_pin(monkeypatch):
     libs = pins.real_libs()
     for check in pins.ALL_CHECKS:
         check(libs)
+
+
+# The closed-loop simulation's oracle (oracle/sim.py): dispatcher batches,
+# clients' stale copies and the timestamps they push with, the refreshes.
+SIM_MUTANTS = {
+    "sim_copy_timestamp_kept": ("                self.clients[c][:] = self.srv.theta.astype(np.float32)\n"
+                                "                self.client_T[c] = T\n",
+                                "                self.clients[c][:] = self.srv.theta.astype(np.float32)\n"),
+    "sim_pushes_timestamp_zero": ("self.srv.push(c, self.client_T[c], g)", "self.srv.push(c, 0, g)"),
+    "sim_grad_count_stuck": ("            self.grad_count[c] += 1\n", ""),
+    "sim_grad_one_stream": ("g = sim_grad(self.clients[c], self.h, self.star, self.sigma, self.seed, c,",
+                            "g = sim_grad(self.clients[c], self.h, self.star, self.sigma, self.seed, 0,"),
+    "sim_param_fetch_dropped": ("                fetch_apply(self.clients[c], idx, val, lib=self.lib)\n", ""),
+    "sim_message_timestamp_always": ("                if self.srv.fetch_message(c, self.clients[c]):\n"
+                                     "                    self.client_T[c] = T",
+                                     "                self.srv.fetch_message(c, self.clients[c])\n"
+                                     "                self.client_T[c] = T"),
+    "sim_budget_fetch_wrong_copy": ("self.srv.fetch_budget(c, self.clients[c], self.fetch_budget)",
+                                    "self.srv.fetch_budget(c, self.clients[0], self.fetch_budget)"),
+}
+
+
+def _load_sim_mutant(name, old, new):
+    import oracle.sim as osim
+    src = open(osim.__file__).read()
+    assert src.count(old) == 1, f"mutant {name}: pattern not (uniquely) in oracle/sim.py"
+    mod = types.ModuleType(f"oracle_sim_mutant_{name}")
+    mod.__file__ = osim.__file__
+    mod.__package__ = "oracle"
+    exec(compile(src.replace(old, new, 1), osim.__file__, "exec"), mod.__dict__)
+    return mod
+
+
+@pytest.mark.parametrize("name", sorted(SIM_MUTANTS))
+def test_sim_mutant_is_caught(monkeypatch, name):
+    import sys
+    old, new = SIM_MUTANTS[name]
+    mutant = _load_sim_mutant(name, old, new)
+    monkeypatch.setitem(sys.modules, "oracle.sim", mutant)
+    monkeypatch.setattr(oracle, "sim", mutant, raising=False)
+    libs = pins.real_libs()
+    caught = None
+    for check in pins.ALL_CHECKS:
+        try:
+            check(libs)
+        except Exception as e:
+            caught = f"{check.__name__}: {type(e).__name__}"
+            break
+    assert caught is not None, f"simulation mutant {name} passed every pin"
