@@ -208,7 +208,8 @@ def _sizes(sizes) -> np.ndarray:
 
 
 def tensor_means(v: np.ndarray, sizes, real: str = "f32", lib=None) -> np.ndarray:
-    """vbar_t: mean of v over each contiguous tensor (fp64 sum, rounded to fp32)."""
+    """vbar_t: mean of v over each contiguous tensor (the exact sum divided by
+    the tensor's size, rounded once to fp32)."""
     s = _sizes(sizes)
     vv = np.ascontiguousarray(v, dtype=_dtype(real))
     assert vv.shape[0] == int(s.sum())

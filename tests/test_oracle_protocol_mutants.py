@@ -65,6 +65,20 @@ PY_MUTANTS = {
                                  "sent, c, m = self._budget_decide(0, client, n, budget)"),
     "budget_fetch_copies_all": ("for t in np.flatnonzero(sent):",
                                 "for t in range(sent.size):"),
+    # the wrappers around the C rules: argument order, streams, counts
+    "select_swaps_grad_and_v": ("ora_select(P, _ptr(g), _ptr(v), c,", "ora_select(P, _ptr(v), _ptr(g), c,"),
+    "fetch_select_swaps_theta_and_v": ("ora_fetch_select(P, _ptr(th), _ptr(v), c,",
+                                       "ora_fetch_select(P, _ptr(v), _ptr(th), c,"),
+    "fetch_apply_applies_nothing": ("ora_fetch_apply(_ptr(theta_client), i.shape[0], _ptr(i), _ptr(x))",
+                                    "ora_fetch_apply(_ptr(theta_client), 0, _ptr(i), _ptr(x))"),
+    "draw_message_one_stream": ("ora_draw_message(seed, stream, client, n)",
+                                "ora_draw_message(seed, 0, client, n)"),
+    "tensor_select_one_stream": ("                                                stream, client, n, _ptr(sent))",
+                                 "                                                0, client, n, _ptr(sent))"),
+    "budget_c_half_budget": ("_ptr(vb), eps_b,\n                                                     int(budget)))",
+                             "_ptr(vb), eps_b,\n                                                     int(budget) // 2))"),
+    "sim_grad_one_client": ("seed, client,\n                                       n, _ptr(g))",
+                            "seed, 0,\n                                       n, _ptr(g))"),
 }
 
 
