@@ -498,9 +498,11 @@ def run_bfasgd(args, w, world, rank, local):
     clocks.start()
     time.sleep(0.3)
     start.record(stream)
+    h0 = time.perf_counter()
     for i in range(args.steps):     # no events inside: they would split the launch chains
         step(t, None, i)
         t += 1
+    host_us = (time.perf_counter() - h0) * 1e6 / args.steps   # above ms_per_step: host-bound
     end.record(stream)
     torch.cuda.synchronize()
     clock_info = clocks.stop()
@@ -539,6 +541,7 @@ def run_bfasgd(args, w, world, rank, local):
                      "apply_gbs": round(alg_apply / (app_ms / 1e3) / 1e9, 1),
                      "fetch_select_ms": round(fsel_ms, 5), "fetch_apply_ms": round(fapp_ms, 5)},
         "clocks": clock_info, "e2e": None, "gpu_launches": launches,
+        "host_us_per_step": round(host_us, 3),
         "pushes_per_s": world / step_s, "sent_fraction": round(frac, 4),
         "fetched_fraction": round(float(fetched.mean() / P), 4),
         "sent_updates_per_s": sent.mean() * world / step_s,
@@ -616,9 +619,11 @@ def run_message(args, w, world, rank, local):
     clocks.start()
     time.sleep(0.3)
     start.record(stream)
+    h0 = time.perf_counter()
     for i in range(args.steps):     # no events inside: they would split the launch chains
         step(t, None, i)
         t += 1
+    host_us = (time.perf_counter() - h0) * 1e6 / args.steps   # above ms_per_step: host-bound
     end.record(stream)
     torch.cuda.synchronize()
     clock_info = clocks.stop()
@@ -654,6 +659,7 @@ def run_message(args, w, world, rank, local):
                      "bytes_per_launch": push_bytes, "launch_ms": round(push_ms, 5),
                      "traffic": None, "fetch_ms": round(fetch_ms, 5)},
         "clocks": clock_info, "e2e": None, "gpu_launches": launches,
+        "host_us_per_step": round(host_us, 3),
         "pushes_per_s": world / step_s, "sent_fraction": round(s_frac, 4),
         "fetched_fraction": round(f_frac, 4),
         "config": {"workload": w.name, "P_per_gpu": P, "P_total": P * world, "lambda": w.lam,
@@ -731,9 +737,11 @@ def run_tensor(args, w, world, rank, local):
     clocks.start()
     time.sleep(0.3)
     start.record(stream)
+    h0 = time.perf_counter()
     for i in range(args.steps):     # no events inside: they would split the launch chains
         step(t, None, i)
         t += 1
+    host_us = (time.perf_counter() - h0) * 1e6 / args.steps   # above ms_per_step: host-bound
     end.record(stream)
     torch.cuda.synchronize()
     clock_info = clocks.stop()
@@ -772,6 +780,7 @@ def run_tensor(args, w, world, rank, local):
                      "traffic": None, "fetch_ms": round(fetch_ms, 5),
                      "fetch_gbs": round(fetch_bytes / (fetch_ms / 1e3) / 1e9, 1)},
         "clocks": clock_info, "e2e": None, "gpu_launches": launches,
+        "host_us_per_step": round(host_us, 3),
         "pushes_per_s": world / step_s, "sent_fraction": round(s_mean / P, 4),
         "fetched_fraction": round(f_mean / P, 4),
         "sent_updates_per_s": s_mean * world / step_s,
